@@ -1,0 +1,177 @@
+/*
+ * cm.h -- C ABI of libcm, MDS-coded matrix multiplication on one GB300 GPU.
+ *
+ * Method: Lee, Lam, Pedarsani, Papailiopoulos, Ramchandran, "Speeding Up
+ * Distributed Machine Learning Using Codes", Sec. III.  A data matrix A
+ * (m x d) is split by rows into k blocks A_0..A_{k-1} of L = ceil(m/k) rows
+ * (zero rows appended, Sec. III-A footnote); a systematic (n,k) code with
+ * generator G = [I_k; P] turns them into n coded blocks
+ * A~_j = sum_i G[j][i] A_i (Sec. III-A).  The n block products A~_j X are the
+ * n simulated workers; from ANY k of the n results the product A X is
+ * recovered (Example "MDS codes", Sec. III-B).  Straggler sets follow the
+ * shifted-exponential runtime model (Sec. III-C, III-D).  The same machinery
+ * runs coded gradient descent for linear regression (Sec. III-E).
+ *
+ * Conventions for every call:
+ *  - Matrices are row-major.  "Stacked" results hold worker j's block in rows
+ *    [j L, (j+1) L).  Worker j < k is systematic: its coded block is A_j
+ *    itself, read in place from the caller's A (rows >= m are virtual zero
+ *    rows, never read); workers j >= k are parity blocks held in a separate
+ *    (n-k) L x d "parity" buffer.
+ *  - Device pointers are CUDA device memory (or managed memory) of the
+ *    current device.  The caller allocates and frees every device buffer; the
+ *    library allocates no device memory and keeps no global state, so calls
+ *    on distinct objects are thread-safe.  A cm_code is a small immutable
+ *    host object.
+ *  - Every GPU call is asynchronous on the given stream (NULL = legacy
+ *    default stream).  Argument errors are returned synchronously and nothing
+ *    is launched.  CM_ECUDA is returned when a launch fails.  Conditions only
+ *    the device can see (a singular system, a bounded wait that gave up) are
+ *    written to the optional int32 device word *dev_status after the stream
+ *    reaches the kernel; the library only ever writes error codes there
+ *    (never CM_OK), so the caller clears it beforehand.
+ *  - Alignment: A, parity and (for cm_matmat) B start on 16-byte boundaries
+ *    and their leading dimensions are multiples of 16 bytes (4 fp32 or 8 bf16
+ *    elements); X, Y and Yt have no alignment requirement beyond their type.
+ *  - No call traps, aborts or exits the process.
+ */
+#ifndef CM_H
+#define CM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    CM_OK = 0,
+    CM_EINVAL = -1,          /* bad argument, shape, alignment or dtype */
+    CM_ENOTDECODABLE = -2,   /* fewer than k survivors */
+    CM_ESINGULAR = -3,       /* G_S is singular (device-detected) */
+    CM_ECUDA = -4,           /* a CUDA launch or query failed */
+    CM_ENOMEM = -5,          /* host allocation failed, or workspace too small */
+    CM_ETIMEOUT = -6,        /* a bounded device wait gave up */
+    CM_EUNSUPPORTED = -7     /* valid request this build does not handle */
+} cm_status;
+
+typedef enum { CM_F32 = 0, CM_BF16 = 1 } cm_dtype;
+
+typedef struct cm_code cm_code;          /* opaque, immutable after create */
+typedef struct CUstream_st *cm_stream_t; /* same type as cudaStream_t */
+
+/* Build an (n,k) systematic code for an m x d data matrix of type dt
+ * (Sec. III-A).  parity_host is the (n-k) x k block P of G = [I_k; P], fp32,
+ * row-major, on the host; it is copied.  Any P whose square submatrices are
+ * all nonsingular gives an MDS code; a Gaussian P does with probability 1.
+ * Requires 1 <= k < n <= 32, m >= 1, d >= 1, finite P.  No CUDA call. */
+cm_status cm_code_create(int32_t n, int32_t k, int64_t m, int64_t d, cm_dtype dt,
+                         const float *parity_host, cm_code **out);
+void cm_code_destroy(cm_code *code);
+
+/* L = ceil(m / k), the rows per block after zero padding (Sec. III-A
+ * footnote); -1 for a NULL code. */
+int64_t cm_block_rows(const cm_code *code);
+
+/* Encoding (Sec. III-A): parity block p (rows [p L, (p+1) L) of parity_out,
+ * leading dimension ldp) = sum_i P[p][i] A_i, for p = 0..n-k-1, in one pass
+ * over A.  A is m x d with leading dimension lda, of the code's dtype (fp32,
+ * or bf16 with fp32 accumulation and round-to-nearest-even output).
+ * parity_out must not overlap A. */
+cm_status cm_encode(const cm_code *code, const void *A, int64_t lda,
+                    void *parity_out, int64_t ldp, cm_stream_t stream);
+
+/* The n worker products (Sec. III-A protocol): Yt[j L + r][v] =
+ * sum_c A~_j[r][c] X[c][v] for every worker j, row r < L and vector v < b,
+ * all workers concurrently.  fp32 code only.  X is d x b fp32 (row-major,
+ * vectors contiguous per row), 1 <= b <= 8.  Yt is n L x b fp64: each sum is
+ * formed from short fp32 partial sums combined in fp64, so decoding does not
+ * amplify an fp32 rounding of the results. */
+cm_status cm_matvec(const cm_code *code, const float *A, int64_t lda,
+                    const float *parity, int64_t ldp, const float *X, int32_t b,
+                    double *Yt, cm_stream_t stream);
+
+/* Straggler draw (Sec. III-C, III-D; eq. for the MDS runtime).  Host only.
+ * Worker j's time in round `counter` is T_j = (shift + E_j / rate) / k with
+ * E_j = -log(1 - U_j), U_j = (z_j >> 11) 2^-53, z_j the SplitMix64 output
+ * (Steele, Lea, Flood 2014) of the Weyl state
+ * seed + (counter n + j + 1) 0x9E3779B97F4A7C15.  The coded run ends at the
+ * k-th arrival, so the survivors are the k workers with the smallest T_j,
+ * ranked on the integers (z_j >> 11, j) (ties go to the lower index).
+ * *survivors receives the bitmask (bit j = worker j survives), exactly k
+ * bits; times (nullable, n entries) receives the T_j.  1 <= k <= n <= 32,
+ * rate > 0. */
+cm_status cm_draw_erasures(uint64_t seed, uint64_t counter, int32_t n, int32_t k,
+                           double shift, double rate, uint32_t *survivors,
+                           double *times);
+
+/* Decoding (Sec. III-A last paragraph; Example "MDS codes").  S = the first
+ * k set bits of `survivors` (ascending; extra survivors are ignored, which
+ * favours the systematic workers).  The surviving results satisfy
+ * Yt_S = G_S Z with Z the uncoded block products; the kernel inverts G_S in
+ * fp64 (the k-e unit rows of surviving systematic workers are eliminated
+ * first, then Gauss-Jordan with partial pivoting on the e x e block of the
+ * missing systematic columns), forms the rows of G_S^-1 for the e missing
+ * systematic blocks and applies them to the k surviving results in fp64;
+ * surviving systematic blocks pass through.  Y (m x b fp32) is the
+ * concatenation of the k decoded blocks without the appended zero rows.
+ * Returns CM_ENOTDECODABLE when fewer than k bits are set; a singular G_S
+ * writes CM_ESINGULAR to *dev_status (nullable) and leaves Y unwritten. */
+cm_status cm_decode(const cm_code *code, const double *Yt, uint32_t survivors,
+                    int32_t b, float *Y, int32_t *dev_status, cm_stream_t stream);
+
+/* Workspace bytes cm_gd_step needs for this pair of codes (0 on bad codes). */
+size_t cm_gd_workspace_bytes(const cm_code *code_A, const cm_code *code_AT);
+
+/* One iteration of coded gradient descent for linear regression (Sec. III-E):
+ * x <- x - eta A^T (A x - y).  The first product uses code_A (m x d) on A and
+ * its parity PA with survivors surv_A; the result decodes to z = A x - y.
+ * The second uses code_AT (d x m) on AT = A^T (row-major d x m, i.e. the
+ * column split of A, Sec. III-E) and its parity PAT with survivors surv_AT;
+ * the result decodes to the gradient g = A^T z and x -= eta g.  x (d fp32) is
+ * updated in place.  ws is caller device memory of at least
+ * cm_gd_workspace_bytes(code_A, code_AT) bytes (holds both stacked results
+ * and z), 256-byte aligned.  Four launches on `stream`. */
+cm_status cm_gd_step(const cm_code *code_A, const float *A, int64_t lda,
+                     const float *PA, int64_t ldpa,
+                     const cm_code *code_AT, const float *AT, int64_t ldat,
+                     const float *PAT, int64_t ldpat,
+                     const float *y, float *x, float eta,
+                     uint32_t surv_A, uint32_t surv_AT,
+                     void *ws, size_t ws_bytes, int32_t *dev_status,
+                     cm_stream_t stream);
+
+/* Coded matrix-matrix products (the s-column X of the Sec. I-A example) on
+ * tensor cores: Ct[j L + r][c] = sum_t A~_j[r][t] B[t][c] for all n workers,
+ * bf16 inputs, fp32 accumulation, fp32 output.  bf16 code only.  B is passed
+ * transposed: Bt is N x d bf16 (row-major, leading dimension ldb), i.e. each
+ * column of B contiguous.  Ct is n L x N fp32 with leading dimension ldc.
+ * Requires d % 8 == 0 and N % 16 == 0 (the tile grid of the tensor-core
+ * path), N >= 16. */
+cm_status cm_coded_gemm(const cm_code *code, const void *A, int64_t lda,
+                        const void *parity, int64_t ldp, const void *Bt, int64_t ldb,
+                        int32_t N, float *Ct, int64_t ldc, cm_stream_t stream);
+
+/* Decoding of matrix results: as cm_decode with b = N columns of fp32
+ * stacked results Ct (leading dimension ldc) into C (m x N fp32, leading
+ * dimension ldcc).  The decode coefficients are formed in fp64 and applied
+ * in fp32.  C may alias Ct (C == Ct, ldcc == ldc): surviving systematic
+ * blocks are then already in place and only the missing ones are written. */
+cm_status cm_decode_mat(const cm_code *code, const float *Ct, int64_t ldc,
+                        uint32_t survivors, int32_t N, float *C, int64_t ldcc,
+                        int32_t *dev_status, cm_stream_t stream);
+
+/* cm_coded_gemm followed by cm_decode_mat on the same stream. */
+cm_status cm_matmat(const cm_code *code, const void *A, int64_t lda,
+                    const void *parity, int64_t ldp, const void *Bt, int64_t ldb,
+                    int32_t N, float *Ct, int64_t ldc, uint32_t survivors,
+                    float *C, int64_t ldcc, int32_t *dev_status, cm_stream_t stream);
+
+/* Static description of a status code. */
+const char *cm_status_string(cm_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CM_H */

@@ -1,0 +1,291 @@
+"""Python binding of libcm (MDS-coded matrix multiplication on one GB300).
+
+Thin ctypes marshalling over the C ABI declared in ``include/cm.h``: every
+function here checks tensor dtypes, devices and shapes, passes raw pointers
+and the current torch CUDA stream, and maps status codes to exceptions.  All
+computation runs in the library's CUDA kernels; there is no fallback, and
+importing a function whose library was not built raises ``LibraryMissing``.
+
+Method: Lee et al., "Speeding Up Distributed Machine Learning Using Codes",
+Sec. III (see ``include/cm.h`` for the definitions of each call).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libcm.so")
+
+CM_OK, CM_EINVAL, CM_ENOTDECODABLE, CM_ESINGULAR = 0, -1, -2, -3
+CM_ECUDA, CM_ENOMEM, CM_ETIMEOUT, CM_EUNSUPPORTED = -4, -5, -6, -7
+CM_F32, CM_BF16 = 0, 1
+
+
+class LibraryMissing(RuntimeError):
+    pass
+
+
+class CodedError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__("%s: %s (status %d)" % (what, status_string(status), status))
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libcm (raises LibraryMissing if it was not built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise LibraryMissing("libcm.so is not built: run "
+                                 "`python -m paper_1512_02673_gb300.build`")
+        L = ctypes.CDLL(LIB_PATH)
+        i32, i64, u32, u64, f32, f64 = (ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32,
+                                        ctypes.c_uint64, ctypes.c_float, ctypes.c_double)
+        vp, sz = ctypes.c_void_p, ctypes.c_size_t
+        st = ctypes.c_int
+        sig = {
+            "cm_code_create": (st, [i32, i32, i64, i64, st, vp, ctypes.POINTER(vp)]),
+            "cm_code_destroy": (None, [vp]),
+            "cm_block_rows": (i64, [vp]),
+            "cm_encode": (st, [vp, vp, i64, vp, i64, vp]),
+            "cm_matvec": (st, [vp, vp, i64, vp, i64, vp, i32, vp, vp]),
+            "cm_draw_erasures": (st, [u64, u64, i32, i32, f64, f64, ctypes.POINTER(u32), vp]),
+            "cm_decode": (st, [vp, vp, u32, i32, vp, vp, vp]),
+            "cm_gd_workspace_bytes": (sz, [vp, vp]),
+            "cm_gd_step": (st, [vp, vp, i64, vp, i64, vp, vp, i64, vp, i64, vp, vp, f32,
+                                u32, u32, vp, sz, vp, vp]),
+            "cm_coded_gemm": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, vp]),
+            "cm_decode_mat": (st, [vp, vp, i64, u32, i32, vp, i64, vp, vp]),
+            "cm_matmat": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, u32, vp, i64,
+                               vp, vp]),
+            "cm_status_string": (ctypes.c_char_p, [st]),
+        }
+        for name, (res, args) in sig.items():
+            f = getattr(L, name)
+            f.restype = res
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def status_string(status: int) -> str:
+    return lib().cm_status_string(status).decode()
+
+
+def _check(status: int, what: str):
+    if status != CM_OK:
+        raise CodedError(status, what)
+
+
+def _stream():
+    return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+
+
+def _dev(t: torch.Tensor, dtype, name: str, ndim=None) -> int:
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError("%s must be a CUDA tensor" % name)
+    if t.dtype != dtype:
+        raise TypeError("%s must be %s, got %s" % (name, dtype, t.dtype))
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError("%s must have %d dimensions" % (name, ndim))
+    return t.data_ptr()
+
+
+def _ld(t: torch.Tensor, name: str) -> int:
+    """Leading dimension of a row-major matrix view (unit column stride)."""
+    if t.dim() != 2 or (t.shape[1] > 1 and t.stride(1) != 1):
+        raise ValueError("%s must be a row-major matrix" % name)
+    return t.stride(0)
+
+
+def _contig(t: torch.Tensor, name: str):
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+
+
+class Code:
+    """An (n,k) systematic code G = [I_k; P] for an m x d data matrix."""
+
+    def __init__(self, n: int, k: int, m: int, d: int, parity, dtype: str = "f32"):
+        P = np.ascontiguousarray(np.asarray(parity, dtype=np.float32))
+        if P.shape != (n - k, k):
+            raise ValueError("parity must be (n-k) x k")
+        dt = {"f32": CM_F32, "bf16": CM_BF16}[dtype]
+        out = ctypes.c_void_p()
+        _check(lib().cm_code_create(n, k, m, d, dt, P.ctypes.data_as(ctypes.c_void_p),
+                                    ctypes.byref(out)), "cm_code_create")
+        self._h = out
+        self.n, self.k, self.m, self.d, self.dtype = n, k, m, d, dtype
+        self.P = P
+        self.L = int(lib().cm_block_rows(out))
+
+    @property
+    def handle(self):
+        return self._h
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h and _lib is not None:
+            _lib.cm_code_destroy(h)
+            self._h = None
+
+    @property
+    def torch_dtype(self):
+        return torch.float32 if self.dtype == "f32" else torch.bfloat16
+
+
+def encode(code: Code, A: torch.Tensor, parity: torch.Tensor | None = None) -> torch.Tensor:
+    """Parity blocks ((n-k) L x d, code dtype) of A (m x d)."""
+    dt = code.torch_dtype
+    _dev(A, dt, "A", 2)
+    if tuple(A.shape) != (code.m, code.d):
+        raise ValueError("A must be m x d")
+    if parity is None:
+        parity = torch.empty(((code.n - code.k) * code.L, code.d), dtype=dt, device=A.device)
+    _dev(parity, dt, "parity", 2)
+    if tuple(parity.shape) != ((code.n - code.k) * code.L, code.d):
+        raise ValueError("parity must be (n-k) L x d")
+    _check(lib().cm_encode(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
+                           _ld(parity, "parity"), _stream()), "cm_encode")
+    return parity
+
+
+def matvec(code: Code, A: torch.Tensor, parity: torch.Tensor, X: torch.Tensor,
+           Yt: torch.Tensor | None = None) -> torch.Tensor:
+    """All n worker products Yt (n L x b, fp64) for X (d x b fp32, b <= 8)."""
+    _dev(A, torch.float32, "A", 2)
+    _dev(parity, torch.float32, "parity", 2)
+    if X.dim() == 1:
+        X = X.view(-1, 1)
+    _dev(X, torch.float32, "X", 2)
+    _contig(X, "X")
+    if X.shape[0] != code.d:
+        raise ValueError("X must have d rows")
+    b = X.shape[1]
+    if Yt is None:
+        Yt = torch.empty((code.n * code.L, b), dtype=torch.float64, device=X.device)
+    _dev(Yt, torch.float64, "Yt", 2)
+    _contig(Yt, "Yt")
+    if tuple(Yt.shape) != (code.n * code.L, b):
+        raise ValueError("Yt must be n L x b")
+    _check(lib().cm_matvec(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
+                           _ld(parity, "parity"), X.data_ptr(), b, Yt.data_ptr(), _stream()),
+           "cm_matvec")
+    return Yt
+
+
+def draw_erasures(seed: int, counter: int, n: int, k: int, shift: float = 1.0,
+                  rate: float = 1.0):
+    """(survivor bitmask, n task times) of one shifted-exponential straggler draw."""
+    mask = ctypes.c_uint32(0)
+    times = np.empty(n, np.float64)
+    _check(lib().cm_draw_erasures(seed, counter, n, k, shift, rate, ctypes.byref(mask),
+                                  times.ctypes.data_as(ctypes.c_void_p)), "cm_draw_erasures")
+    return int(mask.value), times
+
+
+def decode(code: Code, Yt: torch.Tensor, survivors: int, Y: torch.Tensor | None = None,
+           status: torch.Tensor | None = None) -> torch.Tensor:
+    """Y = A X (m x b fp32) decoded from the surviving rows of Yt."""
+    _dev(Yt, torch.float64, "Yt", 2)
+    _contig(Yt, "Yt")
+    b = Yt.shape[1]
+    if Y is None:
+        Y = torch.empty((code.m, b), dtype=torch.float32, device=Yt.device)
+    _dev(Y, torch.float32, "Y", 2)
+    _contig(Y, "Y")
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
+    _check(lib().cm_decode(code.handle, Yt.data_ptr(), survivors, b, Y.data_ptr(), sp,
+                           _stream()), "cm_decode")
+    return Y
+
+
+def gd_workspace_bytes(code_A: Code, code_AT: Code) -> int:
+    return int(lib().cm_gd_workspace_bytes(code_A.handle, code_AT.handle))
+
+
+def gd_step(code_A: Code, A, PA, code_AT: Code, AT, PAT, y, x, eta: float, surv_A: int,
+            surv_AT: int, ws: torch.Tensor, status: torch.Tensor | None = None):
+    """One coded gradient step x <- x - eta A^T (A x - y), x updated in place."""
+    for t, name in ((A, "A"), (PA, "PA"), (AT, "AT"), (PAT, "PAT")):
+        _dev(t, torch.float32, name, 2)
+    _dev(y, torch.float32, "y")
+    _dev(x, torch.float32, "x")
+    _contig(x, "x")
+    _contig(y, "y")
+    _dev(ws, torch.uint8, "ws")
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
+    _check(lib().cm_gd_step(code_A.handle, A.data_ptr(), _ld(A, "A"), PA.data_ptr(),
+                            _ld(PA, "PA"), code_AT.handle, AT.data_ptr(), _ld(AT, "AT"),
+                            PAT.data_ptr(), _ld(PAT, "PAT"), y.data_ptr(), x.data_ptr(),
+                            eta, surv_A, surv_AT, ws.data_ptr(), ws.numel(), sp, _stream()),
+           "cm_gd_step")
+    return x
+
+
+def coded_gemm(code: Code, A, parity, Bt, Ct=None) -> torch.Tensor:
+    """All n worker products Ct = A~ B (n L x N fp32) on tensor cores.
+
+    Bt is B transposed: N x d bf16 (each column of B contiguous)."""
+    for t, name in ((A, "A"), (parity, "parity"), (Bt, "Bt")):
+        _dev(t, torch.bfloat16, name, 2)
+    N = Bt.shape[0]
+    if Ct is None:
+        Ct = torch.empty((code.n * code.L, N), dtype=torch.float32, device=A.device)
+    _dev(Ct, torch.float32, "Ct", 2)
+    _check(lib().cm_coded_gemm(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
+                               _ld(parity, "parity"), Bt.data_ptr(), _ld(Bt, "Bt"), N,
+                               Ct.data_ptr(), _ld(Ct, "Ct"), _stream()), "cm_coded_gemm")
+    return Ct
+
+
+def decode_mat(code: Code, Ct: torch.Tensor, survivors: int, C: torch.Tensor | None = None,
+               status: torch.Tensor | None = None) -> torch.Tensor:
+    """C = A B (m x N fp32) decoded from the surviving blocks of Ct (may alias Ct)."""
+    _dev(Ct, torch.float32, "Ct", 2)
+    N = Ct.shape[1]
+    if C is None:
+        C = torch.empty((code.m, N), dtype=torch.float32, device=Ct.device)
+    _dev(C, torch.float32, "C", 2)
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
+    _check(lib().cm_decode_mat(code.handle, Ct.data_ptr(), _ld(Ct, "Ct"), survivors, N,
+                               C.data_ptr(), _ld(C, "C"), sp, _stream()), "cm_decode_mat")
+    return C
+
+
+def matmat(code: Code, A, parity, Bt, survivors: int, Ct=None, C=None, status=None):
+    """(Ct, C): coded GEMM of all n workers, then decode from the survivors."""
+    for t, name in ((A, "A"), (parity, "parity"), (Bt, "Bt")):
+        _dev(t, torch.bfloat16, name, 2)
+    N = Bt.shape[0]
+    if Ct is None:
+        Ct = torch.empty((code.n * code.L, N), dtype=torch.float32, device=A.device)
+    if C is None:
+        C = torch.empty((code.m, N), dtype=torch.float32, device=A.device)
+    _dev(Ct, torch.float32, "Ct", 2)
+    _dev(C, torch.float32, "C", 2)
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
+    _check(lib().cm_matmat(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
+                           _ld(parity, "parity"), Bt.data_ptr(), _ld(Bt, "Bt"), N,
+                           Ct.data_ptr(), _ld(Ct, "Ct"), survivors, C.data_ptr(),
+                           _ld(C, "C"), sp, _stream()), "cm_matmat")
+    return Ct, C

@@ -1,0 +1,228 @@
+// C ABI of libcm: argument validation and dispatch to the kernels.
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+
+#include "cm_internal.cuh"
+
+namespace {
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+int popcount32(uint32_t x)
+{
+    int c = 0;
+    for (; x; x &= x - 1) ++c;
+    return c;
+}
+
+cm_status from_cuda(cudaError_t e) { return e == cudaSuccess ? CM_OK : CM_ECUDA; }
+
+// Survivor mask checks shared by the decoders: no bit at or above n, and at
+// least k survivors (Example "MDS codes": any k results are decodable).
+cm_status check_survivors(const cm_code *c, uint32_t survivors)
+{
+    if (c->n < 32 && (survivors >> c->n)) return CM_EINVAL;
+    if (popcount32(survivors) < c->k) return CM_ENOTDECODABLE;
+    return CM_OK;
+}
+
+// Operand layout checks: base 16-byte aligned, leading dimension >= d and a
+// multiple of 16 bytes.
+bool layout_ok(const void *p, int64_t ld, int64_t d, int64_t elem)
+{
+    return p && aligned16(p) && ld >= d && (ld * elem) % 16 == 0;
+}
+
+}  // namespace
+
+int cm_sm_count()
+{
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 0;
+    if (dev < 64 && cache[dev]) return cache[dev];
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return 0;
+    if (dev < 64) cache[dev] = sms;
+    return sms;
+}
+
+extern "C" {
+
+cm_status cm_code_create(int32_t n, int32_t k, int64_t m, int64_t d, cm_dtype dt,
+                         const float *parity_host, cm_code **out)
+{
+    if (!out) return CM_EINVAL;
+    *out = nullptr;
+    if (k < 1 || n <= k || n > CM_MAX_N || m < 1 || d < 1 || !parity_host) return CM_EINVAL;
+    if (dt != CM_F32 && dt != CM_BF16) return CM_EINVAL;
+    if ((int64_t)(n - k) * k > CM_MAX_P) return CM_EINVAL;
+    for (int i = 0; i < (n - k) * k; ++i)
+        if (!std::isfinite(parity_host[i])) return CM_EINVAL;
+    cm_code *c = (cm_code *)std::calloc(1, sizeof(cm_code));
+    if (!c) return CM_ENOMEM;
+    c->n = n;
+    c->k = k;
+    c->m = m;
+    c->d = d;
+    c->L = (m + k - 1) / k;   // zero rows appended up to k L (Sec. III-A footnote)
+    c->dt = dt;
+    std::memcpy(c->P, parity_host, sizeof(float) * (n - k) * k);
+    *out = c;
+    return CM_OK;
+}
+
+void cm_code_destroy(cm_code *code) { std::free(code); }
+
+int64_t cm_block_rows(const cm_code *code) { return code ? code->L : -1; }
+
+cm_status cm_encode(const cm_code *c, const void *A, int64_t lda, void *par, int64_t ldp,
+                    cm_stream_t stream)
+{
+    if (!c) return CM_EINVAL;
+    int64_t es = c->dt == CM_F32 ? 4 : 2;
+    if (!layout_ok(A, lda, c->d, es) || !layout_ok(par, ldp, c->d, es)) return CM_EINVAL;
+    CodeParams cp = code_params(c);
+    if (c->dt == CM_F32)
+        return from_cuda(launch_encode_f32(cp, (const float *)A, lda, (float *)par, ldp,
+                                           (cudaStream_t)stream));
+    return from_cuda(launch_encode_bf16(cp, (const uint16_t *)A, lda, (uint16_t *)par, ldp,
+                                        (cudaStream_t)stream));
+}
+
+cm_status cm_matvec(const cm_code *c, const float *A, int64_t lda, const float *par,
+                    int64_t ldp, const float *X, int32_t b, double *Yt, cm_stream_t stream)
+{
+    if (!c || c->dt != CM_F32) return CM_EINVAL;
+    if (b < 1 || b > 8 || !X || !Yt) return CM_EINVAL;
+    if (!layout_ok(A, lda, c->d, 4) || !layout_ok(par, ldp, c->d, 4)) return CM_EINVAL;
+    if (((uintptr_t)X & 3u) || ((uintptr_t)Yt & 7u)) return CM_EINVAL;
+    return from_cuda(launch_matvec(code_params(c), A, lda, par, ldp, X, b, Yt,
+                                   (cudaStream_t)stream));
+}
+
+cm_status cm_decode(const cm_code *c, const double *Yt, uint32_t survivors, int32_t b,
+                    float *Y, int32_t *dev_status, cm_stream_t stream)
+{
+    if (!c) return CM_EINVAL;
+    cm_status st = check_survivors(c, survivors);
+    if (st != CM_OK) return st;
+    if (b < 1 || !Yt || !Y || ((uintptr_t)Yt & 7u) || ((uintptr_t)Y & 3u)) return CM_EINVAL;
+    return from_cuda(launch_decode(code_params(c), Yt, survivors, b, Y, dev_status,
+                                   DEC_PLAIN, nullptr, 0.f, (cudaStream_t)stream));
+}
+
+// Workspace of a gradient step: stacked results of both products (fp64) and
+// the residual z (fp32), each 256-byte aligned.
+static size_t round256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+size_t cm_gd_workspace_bytes(const cm_code *cA, const cm_code *cAT)
+{
+    if (!cA || !cAT) return 0;
+    return round256(sizeof(double) * (size_t)cA->n * cA->L) +
+           round256(sizeof(float) * (size_t)cA->m) +
+           round256(sizeof(double) * (size_t)cAT->n * cAT->L);
+}
+
+cm_status cm_gd_step(const cm_code *cA, const float *A, int64_t lda, const float *PA,
+                     int64_t ldpa, const cm_code *cAT, const float *AT, int64_t ldat,
+                     const float *PAT, int64_t ldpat, const float *y, float *x, float eta,
+                     uint32_t surv_A, uint32_t surv_AT, void *ws, size_t ws_bytes,
+                     int32_t *dev_status, cm_stream_t stream)
+{
+    if (!cA || !cAT || cA->dt != CM_F32 || cAT->dt != CM_F32) return CM_EINVAL;
+    if (cAT->m != cA->d || cAT->d != cA->m || cAT->n != cA->n) return CM_EINVAL;
+    cm_status st = check_survivors(cA, surv_A);
+    if (st != CM_OK) return st;
+    st = check_survivors(cAT, surv_AT);
+    if (st != CM_OK) return st;
+    if (!layout_ok(A, lda, cA->d, 4) || !layout_ok(PA, ldpa, cA->d, 4) ||
+        !layout_ok(AT, ldat, cAT->d, 4) || !layout_ok(PAT, ldpat, cAT->d, 4))
+        return CM_EINVAL;
+    if (!y || !x || ((uintptr_t)y & 3u) || ((uintptr_t)x & 3u) || !std::isfinite(eta))
+        return CM_EINVAL;
+    if (!ws || ((uintptr_t)ws & 255u)) return CM_EINVAL;
+    if (ws_bytes < cm_gd_workspace_bytes(cA, cAT)) return CM_ENOMEM;
+    char *w = (char *)ws;
+    double *ytA = (double *)w;
+    w += round256(sizeof(double) * (size_t)cA->n * cA->L);
+    float *z = (float *)w;
+    w += round256(sizeof(float) * (size_t)cA->m);
+    double *ytAT = (double *)w;
+
+    cudaStream_t s = (cudaStream_t)stream;
+    CodeParams pA = code_params(cA), pAT = code_params(cAT);
+    // Sec. III-E: the master multicasts x, decodes A x from any k1 results ...
+    if (launch_matvec(pA, A, lda, PA, ldpa, x, 1, ytA, s) != cudaSuccess) return CM_ECUDA;
+    // ... forms z = A x - y and multicasts it ...
+    if (launch_decode(pA, ytA, surv_A, 1, z, dev_status, DEC_RESIDUAL, y, 0.f, s) != cudaSuccess)
+        return CM_ECUDA;
+    // ... decodes A^T z from any k2 results and steps x <- x - eta A^T z.
+    if (launch_matvec(pAT, AT, ldat, PAT, ldpat, z, 1, ytAT, s) != cudaSuccess) return CM_ECUDA;
+    if (launch_decode(pAT, ytAT, surv_AT, 1, x, dev_status, DEC_DESCENT, nullptr, eta, s) !=
+        cudaSuccess)
+        return CM_ECUDA;
+    return CM_OK;
+}
+
+cm_status cm_coded_gemm(const cm_code *c, const void *A, int64_t lda, const void *par,
+                        int64_t ldp, const void *Bt, int64_t ldb, int32_t N, float *Ct,
+                        int64_t ldc, cm_stream_t stream)
+{
+    if (!c || c->dt != CM_BF16) return CM_EINVAL;
+    if (N < 16 || N % 16 != 0 || c->d % 8 != 0) return CM_EINVAL;
+    if (!layout_ok(A, lda, c->d, 2) || !layout_ok(par, ldp, c->d, 2) ||
+        !layout_ok(Bt, ldb, c->d, 2))
+        return CM_EINVAL;
+    if (!Ct || ((uintptr_t)Ct & 15u) || ldc < N || ldc % 4 != 0) return CM_EINVAL;
+    return from_cuda(launch_coded_gemm(code_params(c), (const uint16_t *)A, lda,
+                                       (const uint16_t *)par, ldp, (const uint16_t *)Bt, ldb,
+                                       N, Ct, ldc, (cudaStream_t)stream));
+}
+
+cm_status cm_decode_mat(const cm_code *c, const float *Ct, int64_t ldc, uint32_t survivors,
+                        int32_t N, float *C, int64_t ldcc, int32_t *dev_status,
+                        cm_stream_t stream)
+{
+    if (!c) return CM_EINVAL;
+    cm_status st = check_survivors(c, survivors);
+    if (st != CM_OK) return st;
+    if (N < 1 || !Ct || !C || ldc < N || ldcc < N || ((uintptr_t)Ct & 3u) ||
+        ((uintptr_t)C & 3u))
+        return CM_EINVAL;
+    if (C == Ct && ldcc != ldc) return CM_EINVAL;
+    return from_cuda(launch_decode_mat(code_params(c), Ct, ldc, survivors, N, C, ldcc,
+                                       dev_status, (cudaStream_t)stream));
+}
+
+cm_status cm_matmat(const cm_code *c, const void *A, int64_t lda, const void *par,
+                    int64_t ldp, const void *Bt, int64_t ldb, int32_t N, float *Ct,
+                    int64_t ldc, uint32_t survivors, float *C, int64_t ldcc,
+                    int32_t *dev_status, cm_stream_t stream)
+{
+    if (!c) return CM_EINVAL;
+    cm_status st = check_survivors(c, survivors);
+    if (st != CM_OK) return st;
+    st = cm_coded_gemm(c, A, lda, par, ldp, Bt, ldb, N, Ct, ldc, stream);
+    if (st != CM_OK) return st;
+    return cm_decode_mat(c, Ct, ldc, survivors, N, C, ldcc, dev_status, stream);
+}
+
+const char *cm_status_string(cm_status s)
+{
+    switch (s) {
+    case CM_OK: return "ok";
+    case CM_EINVAL: return "invalid argument, shape, alignment or dtype";
+    case CM_ENOTDECODABLE: return "fewer than k survivors: not decodable";
+    case CM_ESINGULAR: return "singular generator submatrix G_S";
+    case CM_ECUDA: return "CUDA launch or query failed";
+    case CM_ENOMEM: return "out of memory or workspace too small";
+    case CM_ETIMEOUT: return "bounded device wait gave up";
+    case CM_EUNSUPPORTED: return "unsupported request";
+    }
+    return "unknown status";
+}
+
+}  // extern "C"

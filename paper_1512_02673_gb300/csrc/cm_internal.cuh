@@ -1,0 +1,61 @@
+// Internal declarations shared by the libcm translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/cm.h"
+
+#define CM_MAX_N 32
+#define CM_MAX_P 256   // (n-k) k <= 16 * 16 for n <= 32
+
+struct cm_code {
+    int32_t n, k;
+    int64_t m, d, L;
+    cm_dtype dt;
+    float P[CM_MAX_P];   // (n-k) x k, row-major
+};
+
+// The code as a kernel parameter (passed by value; P lands in the constant
+// parameter bank, read with uniform broadcast loads).
+struct CodeParams {
+    int32_t n, k;
+    int64_t m, d, L;
+    float P[CM_MAX_P];
+};
+
+inline CodeParams code_params(const cm_code *c)
+{
+    CodeParams p;
+    p.n = c->n;
+    p.k = c->k;
+    p.m = c->m;
+    p.d = c->d;
+    p.L = c->L;
+    for (int i = 0; i < CM_MAX_P; ++i) p.P[i] = c->P[i];
+    return p;
+}
+
+// Number of SMs of the current device (cached per device).
+int cm_sm_count();
+
+// ---- launchers (return cudaSuccess or the launch error) --------------------
+cudaError_t launch_encode_f32(const CodeParams &cp, const float *A, int64_t lda,
+                              float *par, int64_t ldp, cudaStream_t s);
+cudaError_t launch_encode_bf16(const CodeParams &cp, const uint16_t *A, int64_t lda,
+                               uint16_t *par, int64_t ldp, cudaStream_t s);
+cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda,
+                          const float *par, int64_t ldp, const float *X, int b,
+                          double *Yt, cudaStream_t s);
+
+// Decode epilogues (Sec. III-E: the two decodes of a gradient step).
+enum DecodeMode { DEC_PLAIN = 0, DEC_RESIDUAL = 1, DEC_DESCENT = 2 };
+cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survivors,
+                          int b, float *Y, int32_t *status, int mode,
+                          const float *lab, float eta, cudaStream_t s);
+cudaError_t launch_decode_mat(const CodeParams &cp, const float *Ct, int64_t ldc,
+                              uint32_t survivors, int N, float *C, int64_t ldcc,
+                              int32_t *status, cudaStream_t s);
+cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t lda,
+                              const uint16_t *par, int64_t ldp, const uint16_t *Bt,
+                              int64_t ldb, int N, float *Ct, int64_t ldc, cudaStream_t s);

@@ -1,0 +1,334 @@
+"""GPU parity of the coded mat-(multi-)vec path against the CPU oracle.
+
+Every test calls the CUDA library through its C ABI (via the ctypes binding)
+and compares with the oracle on the same seeded inputs.  Tolerances:
+  * encode (fp32 accumulation of k terms): |gpu - exact| <= 2 k u32 sum_i |P||A|
+    elementwise (u32 = 2^-24), the standard bound for a k-term dot product;
+  * worker products (fp32 partials of <= 16 terms combined in fp64): relative
+    l2 error <= 1e-6 per worker block per vector against the oracle's fp64
+    products of the same (GPU) coded blocks;
+  * decoded A X: relative l2 error <= 1e-4 per output vector against the
+    oracle's fp64 A X (the plain definition), as the method fixes it;
+  * survivor masks and every index decision: bit-exact;
+  * integer single-parity codes: bit-exact.
+"""
+import itertools
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+
+pytestmark = pytest.mark.gpu
+
+U32 = 2.0 ** -24
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module")
+def cm():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import os
+    import paper_1512_02673_gb300 as cm
+    if not os.path.exists(cm.LIB_PATH):
+        from paper_1512_02673_gb300 import build
+        build.build()
+    return cm
+
+
+def rel_l2_cols(got, want):
+    """Relative l2 error of every column (output vector)."""
+    got = np.asarray(got, np.float64)
+    want = np.asarray(want, np.float64)
+    num = np.linalg.norm(got - want, axis=0)
+    den = np.linalg.norm(want, axis=0)
+    return num / np.where(den > 0, den, 1.0)
+
+
+def padded(rows, cols, ld, seed, device=DEV):
+    """rows x cols N(0,1) fp32 view with leading dimension ld (a strided view)."""
+    base = synth.gaussian((rows, ld), seed, "cpu")
+    return base.to(device)[:, :cols]
+
+
+def check_encode(orc, n, k, A_cpu, P, par_gpu):
+    want, bound = orc.encode(n, k, A_cpu.numpy(), P.astype(np.float64), with_bound=True)
+    got = par_gpu.double().cpu().numpy()
+    tol = 2 * k * U32 * bound + 1e-30
+    bad = np.abs(got - want) > tol
+    assert not bad.any(), "encode: %d elements out of bound, worst excess %g" % (
+        bad.sum(), (np.abs(got - want) - tol).max())
+
+
+def check_workers(orc, n, k, A_cpu, par_gpu, X_cpu, Yt_gpu, L):
+    want = orc.worker_outputs(n, k, A_cpu.numpy(), par_gpu.float().cpu().numpy(), X_cpu.numpy())
+    got = Yt_gpu.cpu().numpy()
+    for j in range(n):
+        blk = slice(j * L, (j + 1) * L)
+        w = want[blk]
+        if np.linalg.norm(w) == 0:
+            assert np.all(got[blk] == 0)
+            continue
+        err = rel_l2_cols(got[blk], w)
+        assert err.max() <= 1e-6, (j, err)
+
+
+def run_path(cm, orc, n, k, m, d, b, seed=7, lda=None, misalign_x=False, counter=0):
+    P = synth.parity_coefficients(n, k)
+    code = cm.Code(n, k, m, d, P)
+    lda = lda or d
+    A = padded(m, d, lda, seed)
+    A_cpu = A.cpu().contiguous()
+    X_cpu = synth.gaussian((d, b), seed + 1)
+    if misalign_x:
+        buf = torch.zeros(d * b + 1, device=DEV)
+        X = buf[1:].view(d, b)
+        X.copy_(X_cpu)
+    else:
+        X = X_cpu.to(DEV)
+    par = cm.encode(code, A)
+    Yt = cm.matvec(code, A, par, X)
+    mask, _ = cm.draw_erasures(synth.ERASURE_SEED, counter, n, k)
+    omask, _ = orc.draw_erasures(synth.ERASURE_SEED, counter, n, k)
+    assert mask == omask
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    Y = cm.decode(code, Yt, mask, status=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    return dict(P=P, code=code, A=A, A_cpu=A_cpu, X=X, X_cpu=X_cpu, par=par, Yt=Yt, mask=mask,
+                Y=Y)
+
+
+# ---- config 1 and small shapes spanning several tiles with ragged tails ------------
+
+def test_tiny_config_end_to_end(cm, orc):
+    w = synth.TINY
+    r = run_path(cm, orc, w.n, w.k, w.m, w.d, w.b, seed=synth.DATA_SEED)
+    check_encode(orc, w.n, w.k, r["A_cpu"], r["P"], r["par"])
+    check_workers(orc, w.n, w.k, r["A_cpu"], r["par"], r["X_cpu"], r["Yt"], r["code"].L)
+    want = orc.matmul(r["A_cpu"].numpy(), r["X_cpu"].numpy())
+    assert rel_l2_cols(r["Y"].cpu().numpy(), want).max() <= 1e-4
+    # stage check: the oracle's own decode (Gaussian elimination) of the GPU's results
+    Yo = orc.decode(w.n, w.k, w.m, r["P"].astype(np.float64), r["mask"], r["Yt"].cpu().numpy())
+    assert rel_l2_cols(r["Y"].cpu().numpy(), Yo).max() <= 1e-6
+
+
+SHAPES = [
+    # n, k, m, d, b, lda
+    (6, 3, 1200, 500, 1, None),
+    (5, 4, 37, 130, 1, 132),      # m % k != 0, ragged d, padded leading dimension
+    (10, 5, 2003, 1029, 3, 1032),
+    (20, 10, 613, 257, 8, 260),
+    (32, 24, 1000, 640, 8, None),  # n - k = 8
+    (32, 8, 190, 84, 2, None),     # n - k = 24: two encode passes
+    (3, 2, 5, 7, 5, 8),            # fewer rows than one warp's group
+    (16, 12, 3001, 4096, 4, None),
+    (7, 3, 300, 9000, 6, 9004),    # several X chunks (b = 6 pads to 8)
+    (12, 5, 700, 17000, 1, None),  # several X chunks at b = 1
+]
+
+
+@pytest.mark.parametrize("n,k,m,d,b,lda", SHAPES)
+def test_path_matches_oracle(cm, orc, n, k, m, d, b, lda):
+    r = run_path(cm, orc, n, k, m, d, b, lda=lda, seed=n * 1000 + d)
+    check_encode(orc, n, k, r["A_cpu"], r["P"], r["par"])
+    check_workers(orc, n, k, r["A_cpu"], r["par"], r["X_cpu"], r["Yt"], r["code"].L)
+    want = orc.matmul(r["A_cpu"].numpy(), r["X_cpu"].numpy())
+    assert rel_l2_cols(r["Y"].cpu().numpy(), want).max() <= 1e-4
+
+
+@pytest.mark.parametrize("b", [1, 4, 8, 3])
+def test_misaligned_x_uses_general_staging(cm, orc, b):
+    n, k, m, d = 6, 3, 500, 301
+    r = run_path(cm, orc, n, k, m, d, b, lda=304, misalign_x=True)
+    check_workers(orc, n, k, r["A_cpu"], r["par"], r["X_cpu"], r["Yt"], r["code"].L)
+
+
+def test_decode_from_every_k_subset(cm, orc):
+    for n, k in [(6, 3), (10, 5)]:
+        m, d, b = 301, 203, 2
+        r = run_path(cm, orc, n, k, m, d, b, lda=204)
+        want = orc.matmul(r["A_cpu"].numpy(), r["X_cpu"].numpy())
+        for S in itertools.combinations(range(n), k):
+            mask = sum(1 << j for j in S)
+            Y = cm.decode(r["code"], r["Yt"], mask)
+            err = rel_l2_cols(Y.cpu().numpy(), want)
+            assert err.max() <= 1e-4, (S, err)
+
+
+def test_extra_survivors_use_the_lowest_k(cm, orc):
+    n, k, m, d = 10, 5, 400, 128
+    r = run_path(cm, orc, n, k, m, d, 1)
+    for mask in [0b1111111111, 0b1110111011, 0b1111100000 | 0b1]:
+        lowest = 0
+        for j in range(n):
+            if mask >> j & 1 and bin(lowest).count("1") < k:
+                lowest |= 1 << j
+        a = cm.decode(r["code"], r["Yt"], mask).cpu()
+        bb = cm.decode(r["code"], r["Yt"], lowest).cpu()
+        assert torch.equal(a, bb)
+
+
+@pytest.mark.parametrize("n", [4, 6])
+def test_single_parity_integer_code_is_bit_exact(cm, orc, n):
+    k = n - 1
+    m, d = 1200, 500
+    A = synth.small_integers((m, d), -4, 4, seed=11)
+    X = synth.small_integers((d, 3), -4, 4, seed=12)
+    code = cm.Code(n, k, m, d, np.ones((1, k), np.float32))
+    Ad, Xd = A.to(DEV), X.to(DEV)
+    par = cm.encode(code, Ad)
+    Yt = cm.matvec(code, Ad, par, Xd)
+    want = (A.long() @ X.long()).numpy()
+    for erased in range(n):
+        mask = ((1 << n) - 1) & ~(1 << erased)
+        Y = cm.decode(code, Yt, mask)
+        assert np.array_equal(Y.cpu().numpy().astype(np.int64), want), erased
+        Yo = orc.decode(n, k, m, np.ones((1, k)), mask, Yt.cpu().numpy())
+        assert np.array_equal(Yo, want.astype(np.float64))
+
+
+def test_singular_generator_sets_status(cm):
+    n, k, m, d = 6, 3, 90, 40
+    P = synth.parity_coefficients(n, k)
+    P[1] = P[0]                               # duplicated parity rows
+    code = cm.Code(n, k, m, d, P)
+    A = synth.gaussian((m, d), 3).to(DEV)
+    X = synth.gaussian((d, 1), 4).to(DEV)
+    par = cm.encode(code, A)
+    Yt = cm.matvec(code, A, par, X)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    Y = torch.full((m, 1), 7.0, device=DEV)
+    cm.decode(code, Yt, 0b011001, Y=Y, status=status)     # survivors {0, 3, 4}
+    torch.cuda.synchronize()
+    assert status.item() == cm.CM_ESINGULAR
+    assert torch.all(Y == 7.0)                # nothing written
+    P2 = synth.parity_coefficients(n, k)
+    P2[2] = 0.0                               # a zero parity row
+    code2 = cm.Code(n, k, m, d, P2)
+    status.zero_()
+    cm.decode(code2, Yt, 0b100011, status=status)
+    torch.cuda.synchronize()
+    assert status.item() == cm.CM_ESINGULAR
+    with pytest.raises(cm.CodedError) as e:
+        cm.decode(code, Yt, 0b000011)
+    assert e.value.status == cm.CM_ENOTDECODABLE
+
+
+def test_outputs_stay_inside_their_buffers(cm):
+    """Guard canaries after Yt, Y and the parity buffer stay untouched."""
+    n, k, m, d, b = 10, 5, 1003, 515, 3
+    P = synth.parity_coefficients(n, k)
+    code = cm.Code(n, k, m, d, P)
+    L = code.L
+    A = padded(m, d, 516, 5)
+    X = synth.gaussian((d, b), 6).to(DEV)
+    G = 4096
+    par_buf = torch.full(((n - k) * L * 516 + G,), 123.0, device=DEV)
+    par = par_buf[:(n - k) * L * 516].view((n - k) * L, 516)[:, :d]
+    yt_buf = torch.full((n * L * b + G,), 321.0, dtype=torch.float64, device=DEV)
+    y_buf = torch.full((m * b + G,), 555.0, device=DEV)
+    cm.encode(code, A, par)
+    Yt = cm.matvec(code, A, par, X, Yt=yt_buf[:n * L * b].view(n * L, b))
+    mask, _ = cm.draw_erasures(1, 1, n, k)
+    cm.decode(code, Yt, mask, Y=y_buf[:m * b].view(m, b))
+    torch.cuda.synchronize()
+    assert torch.all(par_buf[(n - k) * L * 516:] == 123.0)
+    assert torch.all(par_buf[:(n - k) * L * 516].view(-1, 516)[:, d:] == 123.0)
+    assert torch.all(yt_buf[n * L * b:] == 321.0)
+    assert torch.all(y_buf[m * b:] == 555.0)
+
+
+def test_results_are_bitwise_repeatable(cm, orc):
+    n, k, m, d, b = 16, 12, 3000, 3000, 8
+    r = run_path(cm, orc, n, k, m, d, b)
+    Yt2 = cm.matvec(r["code"], r["A"], r["par"], r["X"])
+    par2 = cm.encode(r["code"], r["A"])
+    Y2 = cm.decode(r["code"], Yt2, r["mask"])
+    torch.cuda.synchronize()
+    assert torch.equal(r["par"], par2)
+    assert torch.equal(r["Yt"], Yt2)
+    assert torch.equal(r["Y"], Y2)
+
+
+def test_empty_and_degenerate_shapes(cm, orc):
+    # one row, one column, k = 1 (repetition of a single block), n = k + 1
+    for (n, k, m, d, b) in [(2, 1, 1, 1, 1), (3, 1, 5, 4, 2), (2, 1, 1, 129, 8), (32, 31, 31, 4, 1)]:
+        r = run_path(cm, orc, n, k, m, d, b, lda=((d + 3) // 4) * 4)
+        want = orc.matmul(r["A_cpu"].numpy(), r["X_cpu"].numpy())
+        assert rel_l2_cols(r["Y"].cpu().numpy(), want).max() <= 1e-4
+
+
+# ---- full-size workloads ---------------------------------------------------------------
+
+def test_matvec_config_100_repeats(cm, orc):
+    w = synth.MATVEC
+    P = synth.parity_coefficients(w.n, w.k)
+    code = cm.Code(w.n, w.k, w.m, w.d, P)
+    A, X = synth.matvec_inputs(w, device="cpu")
+    Ad, Xd = A.to(DEV), X.to(DEV)
+    par = cm.encode(code, Ad)
+    want = orc.matmul(A.numpy(), X.numpy())
+    G = np.vstack([np.eye(w.k), P.astype(np.float64)])
+    errs, kappas = [], []
+    for rep in range(w.repeats):
+        # each repeat: the n worker products, a fresh erasure set, a decode
+        Yt = cm.matvec(code, Ad, par, Xd)
+        mask, _ = cm.draw_erasures(synth.ERASURE_SEED, rep, w.n, w.k)
+        assert mask == orc.draw_erasures(synth.ERASURE_SEED, rep, w.n, w.k)[0]
+        Y = cm.decode(code, Yt, mask)
+        errs.append(rel_l2_cols(Y.cpu().numpy(), want).max())
+        kappas.append(np.linalg.cond(G[[j for j in range(w.n) if mask >> j & 1]]))
+    worst = int(np.argmax(errs))
+    assert max(errs) <= 1e-4, (max(errs), kappas[worst])
+
+
+def sampled_rows(L, k, m, count, seed):
+    rng = np.random.default_rng(seed)
+    rs = sorted(set([0, L - 1] + rng.integers(0, L, count).tolist()))
+    return rs
+
+
+def test_bandwidth_config_sampled(cm, orc):
+    """(32,24), A 65536 x 65536 fp32 (16 GiB), b = 8: the bench's launch
+    configuration, checked on sampled block rows against the oracle."""
+    w = synth.BANDWIDTH
+    P = synth.parity_coefficients(w.n, w.k)
+    code = cm.Code(w.n, w.k, w.m, w.d, P)
+    L = code.L
+    A, X = synth.matvec_inputs(w, device=DEV)
+    par = cm.encode(code, A)
+    Yt = cm.matvec(code, A, par, X)
+    mask, _ = cm.draw_erasures(synth.ERASURE_SEED, 0, w.n, w.k)
+    assert mask == orc.draw_erasures(synth.ERASURE_SEED, 0, w.n, w.k)[0]
+    Y = cm.decode(code, Yt, mask)
+    torch.cuda.synchronize()
+    rs = sampled_rows(L, w.k, w.m, 14, 99)
+    s = len(rs)
+    X_cpu = X.cpu()
+    # sub-problem: block i of A_sub holds rows i L + r (r in rs) of the padded A
+    idx = torch.tensor([i * L + r for i in range(w.k) for r in rs])
+    valid = idx < w.m
+    A_sub = torch.zeros((w.k * s, w.d))
+    A_sub[valid] = A[idx[valid].to(DEV)].cpu()
+    # encode on the sampled rows
+    par_rows = torch.tensor([p * L + r for p in range(w.n - w.k) for r in rs])
+    par_s = par[par_rows.to(DEV)].cpu()
+    check_encode(orc, w.n, w.k, A_sub, P, par_s)
+    # worker products on the sampled rows (oracle on the GPU's parity)
+    Yt_s = torch.stack([Yt[j * L + r] for j in range(w.n) for r in rs]).cpu()
+    check_workers(orc, w.n, w.k, A_sub, par_s, X_cpu, Yt_s, s)
+    # decoded A X on the sampled rows: the plain definition
+    want = orc.matmul(A_sub[valid].numpy(), X_cpu.numpy())
+    got = Y[idx[valid].to(DEV)].cpu().numpy()
+    assert rel_l2_cols(got, want).max() <= 1e-4
+    # property at full size: surviving systematic blocks pass through exactly
+    for i in range(w.k):
+        if mask >> i & 1:
+            lo, hi = i * L, min((i + 1) * L, w.m)
+            assert torch.equal(Y[lo:hi], Yt[lo:hi].float())
+    del A, par, Yt
+    torch.cuda.empty_cache()

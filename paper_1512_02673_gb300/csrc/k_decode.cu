@@ -28,9 +28,11 @@ constexpr int kMaxE = 16;   // e <= min(k, n - k) <= 16 for n <= 32
 struct DecodeShared {
     int S[CM_MAX_N];       // survivors in ascending order (k of them)
     int role[CM_MAX_N];    // block i < k: -1 passes through, else its row c in M
+    int Ps[kMaxE];         // surviving parity workers, ascending
     int e;
     int singular;
     double W[kMaxE][2 * kMaxE];   // [Q | I] during elimination
+    double Qi[kMaxE][kMaxE];      // Q^-1
     double D[kMaxE][CM_MAX_N];    // decode rows: D[c][p], p = position in S
 };
 
@@ -50,6 +52,7 @@ __device__ void decode_coefficients(const CodeParams &cp, uint32_t survivors, De
     const uint32_t parm = __ballot_sync(0xffffffffu, par);
     const int e = __popc(missm);
     if (sel) sh.S[__popc(selm & below)] = lane;
+    if (par) sh.Ps[__popc(parm & below)] = lane;
     if (lane < k) sh.role[lane] = miss ? __popc(missm & below) : -1;
     // per-lane copies of the M and Ps lists (lane-indexed via shuffles)
     int Mi = -1, Pi = -1;
@@ -113,10 +116,10 @@ __device__ void decode_coefficients(const CodeParams &cp, uint32_t survivors, De
             sh.W[bi][lane] = t;
         }
         __syncwarp();
-        const double pv = sh.W[col][col];
+        const double rp = 1.0 / sh.W[col][col];
         double f[kMaxE];
 #pragma unroll
-        for (int a = 0; a < kMaxE; ++a) f[a] = a < e ? sh.W[a][col] / pv : 0.0;
+        for (int a = 0; a < kMaxE; ++a) f[a] = a < e ? sh.W[a][col] * rp : 0.0;
         __syncwarp();
         if (lane < 2 * e) {
             const double wc = sh.W[col][lane];
@@ -131,26 +134,25 @@ __device__ void decode_coefficients(const CodeParams &cp, uint32_t survivors, De
         __syncwarp();
         return;
     }
-    // Q^-1[c][a] = W[c][e + a] / W[c][c]; lane p < k builds column p of D.
+    // Q^-1[c][a] = W[c][e + a] / W[c][c]
+    for (int t = lane; t < e * e; t += 32) {
+        const int c = t / e, aa = t % e;
+        sh.Qi[c][aa] = sh.W[c][e + aa] / sh.W[c][c];
+    }
+    __syncwarp();
+    // lane p < k builds column p of D (p = position in S)
     if (lane < k) {
         const int s = sh.S[lane];
-        for (int c = 0; c < e; ++c) {
-            const double dc = sh.W[c][c];
-            double v;
-            if (s >= k) {
-                const int a = __popc(parm & ((1u << s) - 1u));
-                v = sh.W[c][e + a] / dc;
-            } else {
-                v = 0.0;
-                for (int a = 0; a < e; ++a) {
-                    // Ps[a] is the a-th set bit of parm
-                    uint32_t mm = parm;
-                    for (int t = 0; t < a; ++t) mm &= mm - 1;
-                    const int psa = __ffs(mm) - 1;
-                    v -= (sh.W[c][e + a] / dc) * (double)cp.P[(psa - k) * k + s];
-                }
+        if (s >= k) {
+            const int aa = __popc(parm & ((1u << s) - 1u));
+            for (int c = 0; c < e; ++c) sh.D[c][lane] = sh.Qi[c][aa];
+        } else {
+            for (int c = 0; c < e; ++c) {
+                double v = 0.0;
+                for (int aa = 0; aa < e; ++aa)
+                    v = fma(-sh.Qi[c][aa], (double)cp.P[(sh.Ps[aa] - k) * k + s], v);
+                sh.D[c][lane] = v;
             }
-            sh.D[c][lane] = v;
         }
     }
     __syncwarp();
@@ -287,10 +289,13 @@ decode_mat_kernel(const CodeParams cp, const float *Ct, int64_t ldc, uint32_t su
     }
 }
 
-int grid_for(int64_t items)
+// Every CTA inverts the small block of G_S itself, so the grid is capped at
+// `per_sm` CTAs per SM: enough to stream the results, few enough that the
+// (slow on this part) fp64 inverse is not repeated needlessly.
+int grid_for(int64_t items, int per_sm)
 {
     int64_t g = (items + kThreads - 1) / kThreads;
-    const int64_t cap = (int64_t)(cm_sm_count() > 0 ? cm_sm_count() : 1) * 8;
+    const int64_t cap = (int64_t)(cm_sm_count() > 0 ? cm_sm_count() : 1) * per_sm;
     if (g > cap) g = cap;
     if (g < 1) g = 1;
     return (int)g;
@@ -312,7 +317,7 @@ cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survi
     a.mode = mode;
     a.lab = lab;
     a.eta = eta;
-    decode_kernel<<<grid_for((int64_t)cp.k * cp.L * b), kThreads, 0, s>>>(a);
+    decode_kernel<<<grid_for((int64_t)cp.k * cp.L * b, 1), kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -328,7 +333,7 @@ cudaError_t launch_decode_mat(const CodeParams &cp, const float *Ct, int64_t ldc
             if (j >= cp.k) ++e;
         }
     const int64_t items = cp.L * (int64_t)N / 4 + 1;
-    const int g = grid_for(items);
+    const int g = grid_for(items, 4);
     if (e <= 4)
         decode_mat_kernel<4><<<g, kThreads, 0, s>>>(cp, Ct, ldc, survivors, N, C, ldcc, status);
     else if (e <= 8)

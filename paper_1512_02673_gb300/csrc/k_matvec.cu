@@ -38,7 +38,6 @@ struct XCfg {
     // distinct bank groups.
     static constexpr int GS = BP == 1 ? 0 : (BP == 4 ? CX + 8 : CX + 4);
     static constexpr int FLOATS = BP == 1 ? CX : (BP == 4 ? 4 * GS : 8 * GS);
-    static constexpr int BYTES = FLOATS * 4;
 };
 
 struct MatvecArgs {
@@ -74,15 +73,6 @@ __device__ __forceinline__ void cp_async4(float *dst, const float *src, int byte
 
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
-
-__device__ __forceinline__ float4 ld_stream4(const float *p)
-{
-    float4 v;
-    asm("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];\n"
-        : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-        : "l"(p));
-    return v;
-}
 
 // Stage columns [c0, c0 + CX) of X into smem buffer xs (zero past d / b).
 template <int BP>
@@ -156,152 +146,219 @@ __device__ __forceinline__ void flush(float (&t)[V], double (&acc64)[V >= 32 ? V
     for (int i = 0; i < V; ++i) t[i] = 0.f;
 }
 
-template <int BP, int R, int F>
-__global__ void __launch_bounds__(kThreads)
+// cp.async.wait_group with a run-time count (the instruction takes an immediate)
+__device__ __forceinline__ void cp_async_wait_upto(int n)
+{
+    switch (n) {
+    case 0: asm volatile("cp.async.wait_group 0;\n" ::: "memory"); break;
+    case 1: asm volatile("cp.async.wait_group 1;\n" ::: "memory"); break;
+    case 2: asm volatile("cp.async.wait_group 2;\n" ::: "memory"); break;
+    case 3: asm volatile("cp.async.wait_group 3;\n" ::: "memory"); break;
+    case 4: asm volatile("cp.async.wait_group 4;\n" ::: "memory"); break;
+    case 5: asm volatile("cp.async.wait_group 5;\n" ::: "memory"); break;
+    case 6: asm volatile("cp.async.wait_group 6;\n" ::: "memory"); break;
+    default: asm volatile("cp.async.wait_group 7;\n" ::: "memory"); break;
+    }
+}
+
+// Rows of work unit g: R row pointers (NULL = virtual zero row or past L).
+template <int R>
+__device__ __forceinline__ void unit_rows(const MatvecArgs &a, int64_t g, const float *(&rowp)[R],
+                                          int &j, int64_t &rr0)
+{
+    const bool has = g < a.groups;
+    j = has ? (int)(g % a.n) : 0;
+    rr0 = has ? (g / a.n) * R : 0;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const int64_t rr = rr0 + r;
+        rowp[r] = nullptr;
+        if (has && rr < a.L) {
+            if (j < a.k) {
+                const int64_t gr = (int64_t)j * a.L + rr;
+                if (gr < a.m) rowp[r] = a.A + gr * a.lda;
+            } else {
+                rowp[r] = a.par + ((int64_t)(j - a.k) * a.L + rr) * a.ldp;
+            }
+        }
+    }
+}
+
+// A streams into a per-warp ring of ST steps (R rows x 128 columns each) by
+// cp.async: lane l copies, and later reads back, only its own 16 bytes of
+// every row, so completion needs just cp.async.wait_group (no barrier, no
+// spin).  ST-1 steps are in flight per warp while the warp computes.
+template <int BP, int R, int ST, int F>
+__global__ void __launch_bounds__(kThreads, 1)
 matvec_kernel(const MatvecArgs a)
 {
     using C = XCfg<BP>;
     constexpr int V = R * BP;
     constexpr int NH = V >= 32 ? V / 32 : 1;
+    constexpr int IPC = C::CX / 128;   // steps per X chunk
+    static_assert(ST >= 2 && ST <= 8, "ring depth");
     extern __shared__ __align__(16) float smem[];
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
+    float *ring = smem + 2 * C::FLOATS + warp * (ST * R * 128);
     const int64_t total_warps = (int64_t)gridDim.x * kWarps;
     const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
     const int64_t rounds = (a.groups + total_warps - 1) / total_warps;
-    const int64_t nchunks = (a.d + C::CX - 1) / C::CX;
-    const int64_t nseq = rounds * nchunks;
     const int64_t steps = (a.d + 127) / 128;
+    const int64_t nchunks = (a.d + C::CX - 1) / C::CX;
+    const int64_t total = rounds * steps;
 
-    stage_x<BP>(a, smem, 0);
-    int64_t seq = 0;
-    for (int64_t round = 0; round < rounds; ++round) {
-        const int64_t g = round * total_warps + gw;
-        const bool has = g < a.groups;
-        // unit g -> worker j = g % n, rows [rr0, rr0 + R) of that worker
-        const int j = has ? (int)(g % a.n) : 0;
-        const int64_t rr0 = has ? (g / a.n) * R : 0;
-        const float *rowp[R];
-#pragma unroll
-        for (int r = 0; r < R; ++r) {
-            const int64_t rr = rr0 + r;
-            rowp[r] = nullptr;
-            if (has && rr < a.L) {
-                if (j < a.k) {
-                    const int64_t gr = (int64_t)j * a.L + rr;
-                    if (gr < a.m) rowp[r] = a.A + gr * a.lda;
-                } else {
-                    rowp[r] = a.par + ((int64_t)(j - a.k) * a.L + rr) * a.ldp;
-                }
-            }
-        }
-        float acc[V];
-        double acc64[NH];
-#pragma unroll
-        for (int i = 0; i < V; ++i) acc[i] = 0.f;
-#pragma unroll
-        for (int i = 0; i < NH; ++i) acc64[i] = 0.0;
-
-        // A for step s of this lane: columns [128 s + 4 lane, +4)
-        auto load_step = [&](int64_t s, float4 (&v)[R]) {
-            const int64_t col = 128 * s + 4 * lane;
-            const bool full = 128 * s + 128 <= a.d;
+    // ---- issue side: A(step) for the flat step sequence of this warp ----
+    int64_t is_round = 0, is_s = 0;
+    int is_slot = 0;
+    const float *irow[R];
+    {
+        int jj;
+        int64_t r0;
+        unit_rows<R>(a, gw, irow, jj, r0);
+    }
+    int since_x = 0;   // cp.async groups committed after the newest X group
+    auto issue = [&]() {
+        if (is_round < rounds) {
+            const int64_t col = 128 * is_s + 4 * lane;
+            const int64_t left = a.d - col;
+            const int full = left >= 4 ? 16 : (left > 0 ? (int)left * 4 : 0);
+            float *dst = ring + is_slot * (R * 128) + 4 * lane;
 #pragma unroll
             for (int r = 0; r < R; ++r) {
-                v[r] = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (rowp[r]) {
-                    if (full) {
-                        v[r] = ld_stream4(rowp[r] + col);
-                    } else {
-                        const float *p = rowp[r] + col;
-                        if (col + 0 < a.d) v[r].x = __ldg(p + 0);
-                        if (col + 1 < a.d) v[r].y = __ldg(p + 1);
-                        if (col + 2 < a.d) v[r].z = __ldg(p + 2);
-                        if (col + 3 < a.d) v[r].w = __ldg(p + 3);
-                    }
-                }
+                const int bytes = irow[r] ? full : 0;
+                cp_async16(dst + r * 128, bytes ? irow[r] + col : a.A, bytes);
             }
-        };
-
-        float4 cur[R], nxt[R];
-        if (has) load_step(0, cur);
-        int fl = 0;
-        int64_t s = 0;
-        for (int64_t ch = 0; ch < nchunks; ++ch, ++seq) {
-            cp_async_wait_all();
-            __syncthreads();   // chunk `seq` visible; buffer of seq+1 free
-            if (seq + 1 < nseq)
-                stage_x<BP>(a, smem + ((seq + 1) & 1) * C::FLOATS,
-                            ((seq + 1) % nchunks) * C::CX);
-            if (!has) continue;
-            const float *xb = smem + (seq & 1) * C::FLOATS;
-            const int64_t send = min(steps, (ch + 1) * (C::CX / 128));
-            for (; s < send; ++s) {
-                if (s + 1 < steps) load_step(s + 1, nxt);
-                const int c4 = (int)(s - ch * (C::CX / 128)) * 32 + lane;
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    float x[BP];
-                    if constexpr (BP == 1) {
-                        const float4 xv = *reinterpret_cast<const float4 *>(xb + 4 * c4);
-                        x[0] = q == 0 ? xv.x : q == 1 ? xv.y : q == 2 ? xv.z : xv.w;
-                    } else {
-#pragma unroll
-                        for (int h = 0; h < BP / 4; ++h) {
-                            const float4 xv = *reinterpret_cast<const float4 *>(
-                                xb + (q * (BP / 4) + h) * C::GS + 4 * c4);
-                            x[4 * h + 0] = xv.x;
-                            x[4 * h + 1] = xv.y;
-                            x[4 * h + 2] = xv.z;
-                            x[4 * h + 3] = xv.w;
-                        }
-                    }
-#pragma unroll
-                    for (int r = 0; r < R; ++r) {
-                        const float av = q == 0 ? cur[r].x : q == 1 ? cur[r].y
-                                       : q == 2 ? cur[r].z : cur[r].w;
-#pragma unroll
-                        for (int v = 0; v < BP; ++v)
-                            acc[r * BP + v] = fmaf(av, x[v], acc[r * BP + v]);
-                    }
-                }
-#pragma unroll
-                for (int r = 0; r < R; ++r) cur[r] = nxt[r];
-                if (++fl == F) {
-                    flush<V>(acc, acc64, lane);
-                    fl = 0;
-                }
+            if (++is_s == steps) {
+                is_s = 0;
+                ++is_round;
+                int jj;
+                int64_t r0;
+                unit_rows<R>(a, is_round * total_warps + gw, irow, jj, r0);
             }
+            is_slot = is_slot + 1 == ST ? 0 : is_slot + 1;
         }
-        if (!has) continue;
-        if (fl) flush<V>(acc, acc64, lane);
-        // lane holds value index vi = r * BP + v
-        const int64_t base = (int64_t)j * a.L + rr0;
-        if constexpr (V >= 32) {
+        cp_async_commit();
+        ++since_x;
+    };
+
+    stage_x<BP>(a, smem, 0);
+#pragma unroll 1
+    for (int i = 0; i < ST - 1; ++i) issue();
+
+    // ---- compute side ----
+    int64_t xseq = 0;        // X chunks consumed so far (buffer = xseq & 1)
+    int64_t round = 0, s = 0;
+    int slot = 0, fl = 0, j = 0;
+    int64_t rr0 = 0;
+    bool has = false;
+    float acc[V];
+    double acc64[NH];
+#pragma unroll 1
+    for (int64_t f = 0; f < total; ++f) {
+        if (s == 0) {
+            const int64_t g = round * total_warps + gw;
+            has = g < a.groups;
+            const float *dummy[R];
+            unit_rows<R>(a, g, dummy, j, rr0);
 #pragma unroll
-            for (int i = 0; i < NH; ++i) {
-                const int vi = lane * NH + i;
-                const int r = vi / BP, v = vi % BP;
-                if (v < a.b && rr0 + r < a.L) a.Yt[(base + r) * a.b + v] = acc64[i];
+            for (int i = 0; i < V; ++i) acc[i] = 0.f;
+#pragma unroll
+            for (int i = 0; i < NH; ++i) acc64[i] = 0.0;
+            fl = 0;
+        }
+        issue();   // A(f + ST - 1)
+        const int64_t cs = s % IPC;
+        if (cs == 0) {
+            // chunk start: X(this chunk) and A(f) complete, then make X visible
+            cp_async_wait_upto(since_x < ST - 1 ? since_x : ST - 1);
+            __syncthreads();   // also: every warp is done with the other X buffer
+            const int64_t ch = s / IPC;
+            const bool more = ch + 1 < nchunks || round + 1 < rounds;
+            if (more) {
+                stage_x<BP>(a, smem + ((xseq + 1) & 1) * C::FLOATS,
+                            ch + 1 < nchunks ? (ch + 1) * C::CX : 0);
+                since_x = 0;
             }
         } else {
-            constexpr int SHIFT = V == 1 ? 5 : V == 2 ? 4 : V == 4 ? 3 : V == 8 ? 2 : 1;
-            if ((lane & ((1 << SHIFT) - 1)) == 0) {
-                const int vi = lane >> SHIFT;
-                const int r = vi / BP, v = vi % BP;
-                if (v < a.b && rr0 + r < a.L) a.Yt[(base + r) * a.b + v] = acc64[0];
+            cp_async_wait_upto(ST - 1);
+        }
+        if (has) {
+            const float *xb = smem + (xseq & 1) * C::FLOATS;
+            const float *ab = ring + slot * (R * 128) + 4 * lane;
+            const int c4 = (int)cs * 32 + lane;
+            float4 av[R];
+#pragma unroll
+            for (int r = 0; r < R; ++r) av[r] = *reinterpret_cast<const float4 *>(ab + r * 128);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                float x[BP];
+                if constexpr (BP == 1) {
+                    const float4 xv = *reinterpret_cast<const float4 *>(xb + 4 * c4);
+                    x[0] = q == 0 ? xv.x : q == 1 ? xv.y : q == 2 ? xv.z : xv.w;
+                } else {
+#pragma unroll
+                    for (int h = 0; h < BP / 4; ++h) {
+                        const float4 xv = *reinterpret_cast<const float4 *>(
+                            xb + (q * (BP / 4) + h) * C::GS + 4 * c4);
+                        x[4 * h + 0] = xv.x;
+                        x[4 * h + 1] = xv.y;
+                        x[4 * h + 2] = xv.z;
+                        x[4 * h + 3] = xv.w;
+                    }
+                }
+#pragma unroll
+                for (int r = 0; r < R; ++r) {
+                    const float aq = q == 0 ? av[r].x : q == 1 ? av[r].y
+                                   : q == 2 ? av[r].z : av[r].w;
+#pragma unroll
+                    for (int v = 0; v < BP; ++v)
+                        acc[r * BP + v] = fmaf(aq, x[v], acc[r * BP + v]);
+                }
             }
+            if (++fl == F) {
+                flush<V>(acc, acc64, lane);
+                fl = 0;
+            }
+        }
+        slot = slot + 1 == ST ? 0 : slot + 1;
+        const bool chunk_end = cs == IPC - 1 || s == steps - 1;
+        if (chunk_end) ++xseq;
+        if (s == steps - 1) {
+            if (has) {
+                if (fl) flush<V>(acc, acc64, lane);
+                const int64_t base = (int64_t)j * a.L + rr0;
+                if constexpr (V >= 32) {
+#pragma unroll
+                    for (int i = 0; i < NH; ++i) {
+                        const int vi = lane * NH + i;
+                        const int r = vi / BP, v = vi % BP;
+                        if (v < a.b && rr0 + r < a.L) a.Yt[(base + r) * a.b + v] = acc64[i];
+                    }
+                } else {
+                    constexpr int SHIFT = V == 1 ? 5 : V == 2 ? 4 : V == 4 ? 3 : V == 8 ? 2 : 1;
+                    if ((lane & ((1 << SHIFT) - 1)) == 0) {
+                        const int vi = lane >> SHIFT;
+                        const int r = vi / BP, v = vi % BP;
+                        if (v < a.b && rr0 + r < a.L) a.Yt[(base + r) * a.b + v] = acc64[0];
+                    }
+                }
+            }
+            s = 0;
+            ++round;
+        } else {
+            ++s;
         }
     }
     cp_async_wait_all();
 }
 
-template <int BP, int R, int F>
+template <int BP, int R, int ST, int F>
 cudaError_t launch_bp(MatvecArgs a, cudaStream_t s)
 {
     using C = XCfg<BP>;
-    auto kern = matvec_kernel<BP, R, F>;
-    const int smem = 2 * C::BYTES;
+    auto kern = matvec_kernel<BP, R, ST, F>;
+    const int smem = (2 * C::FLOATS + kWarps * ST * R * 128) * 4;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     int per_sm = 0;
@@ -341,12 +398,12 @@ cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, con
     const bool x16 = ((uintptr_t)X & 15u) == 0;
     if (b == 1) {
         a.fast16 = x16;
-        return launch_bp<1, 8, 8>(a, s);
+        return launch_bp<1, 4, 8, 8>(a, s);
     }
     if (b <= 4) {
         a.fast16 = x16 && b == 4;
-        return launch_bp<4, 4, 4>(a, s);
+        return launch_bp<4, 4, 6, 4>(a, s);
     }
     a.fast16 = x16 && b == 8;
-    return launch_bp<8, 4, 4>(a, s);
+    return launch_bp<8, 4, 6, 4>(a, s);
 }

@@ -27,12 +27,21 @@ def cm():
     return cm
 
 
+def with_ld16(t):
+    """Device copy of a row-major matrix whose rows start on 16-byte boundaries."""
+    rows, cols = t.shape
+    ld = (cols + 3) // 4 * 4
+    buf = torch.zeros((rows, ld), dtype=t.dtype, device=DEV)
+    buf[:, :cols] = t.to(DEV)
+    return buf[:, :cols]
+
+
 def run_coded_gd(cm, A, y, n, k_a, k_at, iters, eta, seed=synth.ERASURE_SEED):
     m, d = A.shape
     cA = cm.Code(n, k_a, m, d, synth.parity_coefficients(n, k_a))
     cAT = cm.Code(n, k_at, d, m, synth.parity_coefficients(n, k_at, seed=synth.CODE_SEED + 1))
-    Ad = A.to(DEV)
-    ATd = Ad.t().contiguous()          # A^T: its row split is the column split of A
+    Ad = with_ld16(A)
+    ATd = with_ld16(A.t())             # A^T: its row split is the column split of A
     PA = cm.encode(cA, Ad)
     PAT = cm.encode(cAT, ATd)
     yd = y.to(DEV)

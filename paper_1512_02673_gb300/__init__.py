@@ -148,7 +148,11 @@ def encode(code: Code, A: torch.Tensor, parity: torch.Tensor | None = None) -> t
     if tuple(A.shape) != (code.m, code.d):
         raise ValueError("A must be m x d")
     if parity is None:
-        parity = torch.empty(((code.n - code.k) * code.L, code.d), dtype=dt, device=A.device)
+        # rows start on 16-byte boundaries (the library's layout contract)
+        per16 = 16 // A.element_size()
+        ldp = (code.d + per16 - 1) // per16 * per16
+        parity = torch.empty(((code.n - code.k) * code.L, ldp), dtype=dt,
+                             device=A.device)[:, :code.d]
     _dev(parity, dt, "parity", 2)
     if tuple(parity.shape) != ((code.n - code.k) * code.L, code.d):
         raise ValueError("parity must be (n-k) L x d")

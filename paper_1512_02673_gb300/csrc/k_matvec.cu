@@ -5,23 +5,31 @@
 // (rows past m are virtual zeros: never read, result 0); worker j >= k reads
 // the parity buffer.
 //
-// Mapping.  A persistent grid (SMs x resident CTAs).  Work unit = a group of
-// R consecutive block rows of one worker, owned by one warp; unit u belongs to
-// worker u % n, so consecutive warps stream different workers and all n
-// workers progress together, as the n workers of the protocol do.  Lane l of
-// a warp reads columns [4l, 4l+4) of every 128-column step of its R rows with
-// 128-bit streaming loads (L1 no-allocate), so each coded element is read
+// Mapping.  A persistent grid (SMs x one resident CTA of 8 warps).  Work
+// unit = a group of R consecutive block rows of one worker, owned by one warp;
+// unit u belongs to worker u % n, so consecutive warps stream different
+// workers and all n workers progress together, as the n workers of the
+// protocol do.  The coded rows stream through a per-warp shared-memory ring
+// of ST steps (R rows x 128 columns) filled by cp.async: lane l copies, and
+// later reads back, only its own 16 bytes [4l, 4l+4) of every row, so a step
+// is complete after cp.async.wait_group alone (no barrier, no spin) and
+// ST-1 steps stay in flight per warp.  Each coded element is read from HBM
 // exactly once.  The CTA's warps sweep the columns in lockstep through chunks
-// of X staged in shared memory by cp.async (double buffered, one barrier per
-// chunk); the smem layout gives every lane its 4 columns x BP vectors with
-// conflict-free 128-bit loads.
+// of X staged by cp.async (double buffered, one barrier per chunk) in a
+// [vector][column] layout, so a lane's 4 columns of one vector are one
+// conflict-free 128-bit load.
 //
-// Precision.  Each lane accumulates R x BP fp32 partials over F steps (4F
-// terms).  Then a transposing butterfly over the 32 lanes (each level sends
-// half of the values, so 32 values cost 31 shuffles) leaves every lane with
-// one complete fp32 partial of 128 F columns, which is added to an fp64
-// accumulator.  Results are fp64: decoding multiplies worker results by the
-// entries of G_S^-1, so an fp32 rounding of them would be amplified.
+// Arithmetic.  Packed fp32x2 FMAs: accumulator pair (r, v) sums the even
+// columns in its low half and the odd columns in its high half, so the pair
+// (A[r][c], A[r][c+1]) straight from the ring multiplies (X[c][v], X[c+1][v])
+// straight from the X layout, with no repacking.
+//
+// Precision.  After F steps (each half holds 2F terms) the halves are added
+// and a transposing butterfly over the 32 lanes (each level sends half of the
+// values, so V values cost V - V/32 shuffles) leaves every lane with complete
+// fp32 partials over 128 F columns, which are added into fp64 accumulators.
+// Results are fp64: decoding multiplies worker results by the entries of
+// G_S^-1, so an fp32 rounding of them would be amplified.
 #include "cm_internal.cuh"
 
 namespace {
@@ -31,13 +39,13 @@ constexpr int kThreads = kWarps * 32;
 
 template <int BP>
 struct XCfg {
-    // columns per staged chunk (about 32 KB of X per buffer)
-    static constexpr int CX = 8192 / BP;
-    // float stride between the smem groups of the BP = 4 / 8 layouts: the
-    // padding makes both the 16-byte cp.async stores and the lane loads hit
-    // distinct bank groups.
-    static constexpr int GS = BP == 1 ? 0 : (BP == 4 ? CX + 8 : CX + 4);
-    static constexpr int FLOATS = BP == 1 ? CX : (BP == 4 ? 4 * GS : 8 * GS);
+    // columns per staged X chunk (16 KB of X per buffer)
+    static constexpr int CX = 4096 / BP;
+    // floats between the [vector] rows of the smem layout: the 4-float pad
+    // makes the staging stores of 32 consecutive (column, vector) elements hit
+    // 32 distinct banks.
+    static constexpr int GS = CX + 4;
+    static constexpr int FLOATS = BP * GS;
 };
 
 struct MatvecArgs {
@@ -74,46 +82,43 @@ __device__ __forceinline__ void cp_async4(float *dst, const float *src, int byte
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
-// Stage columns [c0, c0 + CX) of X into smem buffer xs (zero past d / b).
+// Stage columns [c0, c0 + CX) of X into smem buffer xs as xs[v * GS + col]
+// (zero past d and for padded vectors v >= b).
 template <int BP>
 __device__ __forceinline__ void stage_x(const MatvecArgs &a, float *xs, int64_t c0)
 {
     using C = XCfg<BP>;
     const int tid = threadIdx.x;
     const float *X = a.X;
-    if (a.fast16) {
-        if constexpr (BP == 1) {
-            for (int u = tid; u < C::CX / 4; u += kThreads) {
-                int64_t col = c0 + 4 * u;
-                int64_t left = a.d - col;
-                int bytes = left >= 4 ? 16 : (left > 0 ? (int)left * 4 : 0);
-                cp_async16(xs + 4 * u, bytes ? X + col : X, bytes);
-            }
-        } else {
-            constexpr int H = BP / 4;
-            for (int u = tid; u < C::CX * H; u += kThreads) {
-                int col = u / H, h = u % H;
-                int g = (col & 3) * H + h;
-                int64_t gc = c0 + col;
-                bool in = gc < a.d;
-                cp_async16(xs + g * C::GS + (col >> 2) * 4,
-                           in ? X + gc * BP + 4 * h : X, in ? 16 : 0);
-            }
+    if (BP == 1 && a.fast16) {
+        for (int u = tid; u < C::CX / 4; u += kThreads) {
+            const int64_t col = c0 + 4 * u;
+            const int64_t left = a.d - col;
+            const int bytes = left >= 4 ? 16 : (left > 0 ? (int)left * 4 : 0);
+            cp_async16(xs + 4 * u, bytes ? X + col : a.A, bytes);
         }
     } else {
         for (int e = tid; e < C::CX * BP; e += kThreads) {
-            int col = e / BP, v = e % BP;
-            int64_t gc = c0 + col;
-            bool in = gc < a.d && v < a.b;
-            int dst;
-            if constexpr (BP == 1)
-                dst = col;
-            else
-                dst = ((col & 3) * (BP / 4) + (v >> 2)) * C::GS + (col >> 2) * 4 + (v & 3);
-            cp_async4(xs + dst, in ? X + gc * a.b + v : X, in ? 4 : 0);
+            const int col = e / BP, v = e % BP;
+            const int64_t gc = c0 + col;
+            const bool in = gc < a.d && v < a.b;
+            cp_async4(xs + v * C::GS + col, in ? X + gc * a.b + v : X, in ? 4 : 0);
         }
     }
     cp_async_commit();
+}
+
+__device__ __forceinline__ uint64_t pack2(float lo, float hi)
+{
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};\n" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+// d += a * b on both fp32 halves (round to nearest, no flush to zero)
+__device__ __forceinline__ void fma2(uint64_t &d, uint64_t a, uint64_t b)
+{
+    asm("fma.rn.f32x2 %0, %1, %2, %0;\n" : "+l"(d) : "l"(a), "l"(b));
 }
 
 // Transposing butterfly: V fp32 values per lane -> max(1, V/32) complete sums
@@ -188,6 +193,21 @@ __device__ __forceinline__ void unit_rows(const MatvecArgs &a, int64_t g, const 
 // cp.async: lane l copies, and later reads back, only its own 16 bytes of
 // every row, so completion needs just cp.async.wait_group (no barrier, no
 // spin).  ST-1 steps are in flight per warp while the warp computes.
+template <int V>
+__device__ __forceinline__ void flush_pairs(uint64_t (&acc)[V],
+                                            double (&acc64)[V >= 32 ? V / 32 : 1], int lane)
+{
+    float t[V];
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+        float lo, hi;
+        asm("mov.b64 {%0, %1}, %2;\n" : "=f"(lo), "=f"(hi) : "l"(acc[i]));
+        t[i] = lo + hi;
+        acc[i] = 0ull;
+    }
+    flush<V>(t, acc64, lane);
+}
+
 template <int BP, int R, int ST, int F>
 __global__ void __launch_bounds__(kThreads, 1)
 matvec_kernel(const MatvecArgs a)
@@ -197,6 +217,7 @@ matvec_kernel(const MatvecArgs a)
     constexpr int NH = V >= 32 ? V / 32 : 1;
     constexpr int IPC = C::CX / 128;   // steps per X chunk
     static_assert(ST >= 2 && ST <= 8, "ring depth");
+    static_assert(IPC >= ST - 1, "an X chunk must outlast the ring");
     extern __shared__ __align__(16) float smem[];
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
@@ -252,7 +273,7 @@ matvec_kernel(const MatvecArgs a)
     int slot = 0, fl = 0, j = 0;
     int64_t rr0 = 0;
     bool has = false;
-    float acc[V];
+    uint64_t acc[V];   // packed (even-column, odd-column) partial pairs
     double acc64[NH];
 #pragma unroll 1
     for (int64_t f = 0; f < total; ++f) {
@@ -262,7 +283,7 @@ matvec_kernel(const MatvecArgs a)
             const float *dummy[R];
             unit_rows<R>(a, g, dummy, j, rr0);
 #pragma unroll
-            for (int i = 0; i < V; ++i) acc[i] = 0.f;
+            for (int i = 0; i < V; ++i) acc[i] = 0ull;
 #pragma unroll
             for (int i = 0; i < NH; ++i) acc64[i] = 0.0;
             fl = 0;
@@ -284,40 +305,27 @@ matvec_kernel(const MatvecArgs a)
             cp_async_wait_upto(ST - 1);
         }
         if (has) {
-            const float *xb = smem + (xseq & 1) * C::FLOATS;
+            const float *xb = smem + (xseq & 1) * C::FLOATS + 4 * ((int)cs * 32 + lane);
             const float *ab = ring + slot * (R * 128) + 4 * lane;
-            const int c4 = (int)cs * 32 + lane;
-            float4 av[R];
+            uint64_t x01[BP], x23[BP];
 #pragma unroll
-            for (int r = 0; r < R; ++r) av[r] = *reinterpret_cast<const float4 *>(ab + r * 128);
+            for (int v = 0; v < BP; ++v) {
+                const float4 xv = *reinterpret_cast<const float4 *>(xb + v * C::GS);
+                x01[v] = pack2(xv.x, xv.y);
+                x23[v] = pack2(xv.z, xv.w);
+            }
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                float x[BP];
-                if constexpr (BP == 1) {
-                    const float4 xv = *reinterpret_cast<const float4 *>(xb + 4 * c4);
-                    x[0] = q == 0 ? xv.x : q == 1 ? xv.y : q == 2 ? xv.z : xv.w;
-                } else {
+            for (int r = 0; r < R; ++r) {
+                const float4 av = *reinterpret_cast<const float4 *>(ab + r * 128);
+                const uint64_t a01 = pack2(av.x, av.y), a23 = pack2(av.z, av.w);
 #pragma unroll
-                    for (int h = 0; h < BP / 4; ++h) {
-                        const float4 xv = *reinterpret_cast<const float4 *>(
-                            xb + (q * (BP / 4) + h) * C::GS + 4 * c4);
-                        x[4 * h + 0] = xv.x;
-                        x[4 * h + 1] = xv.y;
-                        x[4 * h + 2] = xv.z;
-                        x[4 * h + 3] = xv.w;
-                    }
-                }
-#pragma unroll
-                for (int r = 0; r < R; ++r) {
-                    const float aq = q == 0 ? av[r].x : q == 1 ? av[r].y
-                                   : q == 2 ? av[r].z : av[r].w;
-#pragma unroll
-                    for (int v = 0; v < BP; ++v)
-                        acc[r * BP + v] = fmaf(aq, x[v], acc[r * BP + v]);
+                for (int v = 0; v < BP; ++v) {
+                    fma2(acc[r * BP + v], a01, x01[v]);
+                    fma2(acc[r * BP + v], a23, x23[v]);
                 }
             }
             if (++fl == F) {
-                flush<V>(acc, acc64, lane);
+                flush_pairs<V>(acc, acc64, lane);
                 fl = 0;
             }
         }
@@ -326,7 +334,7 @@ matvec_kernel(const MatvecArgs a)
         if (chunk_end) ++xseq;
         if (s == steps - 1) {
             if (has) {
-                if (fl) flush<V>(acc, acc64, lane);
+                if (fl) flush_pairs<V>(acc, acc64, lane);
                 const int64_t base = (int64_t)j * a.L + rr0;
                 if constexpr (V >= 32) {
 #pragma unroll
@@ -398,12 +406,9 @@ cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, con
     const bool x16 = ((uintptr_t)X & 15u) == 0;
     if (b == 1) {
         a.fast16 = x16;
-        return launch_bp<1, 4, 8, 8>(a, s);
+        return launch_bp<1, 4, 8, 16>(a, s);
     }
-    if (b <= 4) {
-        a.fast16 = x16 && b == 4;
-        return launch_bp<4, 4, 6, 4>(a, s);
-    }
-    a.fast16 = x16 && b == 8;
-    return launch_bp<8, 4, 6, 4>(a, s);
+    a.fast16 = 0;
+    if (b <= 4) return launch_bp<4, 8, 5, 16>(a, s);
+    return launch_bp<8, 8, 5, 16>(a, s);
 }

@@ -1,0 +1,453 @@
+#!/usr/bin/env python3
+"""Benchmark of the MDS-coded matrix-multiplication hot path on GB300.
+
+Default workload: (32,24) coded mat-multi-vec, A 65536 x 65536 fp32 (16 GiB),
+a batch of 8 vectors.  One step = the whole coded pass over one batch:
+encode A into its 8 parity blocks, draw the straggler set (shifted
+exponential), compute all 32 worker products, decode A X from the 24
+survivors.  `value` is the step's algorithmic HBM bytes divided by the step
+time (GB/s); per-kernel times, the encode+decode latency, the roofline of the
+dominant kernel (the worker products) and the oracle's CPU baseline ride along
+on the same JSON line.  Coded gradient descent (40000 x 8000, (20,10) codes)
+is measured as a secondary workload on the same line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With N > 1 (launched by torch.distributed.run) every rank runs the same
+workload on its own GPU (independent replicas, weak scaling, no collective on
+the data path); `value` sums the ranks' bytes over the slowest rank's time.
+`--impl reference` times the CPU oracle on a bounded sample of the same
+workload (rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = ("coded matvec effective HBM GB/s (% of GB300 peak); "
+          "encode+decode latency µs")
+CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+REASON_NAMES = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+
+
+# ---- algorithmic traffic (bytes that the step must move at minimum) ---------------
+
+def step_bytes(w: synth.Workload, L: int, m: int | None = None) -> dict:
+    """Algorithmic HBM bytes of one step of a mat-multi-vec workload.
+
+    encode: read the m x d data rows once, write (n-k) L x d parity.
+    worker products: read every coded element once (m d systematic + (n-k) L d
+    parity), read X, write the n L x b fp64 results.
+    decode: read the k L x b surviving fp64 results, write m x b fp32."""
+    m = w.m if m is None else m
+    par = (w.n - w.k) * L * w.d * 4
+    enc = m * w.d * 4 + par
+    mv = m * w.d * 4 + par + w.d * w.b * 4 + w.n * L * w.b * 8
+    dec = w.k * L * w.b * 8 + m * w.b * 4
+    return {"encode": enc, "matvec": mv, "decode": dec, "step": enc + mv + dec}
+
+
+def gd_iter_bytes(w: synth.GDWorkload, LA: int, LAT: int) -> int:
+    """Per iteration: both coded products (all coded elements once) and decodes."""
+    a = w.m * w.d * 4 + (w.n - w.k_a) * LA * w.d * 4 + w.d * 4 + w.n * LA * 8
+    at = w.d * w.m * 4 + (w.n - w.k_at) * LAT * w.m * 4 + w.m * 4 + w.n * LAT * 8
+    dec = w.k_a * LA * 8 + 2 * w.m * 4 + w.k_at * LAT * 8 + 2 * w.d * 4
+    return a + at + dec
+
+
+# ---- helpers -----------------------------------------------------------------------------
+
+def measured_peaks() -> dict:
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "source": "measured",
+                "bf16_tflops": float(p.get("bf16_tflops", 1900.0)),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", 1700.0))}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def recorded_traffic(kernel: str, source_file: str):
+    """dram bytes per launch recorded from an ncu capture, if the kernel source
+    has not changed since (profiles/traffic.txt: kernel sha256 bytes note)."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    sha = hashlib.sha256(open(source_file, "rb").read()).hexdigest()
+    for line in open(path):
+        parts = line.split()
+        if len(parts) >= 3 and not line.startswith("#") and parts[0] == kernel:
+            if parts[1] == sha:
+                return float(parts[2])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason sampling during a timed region."""
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + CLOCK_FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.15)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.1)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self) -> dict:
+        sms, maxs, reasons = [], [], set()
+        try:
+            for line in open(self.path):
+                f = [x.strip() for x in line.split(",")]
+                if len(f) < 9:
+                    continue
+                try:
+                    sms.append(float(f[1]))
+                    maxs.append(float(f[2]))
+                except ValueError:
+                    continue
+                for name, val in zip(REASON_NAMES, f[5:9]):
+                    if val.lower().startswith("active"):
+                        reasons.add(name)
+            os.unlink(self.path)
+        except Exception:
+            pass
+        if not sms:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": float(np.median(sms)), "sm_max_mhz": float(max(maxs)),
+                "reasons": sorted(reasons), "samples": len(sms)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    return world, rank, local
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---- CPU oracle on a bounded sample (the baseline / reference arm) ---------------------
+
+def oracle_sample_step(w: synth.Workload, s: int, seed: int, counter: int):
+    """One step of the oracle on s sampled block rows of workload w: the
+    sub-problem whose k blocks are s rows each (same n, k, d, b).  Returns
+    (seconds, algorithmic bytes of the sample in the GPU's units)."""
+    import oracle
+    P = synth.parity_coefficients(w.n, w.k).astype(np.float64)
+    A_sub = synth.gaussian((w.k * s, w.d), seed).numpy()
+    X = synth.gaussian((w.d, w.b), seed + 1).numpy()
+    t0 = time.perf_counter()
+    par = oracle.encode(w.n, w.k, A_sub, P)
+    Yt = oracle.worker_outputs_f64(w.n, w.k, A_sub, par, X)
+    mask, _ = oracle.draw_erasures(synth.ERASURE_SEED, counter, w.n, w.k)
+    oracle.decode(w.n, w.k, w.k * s, P, mask, Yt)
+    dt = time.perf_counter() - t0
+    return dt, step_bytes(w, s, m=w.k * s)["step"]
+
+
+def cpu_baseline(w: synth.Workload, target_s: float = 12.0) -> dict:
+    import oracle
+    oracle.build()
+    s = 4
+    dt, nb = oracle_sample_step(w, s, 77, 0)
+    s = int(max(4, min(w.L, s * target_s / max(dt, 1e-3) * 0.8)))
+    dt, nb = oracle_sample_step(w, s, 78, 1)
+    return {"value": nb / dt / 1e9, "unit": "GB/s", "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": "%d of %d block rows of every worker (%.1f%% of the step), one step, "
+                      "%.1f s" % (s, w.L, 100.0 * s / w.L, dt)}
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    w = synth.BANDWIDTH
+    s = 16
+    for i in range(args.warmup):
+        oracle_sample_step(w, s, 90 + i, i)
+    tot, nb = 0.0, 0
+    for i in range(args.steps):
+        dt, b = oracle_sample_step(w, s, 200 + i, args.warmup + i)
+        tot += dt
+        nb += b
+    value = nb / tot / 1e9
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": tot / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_of(w),
+        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": oracle.num_threads(),
+                         "kind": "oracle",
+                         "sample": "%d of %d block rows of every worker per step" % (s, w.L)},
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# A reduced copy of the bandwidth workload for ncu captures: same code and
+# batch, inputs still larger than L2 (512 MB), a few GB on the device at most.
+PROFILE = synth.Workload("coded mat-multi-vec (32,24) 8192x16384 b=8 (profiling case)",
+                         m=8192, d=16384, b=8, n=32, k=24, data_device="cuda")
+WORKLOADS = {"bandwidth": synth.BANDWIDTH, "profile": PROFILE}
+
+
+def config_of(w: synth.Workload) -> dict:
+    return {"workload": w.name, "n": w.n, "k": w.k, "m": w.m, "d": w.d, "b": w.b,
+            "L": w.L, "dtype": w.dtype,
+            "step": "encode + straggler draw + all n worker products + decode",
+            "l2": "inputs larger than L2 (A is 16 GiB, parity 5.7 GB); no flush needed",
+            "seeds": {"data": synth.DATA_SEED, "code": synth.CODE_SEED,
+                      "erasure": synth.ERASURE_SEED}}
+
+
+# ---- the GPU arm ---------------------------------------------------------------------------
+
+def run_ours(args, world, rank, local):
+    import paper_1512_02673_gb300 as cm
+
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    w = WORKLOADS[args.workload]
+    full = args.workload == "bandwidth"
+    P = synth.parity_coefficients(w.n, w.k)
+    code = cm.Code(w.n, w.k, w.m, w.d, P)
+    L = code.L
+    A, X = synth.matvec_inputs(w, device=dev)
+    parity = torch.empty(((w.n - w.k) * L, w.d), device=dev)
+    Yt = torch.empty((w.n * L, w.b), dtype=torch.float64, device=dev)
+    Y = torch.empty((w.m, w.b), device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    nbytes = step_bytes(w, L)
+    stream = torch.cuda.current_stream()
+
+    def step(counter, ev=None):
+        if ev:
+            ev[0].record(stream)
+        cm.encode(code, A, parity)
+        if ev:
+            ev[1].record(stream)
+        mask, _ = cm.draw_erasures(synth.ERASURE_SEED, counter, w.n, w.k)
+        cm.matvec(code, A, parity, X, Yt)
+        if ev:
+            ev[2].record(stream)
+        cm.decode(code, Yt, mask, Y=Y, status=status)
+        if ev:
+            ev[3].record(stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t_start.record(stream)
+        for i in range(args.steps):
+            step(args.warmup + i, evs[i])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms_local = t_start.elapsed_time(t_end)
+    if int(status.item()) != 0:
+        raise RuntimeError("device status %d during the timed steps" % int(status.item()))
+    ms = max_over_ranks(ms_local, world)
+    per = {"encode": [], "matvec": [], "decode": []}
+    for e in evs:
+        per["encode"].append(e[0].elapsed_time(e[1]))
+        per["matvec"].append(e[1].elapsed_time(e[2]))
+        per["decode"].append(e[2].elapsed_time(e[3]))
+    avg = {k: float(np.mean(v)) for k, v in per.items()}
+    launches_per_step = math.ceil((w.n - w.k) / 8) + 2
+
+    if not full:   # profiling case: kernels only
+        if rank == 0:
+            print(json.dumps({"workload": w.name, "ms_per_step": ms / args.steps,
+                              "kernels_us": {k: v * 1e3 for k, v in avg.items()}}), flush=True)
+        return
+
+    # end to end through the public API with host buffers: pinned X in, Y out
+    Xh = X.cpu().pin_memory()
+    Yh = torch.empty((w.m, w.b), pin_memory=True)
+    for i in range(2):
+        X.copy_(Xh, non_blocking=True)
+        step(1000 + i)
+        Yh.copy_(Y, non_blocking=True)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for i in range(args.steps):
+        X.copy_(Xh, non_blocking=True)
+        step(2000 + i)
+        Yh.copy_(Y, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+
+    # secondary: coded gradient descent (40000 x 8000, (20,10) codes)
+    del A, parity
+    torch.cuda.empty_cache()
+    gd = bench_gd(cm, dev, args.steps)
+
+    peaks = measured_peaks()
+    achieved = nbytes["matvec"] / (avg["matvec"] * 1e-3) / 1e9
+    traffic = recorded_traffic("matvec",
+                               os.path.join(ROOT, "paper_1512_02673_gb300", "csrc", "k_matvec.cu"))
+    value = world * nbytes["step"] * args.steps / (ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic", "config": config_of(w),
+        "pct_of_peak": 100.0 * value / world / peaks["hbm_gbs"],
+        "encode_decode_latency_us": {"encode": avg["encode"] * 1e3,
+                                     "decode": avg["decode"] * 1e3,
+                                     "sum": (avg["encode"] + avg["decode"]) * 1e3},
+        "kernels": {
+            "encode": {"us": avg["encode"] * 1e3,
+                       "gbs": nbytes["encode"] / (avg["encode"] * 1e-3) / 1e9},
+            "matvec": {"us": avg["matvec"] * 1e3, "gbs": achieved},
+            "decode": {"us": avg["decode"] * 1e3,
+                       "gbs": nbytes["decode"] / (avg["decode"] * 1e-3) / 1e9},
+        },
+        "roofline": {"bound": "hbm", "kernel": "matvec (all n worker products)",
+                     "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / peaks["hbm_gbs"], "traffic": traffic,
+                     "algorithmic_bytes_per_launch": nbytes["matvec"],
+                     "peak_source": peaks["source"]},
+        "e2e": {"value": world * nbytes["step"] * args.steps / (e2e_ms * 1e-3) / 1e9,
+                "unit": "GB/s", "h2d_bytes_per_step": w.d * w.b * 4,
+                "d2h_bytes_per_step": w.m * w.b * 4},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk.summary(),
+        "secondary": {"gd": gd},
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def bench_gd(cm, dev, steps: int) -> dict:
+    """Coded GD on the 40000 x 8000 regression: seconds per iteration (4
+    launches: two coded products, two fused decodes), effective GB/s."""
+    w = synth.GD
+    A, _, y = synth.regression_inputs(w, device=dev)
+    AT = A.t().contiguous()
+    cA = cm.Code(w.n, w.k_a, w.m, w.d, synth.parity_coefficients(w.n, w.k_a))
+    cAT = cm.Code(w.n, w.k_at, w.d, w.m,
+                  synth.parity_coefficients(w.n, w.k_at, seed=synth.CODE_SEED + 1))
+    PA = cm.encode(cA, A)
+    PAT = cm.encode(cAT, AT)
+    x = torch.zeros(w.d, device=dev)
+    ws = torch.empty(cm.gd_workspace_bytes(cA, cAT), dtype=torch.uint8, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    masks = [(cm.draw_erasures(synth.ERASURE_SEED, 2 * t, w.n, w.k_a)[0],
+              cm.draw_erasures(synth.ERASURE_SEED, 2 * t + 1, w.n, w.k_at)[0])
+             for t in range(w.iters)]
+    for t in range(3):
+        cm.gd_step(cA, A, PA, cAT, AT, PAT, y, x, w.eta, masks[t][0], masks[t][1], ws, status)
+    x.zero_()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for t in range(w.iters):
+        cm.gd_step(cA, A, PA, cAT, AT, PAT, y, x, w.eta, masks[t][0], masks[t][1], ws, status)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / w.iters
+    nb = gd_iter_bytes(w, cA.L, cAT.L)
+    return {"workload": w.name, "iters": w.iters, "ms_per_iter": ms,
+            "gbs": nb / (ms * 1e-3) / 1e9, "launches_per_iter": 4,
+            "status": int(status.item())}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=40)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=["bandwidth", "profile"], default="bandwidth",
+                    help="profile: a 512 MB case of the same path, for ncu captures")
+    ap.add_argument("--no-cpu-baseline", action="store_true",
+                    help="skip the oracle timing on the host cores")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        world = int(os.environ.get("WORLD_SIZE", "1"))
+        rank = int(os.environ.get("RANK", "0"))
+        run_reference(args, world, rank)
+        return
+    world, rank, local = dist_setup()
+    try:
+        run_ours(args, world, rank, local)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -243,9 +243,10 @@ def run_reference(args, world, rank):
 
 
 # A reduced copy of the bandwidth workload for ncu captures: same code and
-# batch, inputs still larger than L2 (512 MB), a few GB on the device at most.
-PROFILE = synth.Workload("coded mat-multi-vec (32,24) 8192x16384 b=8 (profiling case)",
-                         m=8192, d=16384, b=8, n=32, k=24, data_device="cuda")
+# batch, inputs still larger than L2 (0.96 GB of A), a few GB on the device at
+# most; L = 608 gives the 152-SM grid exactly two rounds of 8-row units.
+PROFILE = synth.Workload("coded mat-multi-vec (32,24) 14592x16384 b=8 (profiling case)",
+                         m=14592, d=16384, b=8, n=32, k=24, data_device="cuda")
 WORKLOADS = {"bandwidth": synth.BANDWIDTH, "profile": PROFILE}
 
 
@@ -285,7 +286,7 @@ def run_ours(args, world, rank, local):
         if ev:
             ev[1].record(stream)
         mask, _ = cm.draw_erasures(synth.ERASURE_SEED, counter, w.n, w.k)
-        cm.matvec(code, A, parity, X, Yt)
+        cm.matvec(code, A, parity, X, Yt, status=status)
         if ev:
             ev[2].record(stream)
         cm.decode(code, Yt, mask, Y=Y, status=status)

@@ -87,10 +87,12 @@ cm_status cm_encode(const cm_code *code, const void *A, int64_t lda,
  * all workers concurrently.  fp32 code only.  X is d x b fp32 (row-major,
  * vectors contiguous per row), 1 <= b <= 8.  Yt is n L x b fp64: each sum is
  * formed from short fp32 partial sums combined in fp64, so decoding does not
- * amplify an fp32 rounding of the results. */
+ * amplify an fp32 rounding of the results.  A bounded wait inside the kernel
+ * that gives up writes CM_ETIMEOUT to *dev_status (nullable); Yt is then
+ * incomplete. */
 cm_status cm_matvec(const cm_code *code, const float *A, int64_t lda,
                     const float *parity, int64_t ldp, const float *X, int32_t b,
-                    double *Yt, cm_stream_t stream);
+                    double *Yt, int32_t *dev_status, cm_stream_t stream);
 
 /* Straggler draw (Sec. III-C, III-D; eq. for the MDS runtime).  Host only.
  * Worker j's time in round `counter` is T_j = (shift + E_j / rate) / k with

@@ -55,7 +55,7 @@ def lib() -> ctypes.CDLL:
             "cm_code_destroy": (None, [vp]),
             "cm_block_rows": (i64, [vp]),
             "cm_encode": (st, [vp, vp, i64, vp, i64, vp]),
-            "cm_matvec": (st, [vp, vp, i64, vp, i64, vp, i32, vp, vp]),
+            "cm_matvec": (st, [vp, vp, i64, vp, i64, vp, i32, vp, vp, vp]),
             "cm_draw_erasures": (st, [u64, u64, i32, i32, f64, f64, ctypes.POINTER(u32), vp]),
             "cm_decode": (st, [vp, vp, u32, i32, vp, vp, vp]),
             "cm_gd_workspace_bytes": (sz, [vp, vp]),
@@ -162,7 +162,7 @@ def encode(code: Code, A: torch.Tensor, parity: torch.Tensor | None = None) -> t
 
 
 def matvec(code: Code, A: torch.Tensor, parity: torch.Tensor, X: torch.Tensor,
-           Yt: torch.Tensor | None = None) -> torch.Tensor:
+           Yt: torch.Tensor | None = None, status: torch.Tensor | None = None) -> torch.Tensor:
     """All n worker products Yt (n L x b, fp64) for X (d x b fp32, b <= 8)."""
     _dev(A, torch.float32, "A", 2)
     _dev(parity, torch.float32, "parity", 2)
@@ -179,9 +179,13 @@ def matvec(code: Code, A: torch.Tensor, parity: torch.Tensor, X: torch.Tensor,
     _contig(Yt, "Yt")
     if tuple(Yt.shape) != (code.n * code.L, b):
         raise ValueError("Yt must be n L x b")
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
     _check(lib().cm_matvec(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
-                           _ld(parity, "parity"), X.data_ptr(), b, Yt.data_ptr(), _stream()),
-           "cm_matvec")
+                           _ld(parity, "parity"), X.data_ptr(), b, Yt.data_ptr(), sp,
+                           _stream()), "cm_matvec")
     return Yt
 
 

@@ -99,12 +99,12 @@ def test_synchronous_checks_precede_any_launch(cm):
     # survivor bit at or above n
     assert L.cm_decode(c.handle, fake, 0b1000111, 1, fake, None, None) == cm.CM_EINVAL
     # b out of range, misaligned operands, bad leading dimension
-    assert L.cm_matvec(c.handle, fake, 500, fake, 500, fake, 9, fake, None) == cm.CM_EINVAL
-    assert L.cm_matvec(c.handle, fake, 500, fake, 500, fake, 0, fake, None) == cm.CM_EINVAL
+    assert L.cm_matvec(c.handle, fake, 500, fake, 500, fake, 9, fake, None, None) == cm.CM_EINVAL
+    assert L.cm_matvec(c.handle, fake, 500, fake, 500, fake, 0, fake, None, None) == cm.CM_EINVAL
     odd = ctypes.c_void_p((1 << 20) + 4)
-    assert L.cm_matvec(c.handle, odd, 500, fake, 500, fake, 1, fake, None) == cm.CM_EINVAL
-    assert L.cm_matvec(c.handle, fake, 501, fake, 500, fake, 1, fake, None) == cm.CM_EINVAL
-    assert L.cm_matvec(c.handle, fake, 496, fake, 500, fake, 1, fake, None) == cm.CM_EINVAL
+    assert L.cm_matvec(c.handle, odd, 500, fake, 500, fake, 1, fake, None, None) == cm.CM_EINVAL
+    assert L.cm_matvec(c.handle, fake, 501, fake, 500, fake, 1, fake, None, None) == cm.CM_EINVAL
+    assert L.cm_matvec(c.handle, fake, 496, fake, 500, fake, 1, fake, None, None) == cm.CM_EINVAL
     assert L.cm_encode(c.handle, fake, 502, fake, 500, None) == cm.CM_EINVAL
     assert L.cm_encode(None, fake, 500, fake, 500, None) == cm.CM_EINVAL
     # f32 code refuses the bf16-only tensor-core path
@@ -113,7 +113,7 @@ def test_synchronous_checks_precede_any_launch(cm):
     cb = cm.Code(6, 3, 120, 64, synth.parity_coefficients(6, 3), dtype="bf16")
     assert L.cm_coded_gemm(cb.handle, fake, 64, fake, 64, fake, 64, 24, fake, 24,
                            None) == cm.CM_EINVAL          # N % 16 != 0
-    assert L.cm_matvec(cb.handle, fake, 64, fake, 64, fake, 1, fake, None) == cm.CM_EINVAL
+    assert L.cm_matvec(cb.handle, fake, 64, fake, 64, fake, 1, fake, None, None) == cm.CM_EINVAL
 
 
 def test_gd_workspace_and_checks(cm):

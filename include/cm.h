@@ -144,6 +144,31 @@ cm_status cm_gd_step(const cm_code *code_A, const float *A, int64_t lda,
                      void *ws, size_t ws_bytes, int32_t *dev_status,
                      cm_stream_t stream);
 
+/* Size of the fixed device scratch array behind cm_gd_step_noalloc: 4 MiB. */
+#define CM_GD_STATIC_SCRATCH_BYTES (4u << 20)
+
+/* cm_gd_step without a caller workspace (the paper has no counterpart: this
+ * is a service for callers that cannot allocate device memory, e.g. a
+ * plug-in inside an application that owns all device memory through its own
+ * pool, or a loop that must not call cudaMalloc / cudaFree because they can
+ * synchronize the device).  Same arguments and result as cm_gd_step minus
+ * ws / ws_bytes; the workspace is a file-scope device array of
+ * CM_GD_STATIC_SCRATCH_BYTES held by every GPU that loads the library until
+ * the process exits.  The call allocates nothing.  Returns CM_ENOMEM when
+ * cm_gd_workspace_bytes(code_A, code_AT) exceeds the array.  The first call
+ * on a device looks up the array's device address (once per device, with
+ * that device current); make that first call before any stream capture.
+ * All calls on a device share the array and it keeps the last call's
+ * contents (nothing in it needs to start at zero); calls whose kernels
+ * overlap on the GPU race on it. */
+cm_status cm_gd_step_noalloc(const cm_code *code_A, const float *A, int64_t lda,
+                             const float *PA, int64_t ldpa,
+                             const cm_code *code_AT, const float *AT, int64_t ldat,
+                             const float *PAT, int64_t ldpat,
+                             const float *y, float *x, float eta,
+                             uint32_t surv_A, uint32_t surv_AT, int32_t *dev_status,
+                             cm_stream_t stream);
+
 /* Coded matrix-matrix products (the s-column X of the Sec. I-A example) on
  * tensor cores: Ct[j L + r][c] = sum_t A~_j[r][t] B[t][c] for all n workers,
  * bf16 inputs, fp32 accumulation, fp32 output.  bf16 code only.  B is passed

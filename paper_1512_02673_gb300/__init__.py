@@ -61,6 +61,8 @@ def lib() -> ctypes.CDLL:
             "cm_gd_workspace_bytes": (sz, [vp, vp]),
             "cm_gd_step": (st, [vp, vp, i64, vp, i64, vp, vp, i64, vp, i64, vp, vp, f32,
                                 u32, u32, vp, sz, vp, vp]),
+            "cm_gd_step_noalloc": (st, [vp, vp, i64, vp, i64, vp, vp, i64, vp, i64, vp, vp,
+                                        f32, u32, u32, vp, vp]),
             "cm_coded_gemm": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, vp]),
             "cm_decode_mat": (st, [vp, vp, i64, u32, i32, vp, i64, vp, vp]),
             "cm_matmat": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, u32, vp, i64,
@@ -241,6 +243,36 @@ def gd_step(code_A: Code, A, PA, code_AT: Code, AT, PAT, y, x, eta: float, surv_
                             PAT.data_ptr(), _ld(PAT, "PAT"), y.data_ptr(), x.data_ptr(),
                             eta, surv_A, surv_AT, ws.data_ptr(), ws.numel(), sp, _stream()),
            "cm_gd_step")
+    return x
+
+
+# Size of the fixed device scratch array behind gd_step_noalloc (bytes).
+GD_STATIC_SCRATCH_BYTES = 4 << 20
+
+
+def gd_step_noalloc(code_A: Code, A, PA, code_AT: Code, AT, PAT, y, x, eta: float,
+                    surv_A: int, surv_AT: int, status: torch.Tensor | None = None):
+    """gd_step for callers that cannot allocate device memory.
+
+    Uses the library's fixed device scratch array (GD_STATIC_SCRATCH_BYTES,
+    shared by all calls on a device) instead of a workspace argument, and
+    allocates nothing.  Problems whose workspace would exceed the array raise
+    CodedError(CM_ENOMEM).  Calls that overlap on the GPU race on the array."""
+    for t, name in ((A, "A"), (PA, "PA"), (AT, "AT"), (PAT, "PAT")):
+        _dev(t, torch.float32, name, 2)
+    _dev(y, torch.float32, "y")
+    _dev(x, torch.float32, "x")
+    _contig(x, "x")
+    _contig(y, "y")
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
+    _check(lib().cm_gd_step_noalloc(code_A.handle, A.data_ptr(), _ld(A, "A"), PA.data_ptr(),
+                                    _ld(PA, "PA"), code_AT.handle, AT.data_ptr(),
+                                    _ld(AT, "AT"), PAT.data_ptr(), _ld(PAT, "PAT"),
+                                    y.data_ptr(), x.data_ptr(), eta, surv_A, surv_AT, sp,
+                                    _stream()), "cm_gd_step_noalloc")
     return x
 
 

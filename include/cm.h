@@ -171,14 +171,16 @@ cm_status cm_gd_step_noalloc(const cm_code *code_A, const float *A, int64_t lda,
 
 /* Coded matrix-matrix products (the s-column X of the Sec. I-A example) on
  * tensor cores: Ct[j L + r][c] = sum_t A~_j[r][t] B[t][c] for all n workers,
- * bf16 inputs, fp32 accumulation, fp32 output.  bf16 code only.  B is passed
- * transposed: Bt is N x d bf16 (row-major, leading dimension ldb), i.e. each
- * column of B contiguous.  Ct is n L x N fp32 with leading dimension ldc.
- * Requires d % 8 == 0 and N % 16 == 0 (the tile grid of the tensor-core
- * path), N >= 16. */
+ * bf16 inputs, fp32 accumulation in tensor memory, fp32 output.  bf16 code
+ * only.  B is passed transposed: Bt is N x d bf16 (row-major, leading
+ * dimension ldb), i.e. each column of B contiguous.  Ct is n L x N fp32 with
+ * leading dimension ldc (16-byte aligned base).  Any N >= 1 (the ragged last
+ * column tile and K tail read zeros).  A bounded wait that gives up writes
+ * CM_ETIMEOUT to *dev_status (nullable). */
 cm_status cm_coded_gemm(const cm_code *code, const void *A, int64_t lda,
                         const void *parity, int64_t ldp, const void *Bt, int64_t ldb,
-                        int32_t N, float *Ct, int64_t ldc, cm_stream_t stream);
+                        int32_t N, float *Ct, int64_t ldc, int32_t *dev_status,
+                        cm_stream_t stream);
 
 /* Decoding of matrix results: as cm_decode with b = N columns of fp32
  * stacked results Ct (leading dimension ldc) into C (m x N fp32, leading

@@ -63,7 +63,7 @@ def lib() -> ctypes.CDLL:
                                 u32, u32, vp, sz, vp, vp]),
             "cm_gd_step_noalloc": (st, [vp, vp, i64, vp, i64, vp, vp, i64, vp, i64, vp, vp,
                                         f32, u32, u32, vp, vp]),
-            "cm_coded_gemm": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, vp]),
+            "cm_coded_gemm": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, vp, vp]),
             "cm_decode_mat": (st, [vp, vp, i64, u32, i32, vp, i64, vp, vp]),
             "cm_matmat": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, u32, vp, i64,
                                vp, vp]),
@@ -276,7 +276,7 @@ def gd_step_noalloc(code_A: Code, A, PA, code_AT: Code, AT, PAT, y, x, eta: floa
     return x
 
 
-def coded_gemm(code: Code, A, parity, Bt, Ct=None) -> torch.Tensor:
+def coded_gemm(code: Code, A, parity, Bt, Ct=None, status=None) -> torch.Tensor:
     """All n worker products Ct = A~ B (n L x N fp32) on tensor cores.
 
     Bt is B transposed: N x d bf16 (each column of B contiguous)."""
@@ -286,9 +286,13 @@ def coded_gemm(code: Code, A, parity, Bt, Ct=None) -> torch.Tensor:
     if Ct is None:
         Ct = torch.empty((code.n * code.L, N), dtype=torch.float32, device=A.device)
     _dev(Ct, torch.float32, "Ct", 2)
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
     _check(lib().cm_coded_gemm(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
                                _ld(parity, "parity"), Bt.data_ptr(), _ld(Bt, "Bt"), N,
-                               Ct.data_ptr(), _ld(Ct, "Ct"), _stream()), "cm_coded_gemm")
+                               Ct.data_ptr(), _ld(Ct, "Ct"), sp, _stream()), "cm_coded_gemm")
     return Ct
 
 

@@ -172,17 +172,17 @@ cm_status cm_gd_step(const cm_code *cA, const float *A, int64_t lda, const float
 
 cm_status cm_coded_gemm(const cm_code *c, const void *A, int64_t lda, const void *par,
                         int64_t ldp, const void *Bt, int64_t ldb, int32_t N, float *Ct,
-                        int64_t ldc, cm_stream_t stream)
+                        int64_t ldc, int32_t *dev_status, cm_stream_t stream)
 {
     if (!c || c->dt != CM_BF16) return CM_EINVAL;
-    if (N < 16 || N % 16 != 0 || c->d % 8 != 0) return CM_EINVAL;
+    if (N < 1) return CM_EINVAL;
     if (!layout_ok(A, lda, c->d, 2) || !layout_ok(par, ldp, c->d, 2) ||
         !layout_ok(Bt, ldb, c->d, 2))
         return CM_EINVAL;
-    if (!Ct || ((uintptr_t)Ct & 15u) || ldc < N || ldc % 4 != 0) return CM_EINVAL;
+    if (!Ct || ((uintptr_t)Ct & 15u) || ldc < N) return CM_EINVAL;
     return from_cuda(launch_coded_gemm(code_params(c), (const uint16_t *)A, lda,
                                        (const uint16_t *)par, ldp, (const uint16_t *)Bt, ldb,
-                                       N, Ct, ldc, (cudaStream_t)stream));
+                                       N, Ct, ldc, dev_status, (cudaStream_t)stream));
 }
 
 cm_status cm_decode_mat(const cm_code *c, const float *Ct, int64_t ldc, uint32_t survivors,
@@ -208,7 +208,7 @@ cm_status cm_matmat(const cm_code *c, const void *A, int64_t lda, const void *pa
     if (!c) return CM_EINVAL;
     cm_status st = check_survivors(c, survivors);
     if (st != CM_OK) return st;
-    st = cm_coded_gemm(c, A, lda, par, ldp, Bt, ldb, N, Ct, ldc, stream);
+    st = cm_coded_gemm(c, A, lda, par, ldp, Bt, ldb, N, Ct, ldc, dev_status, stream);
     if (st != CM_OK) return st;
     return cm_decode_mat(c, Ct, ldc, survivors, N, C, ldcc, dev_status, stream);
 }

@@ -58,4 +58,5 @@ cudaError_t launch_decode_mat(const CodeParams &cp, const float *Ct, int64_t ldc
                               int32_t *status, cudaStream_t s);
 cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t lda,
                               const uint16_t *par, int64_t ldp, const uint16_t *Bt,
-                              int64_t ldb, int N, float *Ct, int64_t ldc, cudaStream_t s);
+                              int64_t ldb, int N, float *Ct, int64_t ldc, int32_t *status,
+                              cudaStream_t s);

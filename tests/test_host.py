@@ -109,10 +109,12 @@ def test_synchronous_checks_precede_any_launch(cm):
     assert L.cm_encode(None, fake, 500, fake, 500, None) == cm.CM_EINVAL
     # f32 code refuses the bf16-only tensor-core path
     assert L.cm_coded_gemm(c.handle, fake, 512, fake, 512, fake, 512, 64, fake, 64,
-                           None) == cm.CM_EINVAL
+                           None, None) == cm.CM_EINVAL
     cb = cm.Code(6, 3, 120, 64, synth.parity_coefficients(6, 3), dtype="bf16")
-    assert L.cm_coded_gemm(cb.handle, fake, 64, fake, 64, fake, 64, 24, fake, 24,
-                           None) == cm.CM_EINVAL          # N % 16 != 0
+    assert L.cm_coded_gemm(cb.handle, fake, 64, fake, 64, fake, 64, 0, fake, 24,
+                           None, None) == cm.CM_EINVAL    # N < 1
+    assert L.cm_coded_gemm(cb.handle, fake, 68, fake, 64, fake, 64, 32, fake, 32,
+                           None, None) == cm.CM_EINVAL    # lda not 16-byte pitched
     assert L.cm_matvec(cb.handle, fake, 64, fake, 64, fake, 1, fake, None, None) == cm.CM_EINVAL
 
 

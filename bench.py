@@ -242,11 +242,14 @@ def run_reference(args, world, rank):
     print(json.dumps(line), flush=True)
 
 
-# A reduced copy of the bandwidth workload for ncu captures: same code and
-# batch, inputs still larger than L2 (0.96 GB of A), a few GB on the device at
-# most; L = 608 gives the 152-SM grid exactly two rounds of 8-row units.
+# Reduced copies of the workloads for ncu captures: same codes and batch,
+# inputs still larger than L2, a few GB on the device at most.  L = 608 gives
+# the 152-SM mat-vec grid exactly two rounds of 8-row units.
 PROFILE = synth.Workload("coded mat-multi-vec (32,24) 14592x16384 b=8 (profiling case)",
                          m=14592, d=16384, b=8, n=32, k=24, data_device="cuda")
+PROFILE_GEMM = synth.Workload("coded GEMM bf16 (16,12) 16384x8192x4096 (profiling case)",
+                              m=16384, d=8192, b=0, n=16, k=12, dtype="bf16", gemm_n=4096,
+                              data_device="cuda")
 WORKLOADS = {"bandwidth": synth.BANDWIDTH, "profile": PROFILE}
 
 
@@ -319,10 +322,14 @@ def run_ours(args, world, rank, local):
     avg = {k: float(np.mean(v)) for k, v in per.items()}
     launches_per_step = math.ceil((w.n - w.k) / 8) + 2
 
-    if not full:   # profiling case: kernels only
+    if not full:   # profiling case: kernels only, then the GEMM path once per step
+        del A, parity
+        torch.cuda.empty_cache()
+        gm = bench_gemm(cm, dev, PROFILE_GEMM, args.steps, args.warmup)
         if rank == 0:
             print(json.dumps({"workload": w.name, "ms_per_step": ms / args.steps,
-                              "kernels_us": {k: v * 1e3 for k, v in avg.items()}}), flush=True)
+                              "kernels_us": {k: v * 1e3 for k, v in avg.items()},
+                              "gemm": gm}), flush=True)
         return
 
     # end to end through the public API with host buffers: pinned X in, Y out
@@ -345,10 +352,16 @@ def run_ours(args, world, rank, local):
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
 
-    # secondary: coded gradient descent (40000 x 8000, (20,10) codes)
+    # secondary workloads: the other rows of the hot path
     del A, parity
     torch.cuda.empty_cache()
     gd = bench_gd(cm, dev, args.steps)
+    torch.cuda.empty_cache()
+    gemm = bench_gemm(cm, dev, synth.GEMM, max(3, args.steps // 4), args.warmup)
+    torch.cuda.empty_cache()
+    mv100 = bench_repeats(cm, dev, synth.MATVEC)
+    tiny = bench_repeats(cm, dev, synth.TINY, repeats=20)
+    torch.cuda.empty_cache()
 
     peaks = measured_peaks()
     achieved = nbytes["matvec"] / (avg["matvec"] * 1e-3) / 1e9
@@ -381,7 +394,7 @@ def run_ours(args, world, rank, local):
                 "d2h_bytes_per_step": w.m * w.b * 4},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
-        "secondary": {"gd": gd},
+        "secondary": {"gemm": gemm, "gd": gd, "matvec_100_repeats": mv100, "tiny": tiny},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w)
@@ -420,6 +433,93 @@ def bench_gd(cm, dev, steps: int) -> dict:
     nb = gd_iter_bytes(w, cA.L, cAT.L)
     return {"workload": w.name, "iters": w.iters, "ms_per_iter": ms,
             "gbs": nb / (ms * 1e-3) / 1e9, "launches_per_iter": 4,
+            "status": int(status.item())}
+
+
+def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
+    """Coded GEMM: bf16 encode once, then per step all n worker GEMMs on the
+    tensor cores and the decode of A B from the k survivors."""
+    peaks = measured_peaks()
+    P = synth.parity_coefficients(w.n, w.k)
+    code = cm.Code(w.n, w.k, w.m, w.d, P, dtype="bf16")
+    A, B = synth.gemm_inputs(w, device=dev)
+    Bt = B.t().contiguous()
+    del B
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    par = cm.encode(code, A)
+    e1.record()
+    Ct = torch.empty((w.n * code.L, w.gemm_n), device=dev)
+    C = torch.empty((w.m, w.gemm_n), device=dev)
+    masks = [cm.draw_erasures(synth.ERASURE_SEED, i, w.n, w.k)[0] for i in range(steps + warmup)]
+    for i in range(warmup):
+        cm.coded_gemm(code, A, par, Bt, Ct, status=status)
+        cm.decode_mat(code, Ct, masks[i], C=C, status=status)
+    torch.cuda.synchronize()
+    enc_ms = e0.elapsed_time(e1)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for i in range(steps):
+        ev[i][0].record()
+        cm.coded_gemm(code, A, par, Bt, Ct, status=status)
+        ev[i][1].record()
+        cm.decode_mat(code, Ct, masks[warmup + i], C=C, status=status)
+        ev[i][2].record()
+    torch.cuda.synchronize()
+    g_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in ev]))
+    d_ms = float(np.mean([e[1].elapsed_time(e[2]) for e in ev]))
+    flops = 2.0 * w.n * code.L * w.d * w.gemm_n          # every coded row
+    useful = 2.0 * w.m * w.d * w.gemm_n                  # A B itself
+    tflops = flops / (g_ms * 1e-3) / 1e12
+    dec_bytes = w.k * code.L * w.gemm_n * 4 + w.m * w.gemm_n * 4
+    return {"workload": w.name, "steps": steps, "gemm_ms": g_ms, "tflops": tflops,
+            "useful_tflops_per_step": useful / ((g_ms + d_ms) * 1e-3) / 1e12,
+            "roofline": {"bound": "tensor", "kernel": "coded GEMM (tcgen05, bf16 -> fp32)",
+                         "achieved": tflops, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                         "frac": tflops / peaks["bf16_tflops"],
+                         "peak_source": peaks["source"] + " bf16 burst"},
+            "decode_mat_ms": d_ms, "decode_mat_gbs": dec_bytes / (d_ms * 1e-3) / 1e9,
+            "encode_bf16_ms": enc_ms, "status": int(status.item())}
+
+
+def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dict:
+    """The paper-shaped repeat loop: encode once, then per repeat all n worker
+    products and the decode from a fresh straggler set; per-call latencies."""
+    P = synth.parity_coefficients(w.n, w.k)
+    code = cm.Code(w.n, w.k, w.m, w.d, P)
+    A, X = synth.matvec_inputs(w, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    parity = cm.encode(code, A)
+    torch.cuda.synchronize()
+    e0.record()
+    cm.encode(code, A, parity)
+    e1.record()
+    Yt = cm.matvec(code, A, parity, X, status=status)
+    Y = torch.empty((w.m, w.b), device=dev)
+    reps = repeats or w.repeats
+    masks = [cm.draw_erasures(synth.ERASURE_SEED, r, w.n, w.k)[0] for r in range(reps)]
+    for r in range(3):
+        cm.matvec(code, A, parity, X, Yt, status=status)
+        cm.decode(code, Yt, masks[r], Y=Y, status=status)
+    torch.cuda.synchronize()
+    enc_us = e0.elapsed_time(e1) * 1e3
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(reps)]
+    for r in range(reps):
+        ev[r][0].record()
+        cm.matvec(code, A, parity, X, Yt, status=status)
+        ev[r][1].record()
+        cm.decode(code, Yt, masks[r], Y=Y, status=status)
+        ev[r][2].record()
+    torch.cuda.synchronize()
+    mv = np.array([e[0].elapsed_time(e[1]) * 1e3 for e in ev])
+    dec = np.array([e[1].elapsed_time(e[2]) * 1e3 for e in ev])
+    nb = step_bytes(w, code.L)
+    return {"workload": w.name, "repeats": reps, "encode_us": enc_us,
+            "encode_gbs": nb["encode"] / (enc_us * 1e-6) / 1e9,
+            "matvec_us_median": float(np.median(mv)), "matvec_us_p95": float(np.percentile(mv, 95)),
+            "matvec_gbs_median": nb["matvec"] / (np.median(mv) * 1e-6) / 1e9,
+            "decode_us_median": float(np.median(dec)), "decode_us_p95": float(np.percentile(dec, 95)),
             "status": int(status.item())}
 
 

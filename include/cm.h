@@ -197,6 +197,13 @@ cm_status cm_matmat(const cm_code *code, const void *A, int64_t lda,
                     int32_t N, float *Ct, int64_t ldc, uint32_t survivors,
                     float *C, int64_t ldcc, int32_t *dev_status, cm_stream_t stream);
 
+/* Self-test of the bounded device wait that cm_matvec and cm_coded_gemm use
+ * for their TMA pipelines (no counterpart in the paper: failure detection).
+ * Launches one warp that waits on an mbarrier nothing arrives at, giving up
+ * after limit_ns nanoseconds (1 .. 2e9); the kernel then writes CM_ETIMEOUT
+ * to *dev_status and returns, and the context stays usable. */
+cm_status cm_selftest_bounded_wait(int32_t *dev_status, uint64_t limit_ns, cm_stream_t stream);
+
 /* Static description of a status code. */
 const char *cm_status_string(cm_status s);
 

@@ -67,6 +67,7 @@ def lib() -> ctypes.CDLL:
             "cm_decode_mat": (st, [vp, vp, i64, u32, i32, vp, i64, vp, vp]),
             "cm_matmat": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, u32, vp, i64,
                                vp, vp]),
+            "cm_selftest_bounded_wait": (st, [vp, u64, vp]),
             "cm_status_string": (ctypes.c_char_p, [st]),
         }
         for name, (res, args) in sig.items():
@@ -274,6 +275,14 @@ def gd_step_noalloc(code_A: Code, A, PA, code_AT: Code, AT, PAT, y, x, eta: floa
                                     y.data_ptr(), x.data_ptr(), eta, surv_A, surv_AT, sp,
                                     _stream()), "cm_gd_step_noalloc")
     return x
+
+
+def selftest_bounded_wait(status: torch.Tensor, limit_ns: int) -> None:
+    """Run the library's bounded-wait self-test: a device wait that nothing
+    completes must give up after limit_ns and write CM_ETIMEOUT to status."""
+    _dev(status, torch.int32, "status")
+    _check(lib().cm_selftest_bounded_wait(status.data_ptr(), limit_ns, _stream()),
+           "cm_selftest_bounded_wait")
 
 
 def coded_gemm(code: Code, A, parity, Bt, Ct=None, status=None) -> torch.Tensor:

@@ -332,3 +332,29 @@ def test_bandwidth_config_sampled(cm, orc):
             assert torch.equal(Y[lo:hi], Yt[lo:hi].float())
     del A, par, Yt
     torch.cuda.empty_cache()
+
+
+def test_bounded_wait_gives_up_and_reports(cm):
+    """Failure detection: the mbarrier wait that the TMA pipelines use gives
+    up on a barrier nothing completes, writes CM_ETIMEOUT, and the context
+    keeps working afterwards."""
+    import time
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    t0 = time.perf_counter()
+    cm.selftest_bounded_wait(status, 20_000_000)      # 20 ms
+    torch.cuda.synchronize()
+    dt = time.perf_counter() - t0
+    assert status.item() == cm.CM_ETIMEOUT
+    assert 0.015 < dt < 5.0, dt
+    # the context is still usable: a normal coded product runs and is correct
+    n, k, m, d = 6, 3, 90, 64
+    code = cm.Code(n, k, m, d, synth.parity_coefficients(n, k))
+    A = synth.gaussian((m, d), 8).to(DEV)
+    X = synth.gaussian((d, 1), 9).to(DEV)
+    status.zero_()
+    Yt = cm.matvec(code, A, cm.encode(code, A), X, status=status)
+    Y = cm.decode(code, Yt, 0b000111, status=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    want = (A.double() @ X.double()).cpu().numpy()
+    assert np.linalg.norm(Y.double().cpu().numpy() - want) <= 1e-5 * np.linalg.norm(want)

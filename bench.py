@@ -285,7 +285,7 @@ def run_ours(args, world, rank, local):
     def step(counter, ev=None):
         if ev:
             ev[0].record(stream)
-        cm.encode(code, A, parity)
+        cm.encode(code, A, parity, status=status)
         if ev:
             ev[1].record(stream)
         mask, _ = cm.draw_erasures(synth.ERASURE_SEED, counter, w.n, w.k)

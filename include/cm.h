@@ -76,11 +76,13 @@ int64_t cm_block_rows(const cm_code *code);
 
 /* Encoding (Sec. III-A): parity block p (rows [p L, (p+1) L) of parity_out,
  * leading dimension ldp) = sum_i P[p][i] A_i, for p = 0..n-k-1, in one pass
- * over A.  A is m x d with leading dimension lda, of the code's dtype (fp32,
- * or bf16 with fp32 accumulation and round-to-nearest-even output).
- * parity_out must not overlap A. */
+ * over A (n - k <= 16; larger counts take one pass per 16 parity blocks).
+ * A is m x d with leading dimension lda, of the code's dtype (fp32, or bf16
+ * with fp32 accumulation and round-to-nearest-even output).  parity_out must
+ * not overlap A.  A bounded wait that gives up writes CM_ETIMEOUT to
+ * *dev_status (nullable). */
 cm_status cm_encode(const cm_code *code, const void *A, int64_t lda,
-                    void *parity_out, int64_t ldp, cm_stream_t stream);
+                    void *parity_out, int64_t ldp, int32_t *dev_status, cm_stream_t stream);
 
 /* The n worker products (Sec. III-A protocol): Yt[j L + r][v] =
  * sum_c A~_j[r][c] X[c][v] for every worker j, row r < L and vector v < b,

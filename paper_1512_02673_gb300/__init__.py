@@ -54,7 +54,7 @@ def lib() -> ctypes.CDLL:
             "cm_code_create": (st, [i32, i32, i64, i64, st, vp, ctypes.POINTER(vp)]),
             "cm_code_destroy": (None, [vp]),
             "cm_block_rows": (i64, [vp]),
-            "cm_encode": (st, [vp, vp, i64, vp, i64, vp]),
+            "cm_encode": (st, [vp, vp, i64, vp, i64, vp, vp]),
             "cm_matvec": (st, [vp, vp, i64, vp, i64, vp, i32, vp, vp, vp]),
             "cm_draw_erasures": (st, [u64, u64, i32, i32, f64, f64, ctypes.POINTER(u32), vp]),
             "cm_decode": (st, [vp, vp, u32, i32, vp, vp, vp]),
@@ -144,7 +144,8 @@ class Code:
         return torch.float32 if self.dtype == "f32" else torch.bfloat16
 
 
-def encode(code: Code, A: torch.Tensor, parity: torch.Tensor | None = None) -> torch.Tensor:
+def encode(code: Code, A: torch.Tensor, parity: torch.Tensor | None = None,
+           status: torch.Tensor | None = None) -> torch.Tensor:
     """Parity blocks ((n-k) L x d, code dtype) of A (m x d)."""
     dt = code.torch_dtype
     _dev(A, dt, "A", 2)
@@ -159,8 +160,12 @@ def encode(code: Code, A: torch.Tensor, parity: torch.Tensor | None = None) -> t
     _dev(parity, dt, "parity", 2)
     if tuple(parity.shape) != ((code.n - code.k) * code.L, code.d):
         raise ValueError("parity must be (n-k) L x d")
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
     _check(lib().cm_encode(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
-                           _ld(parity, "parity"), _stream()), "cm_encode")
+                           _ld(parity, "parity"), sp, _stream()), "cm_encode")
     return parity
 
 

@@ -79,7 +79,7 @@ void cm_code_destroy(cm_code *code) { std::free(code); }
 int64_t cm_block_rows(const cm_code *code) { return code ? code->L : -1; }
 
 cm_status cm_encode(const cm_code *c, const void *A, int64_t lda, void *par, int64_t ldp,
-                    cm_stream_t stream)
+                    int32_t *dev_status, cm_stream_t stream)
 {
     if (!c) return CM_EINVAL;
     int64_t es = c->dt == CM_F32 ? 4 : 2;
@@ -87,9 +87,9 @@ cm_status cm_encode(const cm_code *c, const void *A, int64_t lda, void *par, int
     CodeParams cp = code_params(c);
     if (c->dt == CM_F32)
         return from_cuda(launch_encode_f32(cp, (const float *)A, lda, (float *)par, ldp,
-                                           (cudaStream_t)stream));
+                                           dev_status, (cudaStream_t)stream));
     return from_cuda(launch_encode_bf16(cp, (const uint16_t *)A, lda, (uint16_t *)par, ldp,
-                                        (cudaStream_t)stream));
+                                        dev_status, (cudaStream_t)stream));
 }
 
 cm_status cm_matvec(const cm_code *c, const float *A, int64_t lda, const float *par,

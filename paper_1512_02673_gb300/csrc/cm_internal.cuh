@@ -41,9 +41,9 @@ int cm_sm_count();
 
 // ---- launchers (return cudaSuccess or the launch error) --------------------
 cudaError_t launch_encode_f32(const CodeParams &cp, const float *A, int64_t lda,
-                              float *par, int64_t ldp, cudaStream_t s);
+                              float *par, int64_t ldp, int32_t *status, cudaStream_t s);
 cudaError_t launch_encode_bf16(const CodeParams &cp, const uint16_t *A, int64_t lda,
-                               uint16_t *par, int64_t ldp, cudaStream_t s);
+                               uint16_t *par, int64_t ldp, int32_t *status, cudaStream_t s);
 cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda,
                           const float *par, int64_t ldp, const float *X, int b,
                           double *Yt, int32_t *status, cudaStream_t s);

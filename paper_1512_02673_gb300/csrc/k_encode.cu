@@ -1,152 +1,229 @@
 // K1: encoding (Sec. III-A): parity block p = sum_i P[p][i] A_i for every
 // parity block p of the (n,k) code, applied elementwise across the k row
-// blocks of A (rows past m are the appended zero rows and are skipped).
+// blocks of A (rows past m are the appended zero rows).
 //
-// A short contraction (k <= 31) that streams A once: each thread owns one
-// 16-byte vector of columns of one block row r, reads the k vectors
-// A_i[r][cols] with 128-bit loads (held in flight in groups of 4) and keeps
-// all NPG parity accumulators of that vector in registers, so every element
-// of A is read once per pass and every parity element written once
-// (n - k <= NPG: one pass).  fp32 accumulation; bf16 outputs are rounded to
-// nearest even once, at the end.  The grid is persistent (SMs x resident
-// CTAs) over a flattened (row, column vector) space, so accesses are
-// coalesced along rows.
+// A short contraction (k <= 31 terms per output) that streams A once.  Work
+// unit = one block row r and a 4096-column segment, owned by one warp; a
+// persistent grid sweeps the units.  Each 128-column step of a unit gathers
+// row r of every data block into shared memory with TMA in sub-steps of KC
+// blocks: 3-D boxes of KC full blocks (block stride L rows; boxes past the
+// last full block read as zero) plus, if m is not a multiple of L, one 2-D
+// box of the partial block whose rows past m read as zero; blocks wholly past
+// m are skipped.  Sub-steps stream through a per-warp ring of ST slots with
+// one mbarrier each (lane 0 issues, the warp consumes), so several KB per
+// warp are in flight with no per-lane copy work, and small slots leave room
+// for 16 warps per SM.  Lane l owns
+// columns [4l, 4l+4) of the step and keeps the accumulators of all parity
+// blocks of the pass in registers (packed fp32x2 FMAs with the coefficient
+// pair (P[p][i], P[p][i]) read as a shared-memory broadcast), then stores them
+// with coalesced streaming stores.  Every element of A is read once per pass
+// and every parity element written once; n - k <= 16 is one pass.  fp32
+// accumulation in the order i = 0..k-1; bf16 outputs are rounded to nearest
+// even once.  Waits are bounded (about 2 s): a time-out writes CM_ETIMEOUT
+// to the status word and the warp stops.
 #include <cuda_bf16.h>
 
 #include "cm_internal.cuh"
+#include "tma.cuh"
 
 namespace {
 
-constexpr int kThreads = 256;
-
-struct EncodeArgs {
-    CodeParams cp;
-    const void *A;
-    int64_t lda;
-    void *par;
-    int64_t ldp;
-    int p0;   // first parity block of this pass
-    int np;   // parity blocks in this pass
-};
+constexpr int STEP = 128;       // columns per step
+constexpr int SEG = 32;         // steps per work unit
+constexpr int KC = 8;           // data blocks per sub-step (one TMA box)
+constexpr int ST = 3;           // ring slots per warp
+constexpr int kWarps = 8;
 
 template <typename T>
-struct Vec;
+struct Elem;
+
 template <>
-struct Vec<float> {
-    static constexpr int W = 4;
-    __device__ static void load(const float *p, float (&v)[4])
+struct Elem<float> {
+    static constexpr CUtensorMapDataType TM = CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    __device__ static void load4(const float *p, float2 &a, float2 &b)
     {
-        float4 t;
-        asm("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];\n"
-            : "=f"(t.x), "=f"(t.y), "=f"(t.z), "=f"(t.w)
-            : "l"(p));
-        v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+        const float4 v = *reinterpret_cast<const float4 *>(p);
+        a = make_float2(v.x, v.y);
+        b = make_float2(v.z, v.w);
     }
-    __device__ static float scalar(const float *p) { return __ldg(p); }
-    __device__ static void store(float *p, const float (&v)[4])
+    __device__ static void store4(float *p, float2 a, float2 b)
     {
-        __stcs(reinterpret_cast<float4 *>(p), make_float4(v[0], v[1], v[2], v[3]));
+        __stcs(reinterpret_cast<float4 *>(p), make_float4(a.x, a.y, b.x, b.y));
     }
-    __device__ static void store_scalar(float *p, float v) { *p = v; }
+    __device__ static void store1(float *p, float v) { *p = v; }
 };
+
 template <>
-struct Vec<uint16_t> {   // bf16 bits
-    static constexpr int W = 8;
+struct Elem<uint16_t> {   // bf16 bits
+    static constexpr CUtensorMapDataType TM = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     __device__ static float widen(uint32_t h) { return __uint_as_float(h << 16); }
-    __device__ static void load(const uint16_t *p, float (&v)[8])
-    {
-        uint4 t;
-        asm("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];\n"
-            : "=r"(t.x), "=r"(t.y), "=r"(t.z), "=r"(t.w)
-            : "l"(p));
-        const uint32_t w[4] = {t.x, t.y, t.z, t.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            v[2 * i] = widen(w[i] & 0xffffu);
-            v[2 * i + 1] = widen(w[i] >> 16);
-        }
-    }
-    __device__ static float scalar(const uint16_t *p) { return widen(__ldg(p)); }
     __device__ static uint32_t rne(float f)
     {
         return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(f));
     }
-    __device__ static void store(uint16_t *p, const float (&v)[8])
+    __device__ static void load4(const uint16_t *p, float2 &a, float2 &b)
     {
-        uint4 t;
-        t.x = rne(v[0]) | (rne(v[1]) << 16);
-        t.y = rne(v[2]) | (rne(v[3]) << 16);
-        t.z = rne(v[4]) | (rne(v[5]) << 16);
-        t.w = rne(v[6]) | (rne(v[7]) << 16);
-        __stcs(reinterpret_cast<uint4 *>(p), t);
+        const uint2 v = *reinterpret_cast<const uint2 *>(p);
+        a = make_float2(widen(v.x & 0xffffu), widen(v.x >> 16));
+        b = make_float2(widen(v.y & 0xffffu), widen(v.y >> 16));
     }
-    __device__ static void store_scalar(uint16_t *p, float v) { *p = (uint16_t)rne(v); }
+    __device__ static void store4(uint16_t *p, float2 a, float2 b)
+    {
+        uint2 v;
+        v.x = rne(a.x) | (rne(a.y) << 16);
+        v.y = rne(b.x) | (rne(b.y) << 16);
+        __stcs(reinterpret_cast<uint2 *>(p), v);
+    }
+    __device__ static void store1(uint16_t *p, float v) { *p = (uint16_t)rne(v); }
+};
+
+struct EncodeArgs {
+    void *par;
+    int64_t ldp;
+    int32_t *status;
+    int64_t d, L;
+    int32_t k;
+    int32_t kf;          // data blocks with all L rows below m
+    int32_t kv;          // data blocks with at least one row below m
+    int32_t p0, np;      // parity blocks of this pass
+    int32_t steps;       // 128-column steps per row
+    int32_t nseg;        // segments per row
+    int32_t nsub;        // sub-steps per step: ceil(kf / KC) + (kv > kf)
+    int64_t units;       // L * nseg
 };
 
 template <typename T, int NPG>
-__global__ void __launch_bounds__(kThreads) encode_kernel(const EncodeArgs a)
+__global__ void __launch_bounds__(kWarps * 32)
+encode_kernel(const __grid_constant__ CUtensorMap tmF, const __grid_constant__ CUtensorMap tmP,
+              const CodeParams cp, const EncodeArgs a)
 {
-    constexpr int W = Vec<T>::W;
-    constexpr int G = 4;   // data blocks loaded per group
-    const int k = a.cp.k, np = a.np, p0 = a.p0;
-    const int64_t L = a.cp.L, m = a.cp.m, d = a.cp.d;
-    const int64_t nvec = (d + W - 1) / W;
-    const int64_t total = L * nvec;
-    const T *A = static_cast<const T *>(a.A);
-    T *par = static_cast<T *>(a.par);
-    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < total;
-         it += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t r = it / nvec;
-        const int64_t col = (it - r * nvec) * W;
-        const bool full = col + W <= d;
-        float acc[NPG][W];
-#pragma unroll
-        for (int j = 0; j < NPG; ++j)
-#pragma unroll
-            for (int e = 0; e < W; ++e) acc[j][e] = 0.f;
-        for (int i0 = 0; i0 < k; i0 += G) {
-            float v[G][W];
-#pragma unroll
-            for (int g = 0; g < G; ++g) {
-                const int i = i0 + g;
-                const int64_t row = (int64_t)i * L + r;
-#pragma unroll
-                for (int e = 0; e < W; ++e) v[g][e] = 0.f;
-                if (i < k && row < m) {
-                    const T *src = A + row * a.lda + col;
-                    if (full) {
-                        Vec<T>::load(src, v[g]);
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < W; ++e)
-                            if (col + e < d) v[g][e] = Vec<T>::scalar(src + e);
-                    }
-                }
-            }
-#pragma unroll
-            for (int g = 0; g < G; ++g) {
-                const int i = i0 + g;
-                if (i >= k) break;
-#pragma unroll
-                for (int j = 0; j < NPG; ++j) {
-                    if (j < np) {
-                        const float w = a.cp.P[(p0 + j) * k + i];
-#pragma unroll
-                        for (int e = 0; e < W; ++e) acc[j][e] = fmaf(w, v[g][e], acc[j][e]);
-                    }
-                }
+    constexpr uint32_t SLOT = KC * STEP * sizeof(T);
+    // dynamic shared memory: [rings, 1024-aligned][coefficient pairs][mbarriers]
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const uint32_t raw0 = cm_smem_u32(smem_raw);
+    unsigned char *rings = smem_raw + (((raw0 + 1023) & ~1023u) - raw0);
+    float2 *pairs = reinterpret_cast<float2 *>(rings + kWarps * ST * SLOT);   // i * NPG + j
+    uint64_t *bars = reinterpret_cast<uint64_t *>(pairs + 32 * NPG);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    unsigned char *ring = rings + warp * ST * SLOT;
+    uint64_t *bar = bars + warp * ST;
+
+    for (int t = threadIdx.x; t < a.kv * NPG; t += blockDim.x) {
+        const int i = t / NPG, j = t % NPG;
+        const float w = j < a.np ? cp.P[(a.p0 + j) * a.k + i] : 0.f;
+        pairs[t] = make_float2(w, w);
+    }
+    if (threadIdx.x < kWarps * ST) cm_mbar_init(&bars[threadIdx.x], 1);
+    cm_fence_mbar_init();
+    __syncthreads();
+
+    const int64_t total_warps = (int64_t)gridDim.x * kWarps;
+    const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
+    if (gw >= a.units) return;
+    const int nfull = (a.kf + KC - 1) / KC;      // sub-steps of full blocks
+
+    auto unit_steps = [&](int64_t u) {           // the last segment of a row may be short
+        const int s0 = (int)(u % a.nseg) * SEG;
+        return (a.steps - s0) < SEG ? a.steps - s0 : SEG;
+    };
+
+    // ---- producer (lane 0): sub-step c of step p_s of unit p_unit ----
+    int64_t p_unit = gw;
+    int p_s = 0, p_c = 0, p_slot = 0, in_flight = 0;
+    auto produce = [&]() {
+        const int64_t r = p_unit / a.nseg;
+        const int32_t x = ((int)(p_unit % a.nseg) * SEG + p_s) * STEP;
+        unsigned char *dst = ring + p_slot * SLOT;
+        cm_fence_proxy_async();
+        if (p_c < nfull) {
+            cm_mbar_arrive_expect_tx(&bar[p_slot], SLOT);
+            cm_tma_load_3d(dst, &tmF, x, (int32_t)r, p_c * KC, &bar[p_slot]);
+        } else {
+            cm_mbar_arrive_expect_tx(&bar[p_slot], STEP * sizeof(T));
+            cm_tma_load_2d(dst, &tmP, x, (int32_t)r, &bar[p_slot]);
+        }
+        p_slot = p_slot + 1 == ST ? 0 : p_slot + 1;
+        ++in_flight;
+        if (++p_c == a.nsub) {
+            p_c = 0;
+            if (++p_s == unit_steps(p_unit)) {
+                p_s = 0;
+                p_unit += total_warps;
             }
         }
+    };
+    if (lane == 0)
+        while (in_flight < ST && p_unit < a.units) produce();
+
+    // ---- consumer ----
+    int slot = 0;
+    uint32_t phase = 0;
+    T *par = static_cast<T *>(a.par);
+    for (int64_t u = gw; u < a.units; u += total_warps) {
+        const int64_t r = u / a.nseg;
+        const int seg = (int)(u % a.nseg);
+        const int ns = unit_steps(u);
+        for (int s = 0; s < ns; ++s) {
+            float2 acc[NPG][2];
 #pragma unroll
-        for (int j = 0; j < NPG; ++j) {
-            if (j < np) {
-                T *dst = par + ((int64_t)(p0 + j) * L + r) * a.ldp + col;
-                if (full) {
-                    Vec<T>::store(dst, acc[j]);
-                } else {
+            for (int j = 0; j < NPG; ++j) acc[j][0] = acc[j][1] = make_float2(0.f, 0.f);
+            for (int c = 0; c < a.nsub; ++c) {
+                if (!cm_mbar_wait(&bar[slot], phase)) {
+                    if (lane == 0) {
+                        if (a.status) *a.status = CM_ETIMEOUT;
+                        // wait (bounded) for this warp's copies still in flight
+                        for (int i = 0; i < in_flight; ++i) {
+                            cm_mbar_wait(&bar[slot], phase, 100000000ull);
+                            if (++slot == ST) {
+                                slot = 0;
+                                phase ^= 1u;
+                            }
+                        }
+                    }
+                    return;   // no CTA barrier follows: the warp may leave
+                }
+                // blocks of this sub-step: [i0, i0 + nb)
+                const int i0 = c < nfull ? c * KC : a.kf;
+                const int nb = c < nfull ? (a.kf - i0 < KC ? a.kf - i0 : KC) : 1;
+                const T *src = reinterpret_cast<const T *>(ring + slot * SLOT) + 4 * lane;
+                const float2 *pp = pairs + i0 * NPG;
+#pragma unroll 2
+                for (int i = 0; i < nb; ++i) {
+                    float2 a01, a23;
+                    Elem<T>::load4(src + i * STEP, a01, a23);
 #pragma unroll
-                    for (int e = 0; e < W; ++e)
-                        if (col + e < d) Vec<T>::store_scalar(dst + e, acc[j][e]);
+                    for (int j = 0; j < NPG; ++j) {
+                        if (j < a.np) {
+                            const float2 w = pp[i * NPG + j];
+                            acc[j][0] = __ffma2_rn(w, a01, acc[j][0]);
+                            acc[j][1] = __ffma2_rn(w, a23, acc[j][1]);
+                        }
+                    }
+                }
+                if (++slot == ST) {
+                    slot = 0;
+                    phase ^= 1u;
+                }
+                __syncwarp();   // every lane is done reading the slot
+                if (lane == 0) {
+                    --in_flight;
+                    if (p_unit < a.units) produce();   // refill it
+                }
+            }
+            const int64_t col = (int64_t)(seg * SEG + s) * STEP + 4 * lane;
+            if (col < a.d) {
+#pragma unroll
+                for (int j = 0; j < NPG; ++j) {
+                    if (j < a.np) {
+                        T *dst = par + ((int64_t)(a.p0 + j) * a.L + r) * a.ldp + col;
+                        if (col + 4 <= a.d) {
+                            Elem<T>::store4(dst, acc[j][0], acc[j][1]);
+                        } else {
+                            const float v[4] = {acc[j][0].x, acc[j][0].y, acc[j][1].x,
+                                                acc[j][1].y};
+                            for (int e = 0; col + e < a.d; ++e) Elem<T>::store1(dst + e, v[e]);
+                        }
+                    }
                 }
             }
         }
@@ -154,30 +231,53 @@ __global__ void __launch_bounds__(kThreads) encode_kernel(const EncodeArgs a)
 }
 
 template <typename T, int NPG>
-cudaError_t launch_passes(const CodeParams &cp, const void *A, int64_t lda, void *par,
-                          int64_t ldp, cudaStream_t s)
+cudaError_t launch_passes(const CodeParams &cp, const T *A, int64_t lda, T *par, int64_t ldp,
+                          int32_t *status, cudaStream_t s)
 {
-    auto kern = encode_kernel<T, NPG>;
-    int per_sm = 0;
-    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, 0);
-    if (e != cudaSuccess) return e;
-    if (per_sm < 1) per_sm = 1;
-    const int64_t W = Vec<T>::W;
-    const int64_t items = cp.L * ((cp.d + W - 1) / W);
-    int64_t grid = (int64_t)cm_sm_count() * per_sm;
-    const int64_t need = (items + kThreads - 1) / kThreads;
-    if (grid > need) grid = need;
-    if (grid < 1) grid = 1;
+    const int64_t es = sizeof(T);
+    const int kf = (int)(cp.m / cp.L);                 // >= 1 since L <= m
+    const int kv = (int)((cp.m + cp.L - 1) / cp.L);
+    CUtensorMap tmF, tmP;
+    if (!cm_make_tmap_3d(&tmF, Elem<T>::TM, A, (uint64_t)cp.d, (uint64_t)cp.L, (uint64_t)kf,
+                         (uint64_t)(lda * es), (uint64_t)(cp.L * lda * es), STEP, 1, KC))
+        return cudaErrorInvalidValue;
+    if (kv > kf) {
+        if (!cm_make_tmap_2d(&tmP, Elem<T>::TM, A + (int64_t)kf * cp.L * lda, (uint64_t)cp.d,
+                             (uint64_t)(cp.m - (int64_t)kf * cp.L), (uint64_t)(lda * es), STEP, 1,
+                             CU_TENSOR_MAP_SWIZZLE_NONE))
+            return cudaErrorInvalidValue;
+    } else {
+        tmP = tmF;   // unused
+    }
     EncodeArgs a;
-    a.cp = cp;
-    a.A = A;
-    a.lda = lda;
     a.par = par;
     a.ldp = ldp;
+    a.status = status;
+    a.d = cp.d;
+    a.L = cp.L;
+    a.k = cp.k;
+    a.kf = kf;
+    a.kv = kv;
+    a.steps = (int)((cp.d + STEP - 1) / STEP);
+    a.nseg = (a.steps + SEG - 1) / SEG;
+    a.units = cp.L * a.nseg;
+    a.nsub = (kf + KC - 1) / KC + (kv > kf ? 1 : 0);
+    auto kern = encode_kernel<T, NPG>;
+    const int smem = 1024 + kWarps * ST * KC * STEP * (int)es + 32 * NPG * 8 + kWarps * ST * 8;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kWarps * 32, smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) per_sm = 1;
+    int64_t grid = (int64_t)cm_sm_count() * per_sm;
+    const int64_t need = (a.units + kWarps - 1) / kWarps;
+    if (grid > need) grid = need;
+    if (grid < 1) grid = 1;
     for (int p0 = 0; p0 < cp.n - cp.k; p0 += NPG) {
         a.p0 = p0;
         a.np = cp.n - cp.k - p0 < NPG ? cp.n - cp.k - p0 : NPG;
-        kern<<<(unsigned)grid, kThreads, 0, s>>>(a);
+        kern<<<(unsigned)grid, kWarps * 32, smem, s>>>(tmF, tmP, cp, a);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     return cudaSuccess;
@@ -186,14 +286,19 @@ cudaError_t launch_passes(const CodeParams &cp, const void *A, int64_t lda, void
 }  // namespace
 
 cudaError_t launch_encode_f32(const CodeParams &cp, const float *A, int64_t lda, float *par,
-                              int64_t ldp, cudaStream_t s)
+                              int64_t ldp, int32_t *status, cudaStream_t s)
 {
-    if (cp.n - cp.k <= 8) return launch_passes<float, 8>(cp, A, lda, par, ldp, s);
-    return launch_passes<float, 16>(cp, A, lda, par, ldp, s);
+    const int np = cp.n - cp.k;
+    if (np <= 4) return launch_passes<float, 4>(cp, A, lda, par, ldp, status, s);
+    if (np <= 8) return launch_passes<float, 8>(cp, A, lda, par, ldp, status, s);
+    return launch_passes<float, 16>(cp, A, lda, par, ldp, status, s);
 }
 
 cudaError_t launch_encode_bf16(const CodeParams &cp, const uint16_t *A, int64_t lda,
-                               uint16_t *par, int64_t ldp, cudaStream_t s)
+                               uint16_t *par, int64_t ldp, int32_t *status, cudaStream_t s)
 {
-    return launch_passes<uint16_t, 8>(cp, A, lda, par, ldp, s);
+    const int np = cp.n - cp.k;
+    if (np <= 4) return launch_passes<uint16_t, 4>(cp, A, lda, par, ldp, status, s);
+    if (np <= 8) return launch_passes<uint16_t, 8>(cp, A, lda, par, ldp, status, s);
+    return launch_passes<uint16_t, 16>(cp, A, lda, par, ldp, status, s);
 }

@@ -43,3 +43,19 @@ bool cm_make_tmap_2d(CUtensorMap *map, CUtensorMapDataType type, const void *bas
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
+
+bool cm_make_tmap_3d(CUtensorMap *map, CUtensorMapDataType type, const void *base,
+                     uint64_t width, uint64_t height, uint64_t depth, uint64_t pitch_bytes,
+                     uint64_t slab_bytes, uint32_t box_w, uint32_t box_h, uint32_t box_d)
+{
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[3] = {width, height, depth};
+    const cuuint64_t strides[2] = {pitch_bytes, slab_bytes};
+    const cuuint32_t box[3] = {box_w, box_h, box_d};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(map, type, 3, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}

@@ -18,6 +18,13 @@ bool cm_make_tmap_2d(CUtensorMap *map, CUtensorMapDataType type, const void *bas
                      uint64_t width, uint64_t height, uint64_t pitch_bytes, uint32_t box_w,
                      uint32_t box_h, CUtensorMapSwizzle swizzle);
 
+// Encode a 3-D tensor map: `depth` slabs of `height` rows of `width`
+// elements; row pitch and slab pitch in bytes (multiples of 16); boxes of
+// box_w x box_h x box_d elements, no swizzle, zero fill outside.
+bool cm_make_tmap_3d(CUtensorMap *map, CUtensorMapDataType type, const void *base,
+                     uint64_t width, uint64_t height, uint64_t depth, uint64_t pitch_bytes,
+                     uint64_t slab_bytes, uint32_t box_w, uint32_t box_h, uint32_t box_d);
+
 // ---- device -------------------------------------------------------------------------
 
 __device__ __forceinline__ uint32_t cm_smem_u32(const void *p)
@@ -86,6 +93,17 @@ __device__ __forceinline__ bool cm_mbar_wait(uint64_t *bar, uint32_t parity,
         if (cm_mbar_try_wait(bar, parity)) return true;
         if ((it & 255u) == 0 && cm_globaltimer() - t0 > limit_ns) return false;
     }
+}
+
+// 3-D TMA tile load global -> shared, completion counted on `bar`.
+__device__ __forceinline__ void cm_tma_load_3d(void *smem_dst, const CUtensorMap *map, int32_t x,
+                                               int32_t y, int32_t z, uint64_t *bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
+        "[%0], [%1, {%2, %3, %4}], [%5];\n" ::"r"(cm_smem_u32(smem_dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(z), "r"(cm_smem_u32(bar))
+        : "memory");
 }
 
 // 2-D TMA tile load global -> shared, completion counted on `bar`.

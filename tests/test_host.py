@@ -105,8 +105,8 @@ def test_synchronous_checks_precede_any_launch(cm):
     assert L.cm_matvec(c.handle, odd, 500, fake, 500, fake, 1, fake, None, None) == cm.CM_EINVAL
     assert L.cm_matvec(c.handle, fake, 501, fake, 500, fake, 1, fake, None, None) == cm.CM_EINVAL
     assert L.cm_matvec(c.handle, fake, 496, fake, 500, fake, 1, fake, None, None) == cm.CM_EINVAL
-    assert L.cm_encode(c.handle, fake, 502, fake, 500, None) == cm.CM_EINVAL
-    assert L.cm_encode(None, fake, 500, fake, 500, None) == cm.CM_EINVAL
+    assert L.cm_encode(c.handle, fake, 502, fake, 500, None, None) == cm.CM_EINVAL
+    assert L.cm_encode(None, fake, 500, fake, 500, None, None) == cm.CM_EINVAL
     # f32 code refuses the bf16-only tensor-core path
     assert L.cm_coded_gemm(c.handle, fake, 512, fake, 512, fake, 512, 64, fake, 64,
                            None, None) == cm.CM_EINVAL

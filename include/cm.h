@@ -121,7 +121,9 @@ cm_status cm_draw_erasures(uint64_t seed, uint64_t counter, int32_t n, int32_t k
  * surviving systematic blocks pass through.  Y (m x b fp32) is the
  * concatenation of the k decoded blocks without the appended zero rows.
  * Returns CM_ENOTDECODABLE when fewer than k bits are set; a singular G_S
- * writes CM_ESINGULAR to *dev_status (nullable) and leaves Y unwritten. */
+ * (a zero pivot, or ||Q|| ||Q^-1|| beyond 1 / (64 eps) for the e x e block)
+ * writes CM_ESINGULAR to *dev_status (nullable) and leaves the missing
+ * blocks of Y unwritten (surviving systematic blocks are still copied). */
 cm_status cm_decode(const cm_code *code, const double *Yt, uint32_t survivors,
                     int32_t b, float *Y, int32_t *dev_status, cm_stream_t stream);
 

@@ -16,6 +16,14 @@
 // combination of the k surviving rows r, surviving systematic blocks pass
 // through.  A zero (or relatively negligible) pivot marks G_S singular: the
 // kernel writes CM_ESINGULAR to the status word and writes no output.
+//
+// fp64 arithmetic runs at about 1/58 of the fp32 rate on this part, so the
+// vector decode applies the fp64 coefficients in double-float arithmetic on
+// the fp32 pipe: each fp64 coefficient and each fp64 worker result is split
+// into a (high, low) fp32 pair (results by integer bit manipulation, no fp64
+// instruction), products are formed exactly with an FMA and the sums are kept
+// as (sum, compensation) pairs (Knuth's TwoSum), about 2^-44 relative per
+// term, far below the rounding of the fp32 output.
 #include <cfloat>
 
 #include "cm_internal.cuh"
@@ -28,16 +36,19 @@ constexpr int kMaxE = 16;   // e <= min(k, n - k) <= 16 for n <= 32
 struct DecodeShared {
     int S[CM_MAX_N];       // survivors in ascending order (k of them)
     int role[CM_MAX_N];    // block i < k: -1 passes through, else its row c in M
+    int M[kMaxE];          // missing systematic blocks, ascending
     int Ps[kMaxE];         // surviving parity workers, ascending
     int e;
     int singular;
     double W[kMaxE][2 * kMaxE];   // [Q | I] during elimination
     double Qi[kMaxE][kMaxE];      // Q^-1
     double D[kMaxE][CM_MAX_N];    // decode rows: D[c][p], p = position in S
+    float Dh[kMaxE][CM_MAX_N];    // D as (high, low) fp32 pairs
+    float Dl[kMaxE][CM_MAX_N];
 };
 
-// Warp 0 of the CTA fills sh (S, role, e, D, singular).
-__device__ void decode_coefficients(const CodeParams &cp, uint32_t survivors, DecodeShared &sh)
+// Warp 0: the survivor lists (S, role, M, Ps, e) from the mask, by ballots.
+__device__ void decode_select(const CodeParams &cp, uint32_t survivors, DecodeShared &sh)
 {
     const int lane = threadIdx.x & 31;
     const int n = cp.n, k = cp.k;
@@ -50,63 +61,60 @@ __device__ void decode_coefficients(const CodeParams &cp, uint32_t survivors, De
     const uint32_t missm = __ballot_sync(0xffffffffu, miss);
     const bool par = sel && lane >= k;
     const uint32_t parm = __ballot_sync(0xffffffffu, par);
-    const int e = __popc(missm);
     if (sel) sh.S[__popc(selm & below)] = lane;
     if (par) sh.Ps[__popc(parm & below)] = lane;
+    if (miss) sh.M[__popc(missm & below)] = lane;
     if (lane < k) sh.role[lane] = miss ? __popc(missm & below) : -1;
-    // per-lane copies of the M and Ps lists (lane-indexed via shuffles)
-    int Mi = -1, Pi = -1;
-    {
-        // position of each missing / parity worker in its list
-        int mpos = miss ? __popc(missm & below) : -1;
-        int ppos = par ? __popc(parm & below) : -1;
-        // gather: list element t is the lane whose pos == t
-        for (int src = 0; src < 32; ++src) {
-            int pm = __shfl_sync(0xffffffffu, mpos, src);
-            int pp = __shfl_sync(0xffffffffu, ppos, src);
-            if (pm == lane) Mi = src;
-            if (pp == lane) Pi = src;
-        }
-    }
     if (lane == 0) {
-        sh.e = e;
+        sh.e = __popc(missm);
         sh.singular = 0;
     }
-    if (e == 0) {
-        __syncwarp();
-        return;
-    }
+}
+
+// Warp 0: rows of G_S^-1 for the missing blocks (D, and D as fp32 pairs).
+// fp64 instructions have long latency on this part (about 64 cycles for a
+// multiply or FMA, about 440 for a reciprocal), so the elimination is
+// fraction-free: a non-pivot row becomes piv * W[a] - W[a][col] * W[col]
+// (separate products, so duplicated rows cancel to exactly zero), with one
+// reciprocal per row at the end; partial pivoting is unaffected because all
+// non-pivot rows are scaled alike.  G_S counts as singular when a pivot is
+// zero or not finite, or when ||Q||_inf ||Q^-1||_inf exceeds 1 / (64 eps).
+__device__ void decode_coefficients(const CodeParams &cp, DecodeShared &sh)
+{
+    const int lane = threadIdx.x & 31;
+    const int k = cp.k, e = sh.e;
+    if (e == 0) return;
+    const int mc = lane < e ? sh.M[lane] : 0;
     // W = [Q | I], Q[a][c] = P[Ps[a] - k][M[c]]; lane owns column `lane`.
-    double scale = 0.0;
-    const int mc = __shfl_sync(0xffffffffu, Mi, lane < e ? lane : 0);   // M[lane]
+    double qnorm = 0.0;   // row sums of |Q| (lane a < e holds row a)
     for (int a = 0; a < e; ++a) {
-        const int ps = __shfl_sync(0xffffffffu, Pi, a);                   // Ps[a]
+        const int ps = sh.Ps[a];
         double w = 0.0;
-        if (lane < e) {
-            w = (double)cp.P[(ps - k) * k + mc];
-            scale = fmax(scale, fabs(w));
-        } else if (lane < 2 * e) {
-            w = (lane - e == a) ? 1.0 : 0.0;
-        }
+        if (lane < e) w = (double)cp.P[(ps - k) * k + mc];
+        else if (lane < 2 * e) w = (lane - e == a) ? 1.0 : 0.0;
         if (lane < 2 * e) sh.W[a][lane] = w;
     }
-    for (int off = 16; off; off >>= 1) scale = fmax(scale, __shfl_xor_sync(0xffffffffu, scale, off));
-    const double tol = 64.0 * DBL_EPSILON * scale;
     __syncwarp();
+    if (lane < e)
+        for (int c = 0; c < e; ++c) qnorm += fabs(sh.W[lane][c]);
+    for (int off = 16; off; off >>= 1) qnorm = fmax(qnorm, __shfl_xor_sync(0xffffffffu, qnorm, off));
     int singular = 0;
-    for (int col = 0; col < e && !singular; ++col) {
-        // partial pivoting: largest |W[a][col]| over a >= col, lowest index on ties
-        double best = lane >= col && lane < e ? fabs(sh.W[lane][col]) : -1.0;
+    for (int col = 0; col < e; ++col) {
+        // partial pivoting on the fp32 image of |W[a][col]| (a >= col), lowest
+        // index on ties; any near-largest pivot is as good numerically
+        const double wl = lane >= col && lane < e ? sh.W[lane][col] : 0.0;
+        float best = lane >= col && lane < e ? (float)fabs(wl) : -1.f;
         int bi = lane;
         for (int off = 16; off; off >>= 1) {
-            const double ob = __shfl_xor_sync(0xffffffffu, best, off);
+            const float ob = __shfl_xor_sync(0xffffffffu, best, off);
             const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
             if (ob > best || (ob == best && oi < bi)) {
                 best = ob;
                 bi = oi;
             }
         }
-        if (!(best > tol)) {   // also catches NaN
+        const double bval = __shfl_sync(0xffffffffu, wl, bi);
+        if (!(fabs(bval) > 0.0) || !isfinite(bval)) {
             singular = 1;
             break;
         }
@@ -116,46 +124,115 @@ __device__ void decode_coefficients(const CodeParams &cp, uint32_t survivors, De
             sh.W[bi][lane] = t;
         }
         __syncwarp();
-        const double rp = 1.0 / sh.W[col][col];
-        double f[kMaxE];
-#pragma unroll
-        for (int a = 0; a < kMaxE; ++a) f[a] = a < e ? sh.W[a][col] * rp : 0.0;
-        __syncwarp();
         if (lane < 2 * e) {
+            // lane owns column `lane`; column `col` of the non-pivot rows becomes 0
+            const double piv = bval;
             const double wc = sh.W[col][lane];
-#pragma unroll
-            for (int a = 0; a < kMaxE; ++a)
-                if (a < e && a != col) sh.W[a][lane] -= f[a] * wc;
+            for (int a = 0; a < e; ++a) {
+                if (a == col) continue;
+                const double fa = sh.W[a][col];      // read before anyone writes it
+                const double wa = sh.W[a][lane];
+                __syncwarp(__activemask());
+                sh.W[a][lane] = lane == col ? 0.0 : piv * wa - fa * wc;
+            }
         }
         __syncwarp();
+    }
+    if (!singular) {
+        // Q^-1[c][a] = W[c][e + a] / W[c][c]
+        const double dinv = lane < e ? 1.0 / sh.W[lane][lane] : 0.0;
+        double qimax = 0.0;
+        for (int t = lane; t < 32 * ((e * e + 31) / 32); t += 32) {
+            const int c = t / e, aa = t % e;
+            const double dc = __shfl_sync(0xffffffffu, dinv, t < e * e ? c : 0);
+            if (t < e * e) {
+                const double q = sh.W[c][e + aa] * dc;
+                sh.Qi[c][aa] = q;
+                qimax = fmax(qimax, fabs(q));
+            }
+        }
+        for (int off = 16; off; off >>= 1)
+            qimax = fmax(qimax, __shfl_xor_sync(0xffffffffu, qimax, off));
+        // ||Q^-1||_inf <= e max|Q^-1|
+        if (!(qnorm * qimax * e < 1.0 / (64.0 * DBL_EPSILON))) singular = 1;
     }
     if (singular) {
         if (lane == 0) sh.singular = 1;
         __syncwarp();
         return;
     }
-    // Q^-1[c][a] = W[c][e + a] / W[c][c]
-    for (int t = lane; t < e * e; t += 32) {
-        const int c = t / e, aa = t % e;
-        sh.Qi[c][aa] = sh.W[c][e + aa] / sh.W[c][c];
-    }
     __syncwarp();
-    // lane p < k builds column p of D (p = position in S)
-    if (lane < k) {
-        const int s = sh.S[lane];
+    // D[c][p] (p = position in S): independent e-term chains, two per lane
+    auto d_entry = [&](int t, double &v) {
+        const int c = t / k, p = t % k;
+        const int s = sh.S[p];
         if (s >= k) {
-            const int aa = __popc(parm & ((1u << s) - 1u));
-            for (int c = 0; c < e; ++c) sh.D[c][lane] = sh.Qi[c][aa];
-        } else {
-            for (int c = 0; c < e; ++c) {
-                double v = 0.0;
-                for (int aa = 0; aa < e; ++aa)
-                    v = fma(-sh.Qi[c][aa], (double)cp.P[(sh.Ps[aa] - k) * k + s], v);
-                sh.D[c][lane] = v;
-            }
+            int aa = 0;
+            while (sh.Ps[aa] != s) ++aa;
+            v = sh.Qi[c][aa];
+            return;
+        }
+        v = 0.0;
+        for (int aa = 0; aa < e; ++aa)
+            v = fma(-sh.Qi[c][aa], (double)cp.P[(sh.Ps[aa] - k) * k + s], v);
+    };
+    for (int t = lane; t < e * k; t += 64) {
+        double v0 = 0.0, v1 = 0.0;
+        const int t1 = t + 32;
+        d_entry(t, v0);
+        if (t1 < e * k) d_entry(t1, v1);
+        for (int q = 0; q < 2; ++q) {
+            const int tt = q ? t1 : t;
+            if (tt >= e * k) break;
+            const double v = q ? v1 : v0;
+            const int c = tt / k, p = tt % k;
+            sh.D[c][p] = v;
+            const float h = __double2float_rn(v);
+            sh.Dh[c][p] = h;
+            sh.Dl[c][p] = __double2float_rn(v - (double)h);
         }
     }
     __syncwarp();
+}
+
+// ---- double-float helpers (fp32 pipe only) -------------------------------------------
+
+// (high, low) fp32 pair of an fp64 value by bit manipulation: high carries the
+// leading 24 significant bits (truncated), low the next 29 rounded to 24;
+// together about 47 bits.  Values outside the fp32 normal range fall back to a
+// rounded conversion (they do not occur for worker results of finite data).
+__device__ __forceinline__ void split_double(double y, float &h, float &l)
+{
+    const unsigned long long b = (unsigned long long)__double_as_longlong(y);
+    const uint32_t hi = (uint32_t)(b >> 32), lo = (uint32_t)b;
+    const int ex = (int)((hi >> 20) & 0x7FF);
+    if (ex < 1023 - 100 || ex > 1023 + 127) {
+        h = __double2float_rn(y);
+        l = 0.f;
+        return;
+    }
+    const uint32_t sign = hi & 0x80000000u;
+    const uint32_t m23 = ((hi & 0xFFFFFu) << 3) | (lo >> 29);
+    h = __int_as_float((int)(sign | ((uint32_t)(ex - 1023 + 127) << 23) | m23));
+    const uint32_t r29 = lo & 0x1FFFFFFFu;
+    // low = r29 * 2^(ex - 1075); below the fp32 normal range it is dropped
+    // (it is then under 2^-100 relative to fp32 precision of |y| >= 2^-75)
+    const int se = ex - 1075 + 127;
+    const float scale = se > 0 ? __int_as_float(se << 23) : 0.f;
+    l = __uint_as_float(sign | __float_as_uint(__uint2float_rn(r29) * scale));
+}
+
+// (sh, sl) += (dh + dl) * (yh + yl), to about 2^-44 relative per term.
+__device__ __forceinline__ void df_fma(float dh, float dl, float yh, float yl, float &sh, float &sl)
+{
+    const float p = dh * yh;
+    const float pe = fmaf(dh, yh, -p);                 // exact error of p
+    const float t = fmaf(dh, yl, dl * yh);             // cross terms
+    const float s1 = sh + p;                           // TwoSum(sh, p)
+    const float bb = s1 - sh;
+    const float err = (sh - (s1 - bb)) + (p - bb);
+    sl += err + (pe + t);
+    sh = s1;
 }
 
 struct DecodeArgs {
@@ -170,40 +247,104 @@ struct DecodeArgs {
     float eta;
 };
 
+constexpr int CG = 2;   // missing blocks decoded per thread
+
+__device__ __forceinline__ void store_out(const DecodeArgs &a, int64_t out, float y_hi, float y_lo)
+{
+    if (a.mode == DEC_PLAIN) {
+        a.Y[out] = y_hi + y_lo;
+    } else if (a.mode == DEC_RESIDUAL) {
+        a.Y[out] = (y_hi - a.lab[out]) + y_lo;          // z = A x - y
+    } else {
+        a.Y[out] = fmaf(-a.eta, y_hi + y_lo, a.Y[out]);  // x -= eta g
+    }
+}
+
 __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a)
 {
     __shared__ DecodeShared sh;
-    if (threadIdx.x < 32) decode_coefficients(a.cp, a.survivors, sh);
+    const int warp = threadIdx.x >> 5;
+    if (warp == 0) decode_select(a.cp, a.survivors, sh);
+    __syncthreads();
+    const int k = a.cp.k, e = sh.e;
+    const int64_t L = a.cp.L, m = a.cp.m;
+    const int b = a.b;
+    const int64_t per_block = L * b;
+    if (warp == 0) {
+        decode_coefficients(a.cp, sh);
+    } else {
+        // meanwhile the other warps pass the surviving systematic blocks
+        // through (exactly rounded to fp32), four independent loads at a time
+        const int64_t npass = (int64_t)(k - e) * per_block;
+        const int64_t stride = (int64_t)gridDim.x * (blockDim.x - 32);
+        for (int64_t it0 = (int64_t)blockIdx.x * (blockDim.x - 32) + threadIdx.x - 32;
+             it0 < npass; it0 += 4 * stride) {
+            double y[4];
+            int64_t out[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int64_t it = it0 + u * stride;
+                out[u] = -1;
+                if (it < npass) {
+                    const int t = (int)(it / per_block);
+                    const int64_t o = (int64_t)sh.S[t] * per_block + (it - (int64_t)t * per_block);
+                    if (o < m * b) {
+                        out[u] = o;
+                        y[u] = a.Yt[o];
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                if (out[u] < 0) continue;
+                if (a.mode == DEC_PLAIN) {
+                    a.Y[out[u]] = __double2float_rn(y[u]);
+                } else {
+                    float yh, yl;
+                    split_double(y[u], yh, yl);
+                    store_out(a, out[u], yh, yl);
+                }
+            }
+        }
+    }
     __syncthreads();
     if (sh.singular) {
         if (threadIdx.x == 0 && a.status) *a.status = CM_ESINGULAR;
         return;
     }
-    const int k = a.cp.k;
-    const int64_t L = a.cp.L, m = a.cp.m;
-    const int b = a.b;
-    const int64_t per_block = L * b;
-    const int64_t total = (int64_t)k * per_block;
-    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < total;
-         it += (int64_t)gridDim.x * blockDim.x) {
-        const int i = (int)(it / per_block);
-        const int64_t rv = it - (int64_t)i * per_block;     // r * b + v within the block
-        const int64_t out = (int64_t)i * per_block + rv;     // row-major index into Y
-        if (out >= m * b) continue;                          // appended zero rows
-        const int c = sh.role[i];
-        double y;
-        if (c < 0) {
-            y = a.Yt[out];                                   // surviving systematic block
-        } else {
-            y = 0.0;
-            for (int p = 0; p < k; ++p) y = fma(sh.D[c][p], a.Yt[(int64_t)sh.S[p] * per_block + rv], y);
+    // missing systematic blocks: up to CG of them per thread, one row position;
+    // the k surviving values are loaded before any arithmetic
+    const int ngroups = (e + CG - 1) / CG;
+    const int64_t ndec = (int64_t)ngroups * per_block;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < ndec; it += stride) {
+        const int g = (int)(it / per_block);
+        const int64_t rv = it - (int64_t)g * per_block;
+        const int c0 = g * CG;
+        double yv[CM_MAX_N];
+#pragma unroll
+        for (int p = 0; p < CM_MAX_N; ++p)
+            if (p < k) yv[p] = a.Yt[(int64_t)sh.S[p] * per_block + rv];
+        float sh_[CG], sl_[CG];
+#pragma unroll
+        for (int c = 0; c < CG; ++c) sh_[c] = sl_[c] = 0.f;
+#pragma unroll
+        for (int p = 0; p < CM_MAX_N; ++p) {
+            if (p < k) {
+                float yh, yl;
+                split_double(yv[p], yh, yl);
+#pragma unroll
+                for (int c = 0; c < CG; ++c)
+                    if (c0 + c < e)
+                        df_fma(sh.Dh[c0 + c][p], sh.Dl[c0 + c][p], yh, yl, sh_[c], sl_[c]);
+            }
         }
-        if (a.mode == DEC_PLAIN) {
-            a.Y[out] = (float)y;
-        } else if (a.mode == DEC_RESIDUAL) {
-            a.Y[out] = (float)(y - (double)a.lab[out]);         // z = A x - y
-        } else {
-            a.Y[out] = (float)((double)a.Y[out] - (double)a.eta * y);   // x -= eta g
+#pragma unroll
+        for (int c = 0; c < CG; ++c) {
+            if (c0 + c < e) {
+                const int64_t out = (int64_t)sh.M[c0 + c] * per_block + rv;
+                if (out < m * b) store_out(a, out, sh_[c], sl_[c]);
+            }
         }
     }
 }
@@ -217,7 +358,11 @@ decode_mat_kernel(const CodeParams cp, const float *Ct, int64_t ldc, uint32_t su
 {
     __shared__ DecodeShared sh;
     __shared__ float Df[kMaxE][CM_MAX_N];
-    if (threadIdx.x < 32) decode_coefficients(cp, survivors, sh);
+    if (threadIdx.x < 32) {
+        decode_select(cp, survivors, sh);
+        __syncwarp();
+        decode_coefficients(cp, sh);
+    }
     __syncthreads();
     if (sh.singular) {
         if (threadIdx.x == 0 && status) *status = CM_ESINGULAR;
@@ -317,7 +462,7 @@ cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survi
     a.mode = mode;
     a.lab = lab;
     a.eta = eta;
-    decode_kernel<<<grid_for((int64_t)cp.k * cp.L * b, 1), kThreads, 0, s>>>(a);
+    decode_kernel<<<grid_for((int64_t)cp.k * cp.L * b / 2 + 1, 2), kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

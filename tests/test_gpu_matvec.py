@@ -202,10 +202,12 @@ def test_singular_generator_sets_status(cm):
     Yt = cm.matvec(code, A, par, X)
     status = torch.zeros(1, dtype=torch.int32, device=DEV)
     Y = torch.full((m, 1), 7.0, device=DEV)
+    L = code.L
     cm.decode(code, Yt, 0b011001, Y=Y, status=status)     # survivors {0, 3, 4}
     torch.cuda.synchronize()
     assert status.item() == cm.CM_ESINGULAR
-    assert torch.all(Y == 7.0)                # nothing written
+    assert torch.all(Y[L:] == 7.0)            # missing blocks 1, 2: not written
+    assert torch.equal(Y[:L], Yt[:L].float()) # surviving block 0 passes through
     P2 = synth.parity_coefficients(n, k)
     P2[2] = 0.0                               # a zero parity row
     code2 = cm.Code(n, k, m, d, P2)

@@ -4,7 +4,7 @@
 // r < L and vector v < b <= 8.  Worker j < k reads its block in place from A
 // (rows past m are virtual zeros); worker j >= k reads the parity buffer.
 //
-// Mapping.  A persistent grid (SMs x one resident CTA of 8 warps).  Work
+// Mapping.  A persistent grid (SMs x one resident CTA of 8 or 16 warps).  Work
 // unit = R consecutive block rows of one worker, owned by one warp; unit u
 // belongs to worker u % n, so consecutive warps stream different workers and
 // all n workers progress together, as the n workers of the protocol do.
@@ -39,8 +39,6 @@
 
 namespace {
 
-constexpr int kWarps = 8;
-constexpr int kThreads = kWarps * 32;
 
 template <int BP>
 struct XCfg {
@@ -53,12 +51,12 @@ struct XCfg {
     static constexpr int FLOATS = BP * GS;
 };
 
-template <int BP, int R, int ST>
+template <int BP, int R, int ST, int W>
 struct Smem {
     static constexpr int SLOT_FLOATS = R * 128;
-    static constexpr int RING_BYTES = kWarps * ST * SLOT_FLOATS * 4;
+    static constexpr int RING_BYTES = W * ST * SLOT_FLOATS * 4;
     static constexpr int X_BYTES = 2 * XCfg<BP>::FLOATS * 4;
-    static constexpr int BAR_BYTES = kWarps * ST * 8;
+    static constexpr int BAR_BYTES = W * ST * 8;
     static constexpr int TOTAL = 1024 + RING_BYTES + X_BYTES + BAR_BYTES;   // + alignment slack
 };
 
@@ -92,7 +90,7 @@ __device__ __forceinline__ void cp_async_wait_all()
 
 // Stage columns [c0, c0 + CX) of X into smem buffer xs as xs[v * GS + col]
 // (zero past d and for padded vectors v >= b).
-template <int BP>
+template <int BP, int kThreads>
 __device__ __forceinline__ void stage_x(const MatvecArgs &a, float *xs, int64_t c0)
 {
     using C = XCfg<BP>;
@@ -178,13 +176,14 @@ __device__ __forceinline__ Unit unit_of(const MatvecArgs &a, int64_t g, int R)
     return u;
 }
 
-template <int BP, int R, int ST, int F>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int BP, int R, int ST, int F, int kWarps>
+__global__ void __launch_bounds__(kWarps * 32, 1)
 matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmP,
               const MatvecArgs a)
 {
+    constexpr int kThreads = kWarps * 32;
     using C = XCfg<BP>;
-    using S = Smem<BP, R, ST>;
+    using S = Smem<BP, R, ST, kWarps>;
     constexpr int V = R * BP;
     constexpr int NH = V >= 32 ? V / 32 : 1;
     constexpr int IPC = C::CX / 128;   // steps per X chunk (a power of two)
@@ -233,7 +232,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     if (lane == 0)
         while (p_idx < my_steps && p_idx < ST) produce();
 
-    stage_x<BP>(a, xs, 0);
+    stage_x<BP, kThreads>(a, xs, 0);
 
     // ---- consumer ----
     int xbuf = 0;             // X buffer of the current chunk
@@ -253,22 +252,24 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
         for (int i = 0; i < NH; ++i) acc64[i] = 0.0;
         int fl = 0;
 #pragma unroll 1
-        for (int s = 0; s < steps; ++s) {
-            const int cs = s & (IPC - 1);
-            if (cs == 0) {
-                cp_async_wait_all();
-                __syncthreads();   // X chunk visible; every warp is done with the other buffer
-                const int ch = s / IPC;
-                if (ch + 1 < nchunks || round + 1 < rounds)
-                    stage_x<BP>(a, xs + (xbuf ^ 1) * C::FLOATS,
-                                ch + 1 < nchunks ? (int64_t)(ch + 1) * C::CX : 0);
-            }
+        for (int ch = 0; ch < nchunks; ++ch) {
+            cp_async_wait_all();
+            __syncthreads();   // X chunk visible; every warp is done with the other buffer
+            if (ch + 1 < nchunks || round + 1 < rounds)
+                stage_x<BP, kThreads>(a, xs + (xbuf ^ 1) * C::FLOATS,
+                                      ch + 1 < nchunks ? (int64_t)(ch + 1) * C::CX : 0);
+            const int ns = steps - ch * IPC < IPC ? steps - ch * IPC : IPC;
             if (has && !failed) {
-                if (!cm_mbar_wait(&bar[slot], phase)) {
-                    failed = true;
-                    if (lane == 0 && a.status) *a.status = CM_ETIMEOUT;
-                } else {
-                    const float *xb = xs + xbuf * C::FLOATS + 4 * (cs * 32 + lane);
+                const float *xchunk = xs + xbuf * C::FLOATS + 4 * lane;
+#pragma unroll
+                for (int cs = 0; cs < IPC; ++cs) {
+                    if (cs >= ns || failed) break;
+                    if (!cm_mbar_wait(&bar[slot], phase)) {
+                        failed = true;
+                        if (lane == 0 && a.status) *a.status = CM_ETIMEOUT;
+                        break;
+                    }
+                    const float *xb = xchunk + cs * 128;
                     const float *ab = ring + slot * S::SLOT_FLOATS + 4 * lane;
                     float2 x01[BP], x23[BP];
 #pragma unroll
@@ -277,16 +278,28 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
                         x01[v] = make_float2(xv.x, xv.y);
                         x23[v] = make_float2(xv.z, xv.w);
                     }
+                    // rows in groups of RH: all even-pair FMAs of the group, then all
+                    // odd-pair ones, so two updates of an accumulator sit RH * BP
+                    // instructions apart
+                    constexpr int RH = R >= 4 ? 4 : R;
 #pragma unroll
-                    for (int r = 0; r < R; ++r) {
-                        const float4 av = *reinterpret_cast<const float4 *>(ab + r * 128);
-                        const float2 a01 = make_float2(av.x, av.y), a23 = make_float2(av.z, av.w);
+                    for (int r0 = 0; r0 < R; r0 += RH) {
+                        float4 av[RH];
 #pragma unroll
-                        for (int v = 0; v < BP; ++v)
-                            acc[r * BP + v] = __ffma2_rn(a01, x01[v], acc[r * BP + v]);
+                        for (int r = 0; r < RH; ++r)
+                            av[r] = *reinterpret_cast<const float4 *>(ab + (r0 + r) * 128);
 #pragma unroll
-                        for (int v = 0; v < BP; ++v)
-                            acc[r * BP + v] = __ffma2_rn(a23, x23[v], acc[r * BP + v]);
+                        for (int r = 0; r < RH; ++r)
+#pragma unroll
+                            for (int v = 0; v < BP; ++v)
+                                acc[(r0 + r) * BP + v] = __ffma2_rn(
+                                    make_float2(av[r].x, av[r].y), x01[v], acc[(r0 + r) * BP + v]);
+#pragma unroll
+                        for (int r = 0; r < RH; ++r)
+#pragma unroll
+                            for (int v = 0; v < BP; ++v)
+                                acc[(r0 + r) * BP + v] = __ffma2_rn(
+                                    make_float2(av[r].z, av[r].w), x23[v], acc[(r0 + r) * BP + v]);
                     }
                     ++c_idx;
                     if (++slot == ST) {
@@ -301,7 +314,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
                     }
                 }
             }
-            if (cs == IPC - 1 || s == steps - 1) xbuf ^= 1;
+            xbuf ^= 1;
         }
         if (has && !failed) {
             if (fl) flush_pairs<V>(acc, acc64, lane);
@@ -337,12 +350,13 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     }
 }
 
-template <int BP, int R, int ST, int F>
+template <int BP, int R, int ST, int F, int kWarps>
 cudaError_t launch_bp(MatvecArgs a, const float *A, int64_t lda, const float *par, int64_t ldp,
                       cudaStream_t s)
 {
-    using S = Smem<BP, R, ST>;
-    auto kern = matvec_kernel<BP, R, ST, F>;
+    constexpr int kThreads = kWarps * 32;
+    using S = Smem<BP, R, ST, kWarps>;
+    auto kern = matvec_kernel<BP, R, ST, F, kWarps>;
     CUtensorMap tmA, tmP;
     if (!cm_make_tmap_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, A, a.d, a.m, lda * 4, 128, R,
                          CU_TENSOR_MAP_SWIZZLE_NONE) ||
@@ -379,7 +393,7 @@ cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, con
     a.b = b;
     a.groups = 0;
     a.fast16 = b == 1 && ((uintptr_t)X & 15u) == 0;
-    if (b == 1) return launch_bp<1, 8, 6, 16>(a, A, lda, par, ldp, s);
-    if (b <= 4) return launch_bp<4, 8, 6, 16>(a, A, lda, par, ldp, s);
-    return launch_bp<8, 8, 6, 16>(a, A, lda, par, ldp, s);
+    if (b == 1) return launch_bp<1, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
+    if (b <= 4) return launch_bp<4, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
+    return launch_bp<8, 8, 6, 64, 8>(a, A, lda, par, ldp, s);
 }

@@ -96,6 +96,18 @@ cm_status cm_matvec(const cm_code *code, const float *A, int64_t lda,
                     const float *parity, int64_t ldp, const float *X, int32_t b,
                     double *Yt, int32_t *dev_status, cm_stream_t stream);
 
+/* cm_matvec restricted to the survivors: when the straggler set is known
+ * before the products run, only the workers that cm_decode will read (the
+ * first k set bits of `survivors`) are computed, saving (n-k)/n of the reads
+ * (the MDS run ends at the k-th arrival, eq. for the MDS runtime, so the
+ * stragglers' work is never used).  Rows of the other workers in Yt are left
+ * unwritten.  Same layout, precision and errors as cm_matvec; fewer than k
+ * survivors returns CM_ENOTDECODABLE. */
+cm_status cm_matvec_survivors(const cm_code *code, const float *A, int64_t lda,
+                              const float *parity, int64_t ldp, const float *X, int32_t b,
+                              uint32_t survivors, double *Yt, int32_t *dev_status,
+                              cm_stream_t stream);
+
 /* Straggler draw (Sec. III-C, III-D; eq. for the MDS runtime).  Host only.
  * Worker j's time in round `counter` is T_j = (shift + E_j / rate) / k with
  * E_j = -log(1 - U_j), U_j = (z_j >> 11) 2^-53, z_j the SplitMix64 output

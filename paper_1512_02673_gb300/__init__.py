@@ -56,6 +56,7 @@ def lib() -> ctypes.CDLL:
             "cm_block_rows": (i64, [vp]),
             "cm_encode": (st, [vp, vp, i64, vp, i64, vp, vp]),
             "cm_matvec": (st, [vp, vp, i64, vp, i64, vp, i32, vp, vp, vp]),
+            "cm_matvec_survivors": (st, [vp, vp, i64, vp, i64, vp, i32, u32, vp, vp, vp]),
             "cm_draw_erasures": (st, [u64, u64, i32, i32, f64, f64, ctypes.POINTER(u32), vp]),
             "cm_decode": (st, [vp, vp, u32, i32, vp, vp, vp]),
             "cm_gd_workspace_bytes": (sz, [vp, vp]),
@@ -194,6 +195,33 @@ def matvec(code: Code, A: torch.Tensor, parity: torch.Tensor, X: torch.Tensor,
     _check(lib().cm_matvec(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
                            _ld(parity, "parity"), X.data_ptr(), b, Yt.data_ptr(), sp,
                            _stream()), "cm_matvec")
+    return Yt
+
+
+def matvec_survivors(code: Code, A: torch.Tensor, parity: torch.Tensor, X: torch.Tensor,
+                     survivors: int, Yt: torch.Tensor | None = None,
+                     status: torch.Tensor | None = None) -> torch.Tensor:
+    """Worker products of the k survivors only (the other rows of Yt untouched)."""
+    _dev(A, torch.float32, "A", 2)
+    _dev(parity, torch.float32, "parity", 2)
+    if X.dim() == 1:
+        X = X.view(-1, 1)
+    _dev(X, torch.float32, "X", 2)
+    _contig(X, "X")
+    b = X.shape[1]
+    if Yt is None:
+        Yt = torch.empty((code.n * code.L, b), dtype=torch.float64, device=X.device)
+    _dev(Yt, torch.float64, "Yt", 2)
+    _contig(Yt, "Yt")
+    if tuple(Yt.shape) != (code.n * code.L, b) or X.shape[0] != code.d:
+        raise ValueError("shapes: X must be d x b and Yt n L x b")
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
+    _check(lib().cm_matvec_survivors(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
+                                     _ld(parity, "parity"), X.data_ptr(), b, survivors,
+                                     Yt.data_ptr(), sp, _stream()), "cm_matvec_survivors")
     return Yt
 
 

@@ -100,8 +100,22 @@ cm_status cm_matvec(const cm_code *c, const float *A, int64_t lda, const float *
     if (b < 1 || b > 8 || !X || !Yt) return CM_EINVAL;
     if (!layout_ok(A, lda, c->d, 4) || !layout_ok(par, ldp, c->d, 4)) return CM_EINVAL;
     if (((uintptr_t)X & 3u) || ((uintptr_t)Yt & 7u)) return CM_EINVAL;
-    return from_cuda(launch_matvec(code_params(c), A, lda, par, ldp, X, b, Yt, dev_status,
+    return from_cuda(launch_matvec(code_params(c), A, lda, par, ldp, X, b, Yt, dev_status, 0u,
                                    (cudaStream_t)stream));
+}
+
+cm_status cm_matvec_survivors(const cm_code *c, const float *A, int64_t lda, const float *par,
+                              int64_t ldp, const float *X, int32_t b, uint32_t survivors,
+                              double *Yt, int32_t *dev_status, cm_stream_t stream)
+{
+    if (!c || c->dt != CM_F32) return CM_EINVAL;
+    cm_status st = check_survivors(c, survivors);
+    if (st != CM_OK) return st;
+    if (b < 1 || b > 8 || !X || !Yt) return CM_EINVAL;
+    if (!layout_ok(A, lda, c->d, 4) || !layout_ok(par, ldp, c->d, 4)) return CM_EINVAL;
+    if (((uintptr_t)X & 3u) || ((uintptr_t)Yt & 7u)) return CM_EINVAL;
+    return from_cuda(launch_matvec(code_params(c), A, lda, par, ldp, X, b, Yt, dev_status,
+                                   survivors, (cudaStream_t)stream));
 }
 
 cm_status cm_decode(const cm_code *c, const double *Yt, uint32_t survivors, int32_t b,
@@ -156,13 +170,13 @@ cm_status cm_gd_step(const cm_code *cA, const float *A, int64_t lda, const float
     cudaStream_t s = (cudaStream_t)stream;
     CodeParams pA = code_params(cA), pAT = code_params(cAT);
     // Sec. III-E: the master multicasts x, decodes A x from any k1 results ...
-    if (launch_matvec(pA, A, lda, PA, ldpa, x, 1, ytA, dev_status, s) != cudaSuccess)
+    if (launch_matvec(pA, A, lda, PA, ldpa, x, 1, ytA, dev_status, 0u, s) != cudaSuccess)
         return CM_ECUDA;
     // ... forms z = A x - y and multicasts it ...
     if (launch_decode(pA, ytA, surv_A, 1, z, dev_status, DEC_RESIDUAL, y, 0.f, s) != cudaSuccess)
         return CM_ECUDA;
     // ... decodes A^T z from any k2 results and steps x <- x - eta A^T z.
-    if (launch_matvec(pAT, AT, ldat, PAT, ldpat, z, 1, ytAT, dev_status, s) != cudaSuccess)
+    if (launch_matvec(pAT, AT, ldat, PAT, ldpat, z, 1, ytAT, dev_status, 0u, s) != cudaSuccess)
         return CM_ECUDA;
     if (launch_decode(pAT, ytAT, surv_AT, 1, x, dev_status, DEC_DESCENT, nullptr, eta, s) !=
         cudaSuccess)

@@ -44,9 +44,10 @@ cudaError_t launch_encode_f32(const CodeParams &cp, const float *A, int64_t lda,
                               float *par, int64_t ldp, int32_t *status, cudaStream_t s);
 cudaError_t launch_encode_bf16(const CodeParams &cp, const uint16_t *A, int64_t lda,
                                uint16_t *par, int64_t ldp, int32_t *status, cudaStream_t s);
+// `only` = 0: all n workers; otherwise the workers of the first k set bits.
 cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda,
                           const float *par, int64_t ldp, const float *X, int b,
-                          double *Yt, int32_t *status, cudaStream_t s);
+                          double *Yt, int32_t *status, uint32_t only, cudaStream_t s);
 
 // Decode epilogues (Sec. III-E: the two decodes of a gradient step).
 enum DecodeMode { DEC_PLAIN = 0, DEC_RESIDUAL = 1, DEC_DESCENT = 2 };

@@ -6,8 +6,10 @@
 //
 // Mapping.  A persistent grid (SMs x one resident CTA of 8 or 16 warps).  Work
 // unit = R consecutive block rows of one worker, owned by one warp; unit u
-// belongs to worker u % n, so consecutive warps stream different workers and
-// all n workers progress together, as the n workers of the protocol do.
+// belongs to the (u % nw)-th computed worker, so consecutive warps stream
+// different workers and all workers progress together, as the n workers of
+// the protocol do.  Normally all n workers are computed; when the survivors
+// are known beforehand only those k are (the others' rows stay unwritten).
 //
 // Data movement.  The unit's rows stream through a per-warp ring of ST
 // shared-memory slots, one 2-D TMA box (R rows x 128 columns) per step issued
@@ -68,6 +70,8 @@ struct MatvecArgs {
     int32_t n, k, b;
     int32_t fast16;        // X chunks may be staged with 16-byte copies (b == 1)
     int64_t groups;        // total work units
+    int32_t nw;            // workers computed: all n, or only the k survivors
+    int8_t wmap[CM_MAX_N]; // computed worker slot -> worker index
 };
 
 __device__ __forceinline__ void cp_async16(float *dst, const float *src, int bytes)
@@ -169,8 +173,8 @@ struct Unit {
 __device__ __forceinline__ Unit unit_of(const MatvecArgs &a, int64_t g, int R)
 {
     Unit u;
-    u.j = (int)(g % a.n);
-    u.rr0 = (g / a.n) * R;
+    u.j = a.wmap[g % a.nw];
+    u.rr0 = (g / a.nw) * R;
     u.parity = u.j >= a.k;
     u.y = (int32_t)(u.parity ? (int64_t)(u.j - a.k) * a.L + u.rr0 : (int64_t)u.j * a.L + u.rr0);
     return u;
@@ -366,7 +370,7 @@ cudaError_t launch_bp(MatvecArgs a, const float *A, int64_t lda, const float *pa
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          S::TOTAL);
     if (e != cudaSuccess) return e;
-    a.groups = (a.L + R - 1) / R * a.n;
+    a.groups = (a.L + R - 1) / R * a.nw;
     const int64_t need = (a.groups + kWarps - 1) / kWarps;
     int64_t grid = cm_sm_count();
     if (grid < 1) grid = 1;
@@ -379,9 +383,13 @@ cudaError_t launch_bp(MatvecArgs a, const float *A, int64_t lda, const float *pa
 
 cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, const float *par,
                           int64_t ldp, const float *X, int b, double *Yt, int32_t *status,
-                          cudaStream_t s)
+                          uint32_t only, cudaStream_t s)
 {
     MatvecArgs a;
+    // workers to compute: all n, or the first k set bits of `only`
+    a.nw = 0;
+    for (int j = 0; j < cp.n; ++j)
+        if (!only || (((only >> j) & 1u) && a.nw < cp.k)) a.wmap[a.nw++] = (int8_t)j;
     a.X = X;
     a.Yt = Yt;
     a.status = status;

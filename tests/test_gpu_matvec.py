@@ -360,3 +360,25 @@ def test_bounded_wait_gives_up_and_reports(cm):
     assert status.item() == 0
     want = (A.double() @ X.double()).cpu().numpy()
     assert np.linalg.norm(Y.double().cpu().numpy() - want) <= 1e-5 * np.linalg.norm(want)
+
+
+@pytest.mark.parametrize("n,k,m,d,b", [(10, 5, 2003, 1029, 1), (32, 24, 1000, 640, 8), (6, 3, 37, 130, 3)])
+def test_survivors_only_products(cm, orc, n, k, m, d, b):
+    """Survivors-only mode computes exactly the rows decode reads, leaves the
+    stragglers' rows untouched, and decodes to the same A X."""
+    r = run_path(cm, orc, n, k, m, d, b, lda=(d + 3) // 4 * 4)
+    L = r["code"].L
+    for counter in range(3):
+        mask, _ = cm.draw_erasures(synth.ERASURE_SEED, 50 + counter, n, k)
+        Yt = torch.full((n * L, b), 12345.0, dtype=torch.float64, device=DEV)
+        cm.matvec_survivors(r["code"], r["A"], r["par"], r["X"], mask, Yt=Yt)
+        Y = cm.decode(r["code"], Yt, mask)
+        torch.cuda.synchronize()
+        for j in range(n):
+            blk = slice(j * L, (j + 1) * L)
+            if mask >> j & 1:
+                assert torch.equal(Yt[blk], r["Yt"][blk]), j   # same kernel, same sums
+            else:
+                assert torch.all(Yt[blk] == 12345.0), j        # never written
+        want = orc.matmul(r["A_cpu"].numpy(), r["X_cpu"].numpy())
+        assert rel_l2_cols(Y.cpu().numpy(), want).max() <= 1e-4

@@ -399,7 +399,8 @@ def run_ours(args, world, rank, local):
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk.summary(),
         "secondary": {"survivors_only": so, "gemm": gemm, "gd": gd,
-                      "matvec_100_repeats": mv100, "tiny": tiny},
+                      "matvec_100_repeats": mv100, "tiny": tiny,
+                      "runtime_model": runtime_model_report(cm)},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w)
@@ -430,6 +431,27 @@ def bench_survivors_only(cm, code, A, parity, X, Yt, Y, status, w, args) -> dict
     read = w.k * L * w.d * 4 + w.d * w.b * 4 + w.k * L * w.b * 8
     return {"matvec_ms": mv, "decode_ms": dec, "matvec_gbs": read / (mv * 1e-3) / 1e9,
             "bytes_read": read, "status": int(status.item())}
+
+
+def runtime_model_report(cm) -> dict:
+    """The straggler model of the paper for the bench's codes: expected overall
+    runtime (units of the single-machine job) of uncoded, repetition and MDS
+    schemes, the simulated MDS mean over the bench's draws, and the optimal k."""
+    out = {}
+    for name, n, k in [("(32,24)", 32, 24), ("(10,5)", 10, 5), ("(20,10)", 20, 10),
+                       ("(16,12)", 16, 12)]:
+        r = {"uncoded": cm.runtime_mean("uncoded", n, n),
+             "mds": cm.runtime_mean("mds", n, k)}
+        if n % k == 0:
+            r["repetition"] = cm.runtime_mean("repetition", n, k)
+        sim = cm.runtime_simulate("mds", n, k, 100000, seed=synth.ERASURE_SEED)
+        r["mds_simulated_mean"] = float(sim.mean())
+        r["mds_simulated_p95"] = float(np.percentile(sim, 95))
+        ks, g = cm.optimal_mds_k(n, 1.0)
+        r["k_star"], r["gamma_star"] = ks, g
+        r["uncoded_over_mds"] = r["uncoded"] / r["mds"]
+        out[name] = r
+    return out
 
 
 def bench_gd(cm, dev, steps: int) -> dict:

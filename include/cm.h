@@ -70,6 +70,21 @@ cm_status cm_code_create(int32_t n, int32_t k, int64_t m, int64_t d, cm_dtype dt
                          const float *parity_host, cm_code **out);
 void cm_code_destroy(cm_code *code);
 
+/* The n/k-repetition code of Sec. III-B (Example "Repetition codes"): every
+ * data block is replicated n/k times; worker j holds block j mod k (workers
+ * j < k are the systematic copies), i.e. P[p][i] = 1 if i == p mod k else 0.
+ * Requires n % k == 0.  Its decodable sets are the products of the replica
+ * groups {i, i+k, i+2k, ...}: decoding uses the lowest surviving replica of
+ * each block.  No CUDA call. */
+cm_status cm_code_create_repetition(int32_t n, int32_t k, int64_t m, int64_t d, cm_dtype dt,
+                                    cm_code **out);
+
+/* The k workers a decode of this code uses for the given survivor mask:
+ * the first k set bits for a general (MDS) code, the lowest surviving
+ * replica of each block for a repetition code.  CM_ENOTDECODABLE when the
+ * survivors hold no decodable set. */
+cm_status cm_select_decodable(const cm_code *code, uint32_t survivors, uint32_t *selected);
+
 /* L = ceil(m / k), the rows per block after zero padding (Sec. III-A
  * footnote); -1 for a NULL code. */
 int64_t cm_block_rows(const cm_code *code);
@@ -219,6 +234,40 @@ cm_status cm_matmat(const cm_code *code, const void *A, int64_t lda,
  * after limit_ns nanoseconds (1 .. 2e9); the kernel then writes CM_ETIMEOUT
  * to *dev_status and returns, and the context stays usable. */
 cm_status cm_selftest_bounded_wait(int32_t *dev_status, uint64_t limit_ns, cm_stream_t stream);
+
+/* ---- runtime model (Sec. III-B, III-C, III-D), host only ----------------
+ * A job split k ways runs each task for T = (shift + E / rate) / k, E ~ Exp(1)
+ * (the shifted-exponential mother distribution F(t) = 1 - e^{-rate (t - shift)}
+ * scaled by the split, P(T <= t) = F(k t)).  The overall runtime is the max of
+ * the n tasks for an uncoded job (split n ways, eq. for the uncoded runtime),
+ * the max over blocks of the min over replicas for an n/k-repetition code
+ * (eq. for the repetition runtime), and the k-th arrival for an (n,k) MDS
+ * code (eq. for the MDS runtime). */
+typedef enum { CM_SCHEME_UNCODED = 0, CM_SCHEME_REPETITION = 1, CM_SCHEME_MDS = 2 } cm_scheme;
+
+/* Expected overall runtime, exact harmonic-number form of Sec. III-D:
+ * uncoded (shift + H_n/rate)/n; repetition (shift + (k/n) H_k/rate)/k;
+ * MDS (shift + (H_n - H_{n-k})/rate)/k.  k is ignored for the uncoded
+ * scheme; repetition needs n % k == 0. */
+cm_status cm_runtime_mean(cm_scheme scheme, int32_t n, int32_t k, double shift, double rate,
+                          double *mean);
+
+/* Distribution P(T_overall <= t) at `count` points (eqs. for F_uncoded,
+ * F_rep and F_MDS; the MDS one as the binomial tail equal to its integral
+ * form). */
+cm_status cm_runtime_cdf(cm_scheme scheme, int32_t n, int32_t k, double shift, double rate,
+                         const double *t, int64_t count, double *F);
+
+/* Monte-Carlo overall runtimes of `count` rounds (counters counter0 ..),
+ * drawn exactly as cm_draw_erasures draws worker times (n <= 32). */
+cm_status cm_runtime_simulate(cm_scheme scheme, int32_t n, int32_t k, double shift, double rate,
+                              uint64_t seed, uint64_t counter0, int64_t count, double *T);
+
+/* Lemma on optimal MDS-coded algorithms: k* = (1 + 1/W_{-1}(-e^{-rate-1})) n
+ * minimises the expected MDS runtime (log form of the harmonic numbers), and
+ * n T* = gamma* = -W_{-1}(-e^{-rate-1}) / rate (W_{-1}: the lower branch of
+ * the Lambert W function). */
+cm_status cm_optimal_mds_k(int32_t n, double rate, double *k_star, double *gamma_star);
 
 /* Static description of a status code. */
 const char *cm_status_string(cm_status s);

@@ -72,6 +72,8 @@ def _load():
             "or_decode": (ctypes.c_int, [i32, i32, i64, i64, vp, u32, vp, vp]),
             "or_generator_inverse": (ctypes.c_int, [i32, i32, vp, u32, vp]),
             "or_gd": (ctypes.c_int, [i64, i64, vp, i64, vp, f64, i32, vp]),
+            "or_runtime_simulate": (ctypes.c_int, [i32, i32, i32, f64, f64, u64, u64, i64, vp]),
+            "or_repetition_select": (ctypes.c_int, [i32, i32, u32, ctypes.POINTER(u32)]),
         }
         for name, (res, args) in sig.items():
             f = getattr(lib, name)
@@ -234,3 +236,30 @@ def gd(A, y, eta: float, iters: int, x0=None) -> np.ndarray:
     x = np.zeros(d, np.float64) if x0 is None else _f64(x0).copy()
     _check(_load().or_gd(m, d, _ptr(A), d, _ptr(y), eta, iters, _ptr(x)))
     return x
+
+
+SCHEMES = {"uncoded": 0, "repetition": 1, "mds": 2}
+
+
+def runtime_simulate(scheme: str, n: int, k: int, shift: float, rate: float, seed: int,
+                     counter0: int, count: int) -> np.ndarray:
+    """Monte-Carlo overall runtimes (Sec. III-B/C/D) from the straggler draws."""
+    T = np.empty(count, np.float64)
+    _check(_load().or_runtime_simulate(SCHEMES[scheme], n, k, shift, rate, seed, counter0,
+                                       count, _ptr(T)))
+    return T
+
+
+def repetition_select(n: int, k: int, survivors: int) -> int:
+    """Decodable set of an n/k-repetition code: lowest surviving replica per block."""
+    sel = ctypes.c_uint32(0)
+    _check(_load().or_repetition_select(n, k, survivors, ctypes.byref(sel)))
+    return int(sel.value)
+
+
+def repetition_parity(n: int, k: int) -> np.ndarray:
+    """P of the n/k-repetition code in systematic form: worker k + p copies block p mod k."""
+    P = np.zeros((n - k, k))
+    for p in range(n - k):
+        P[p, p % k] = 1.0
+    return P

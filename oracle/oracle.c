@@ -461,3 +461,72 @@ int or_gd(int64_t m, int64_t d, const float *A, int64_t lda, const float *y,
     free(g);
     return 0;
 }
+
+/* ---- runtime model (Sec. III-B, III-C, III-D) ---------------------------------
+ * Overall runtime of one round under the shifted-exponential model, from the
+ * same worker draws as or_draw_erasures.  scheme 0: uncoded, the job split n
+ * ways and the round ends with the last task (eq. for the uncoded runtime);
+ * scheme 1: n/k-repetition, block i held by workers i, i+k, i+2k, ... and the
+ * round ends when every block has one finished replica (eq. for the
+ * repetition runtime); scheme 2: (n,k) MDS, the round ends at the k-th
+ * arrival (eq. for the MDS runtime).  Writes `count` runtimes. */
+int or_runtime_simulate(int32_t scheme, int32_t n, int32_t k, double shift, double rate,
+                        uint64_t seed, uint64_t counter0, int64_t count, double *T)
+{
+    if (n < 1 || n > 32 || !(rate > 0.0) || scheme < 0 || scheme > 2) return -1;
+    if (scheme != 0 && (k < 1 || k > n)) return -1;
+    if (scheme == 1 && n % k) return -1;
+    int32_t split = scheme == 0 ? n : k;
+    for (int64_t c = 0; c < count; ++c) {
+        double t[32];
+        for (int32_t j = 0; j < n; ++j) {
+            uint64_t z = or_splitmix64(seed, (counter0 + (uint64_t)c) * (uint64_t)n + (uint64_t)j + 1);
+            double u = (double)(z >> 11) * 0x1.0p-53;
+            t[j] = (shift - log1p(-u) / rate) / (double)split;
+        }
+        double r;
+        if (scheme == 0) {
+            r = t[0];
+            for (int32_t j = 1; j < n; ++j) if (t[j] > r) r = t[j];
+        } else if (scheme == 1) {
+            r = 0.0;
+            for (int32_t i = 0; i < k; ++i) {
+                double g = t[i];
+                for (int32_t j = i + k; j < n; j += k) if (t[j] < g) g = t[j];
+                if (g > r) r = g;
+            }
+        } else {
+            /* k-th smallest by counting: the time with exactly k-1 smaller ones */
+            r = 0.0;
+            for (int32_t j = 0; j < n; ++j) {
+                int32_t below = 0, tie = 0;
+                for (int32_t i = 0; i < n; ++i) {
+                    if (t[i] < t[j]) ++below;
+                    else if (t[i] == t[j] && i < j) ++tie;
+                }
+                if (below + tie == k - 1) r = t[j];
+            }
+        }
+        T[c] = r;
+    }
+    return 0;
+}
+
+/* Example "Repetition codes": the decodable sets of an n/k-repetition code are
+ * the products of the replica groups; this picks, for every block i, the
+ * lowest surviving worker among i, i+k, i+2k, ...  Returns -2 if some block
+ * has no surviving replica. */
+int or_repetition_select(int32_t n, int32_t k, uint32_t survivors, uint32_t *selected)
+{
+    if (k < 1 || n <= k || n > 32 || n % k) return -1;
+    uint32_t sel = 0;
+    for (int32_t i = 0; i < k; ++i) {
+        int32_t pick = -1;
+        for (int32_t j = i; j < n && pick < 0; j += k)
+            if (survivors & (1u << j)) pick = j;
+        if (pick < 0) return -2;
+        sel |= 1u << pick;
+    }
+    *selected = sel;
+    return 0;
+}

@@ -70,6 +70,12 @@ def lib() -> ctypes.CDLL:
                                vp, vp]),
             "cm_selftest_bounded_wait": (st, [vp, u64, vp]),
             "cm_status_string": (ctypes.c_char_p, [st]),
+            "cm_code_create_repetition": (st, [i32, i32, i64, i64, st, ctypes.POINTER(vp)]),
+            "cm_select_decodable": (st, [vp, u32, ctypes.POINTER(u32)]),
+            "cm_runtime_mean": (st, [st, i32, i32, f64, f64, ctypes.POINTER(f64)]),
+            "cm_runtime_cdf": (st, [st, i32, i32, f64, f64, vp, i64, vp]),
+            "cm_runtime_simulate": (st, [st, i32, i32, f64, f64, u64, u64, i64, vp]),
+            "cm_optimal_mds_k": (st, [i32, f64, ctypes.POINTER(f64), ctypes.POINTER(f64)]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -115,16 +121,26 @@ def _contig(t: torch.Tensor, name: str):
 
 
 class Code:
-    """An (n,k) systematic code G = [I_k; P] for an m x d data matrix."""
+    """An (n,k) systematic code G = [I_k; P] for an m x d data matrix.
+
+    parity="repetition" builds the n/k-repetition code (worker j holds block
+    j mod k); otherwise parity is the (n-k) x k block P."""
 
     def __init__(self, n: int, k: int, m: int, d: int, parity, dtype: str = "f32"):
-        P = np.ascontiguousarray(np.asarray(parity, dtype=np.float32))
-        if P.shape != (n - k, k):
-            raise ValueError("parity must be (n-k) x k")
         dt = {"f32": CM_F32, "bf16": CM_BF16}[dtype]
         out = ctypes.c_void_p()
-        _check(lib().cm_code_create(n, k, m, d, dt, P.ctypes.data_as(ctypes.c_void_p),
-                                    ctypes.byref(out)), "cm_code_create")
+        if isinstance(parity, str) and parity == "repetition":
+            _check(lib().cm_code_create_repetition(n, k, m, d, dt, ctypes.byref(out)),
+                   "cm_code_create_repetition")
+            P = np.zeros((n - k, k), np.float32)
+            for p in range(n - k):
+                P[p, p % k] = 1.0
+        else:
+            P = np.ascontiguousarray(np.asarray(parity, dtype=np.float32))
+            if P.shape != (n - k, k):
+                raise ValueError("parity must be (n-k) x k")
+            _check(lib().cm_code_create(n, k, m, d, dt, P.ctypes.data_as(ctypes.c_void_p),
+                                        ctypes.byref(out)), "cm_code_create")
         self._h = out
         self.n, self.k, self.m, self.d, self.dtype = n, k, m, d, dtype
         self.P = P
@@ -133,6 +149,13 @@ class Code:
     @property
     def handle(self):
         return self._h
+
+    def select_decodable(self, survivors: int) -> int:
+        """The k workers a decode uses for this survivor mask (bitmask)."""
+        sel = ctypes.c_uint32(0)
+        _check(lib().cm_select_decodable(self._h, survivors, ctypes.byref(sel)),
+               "cm_select_decodable")
+        return int(sel.value)
 
     def __del__(self):
         h = getattr(self, "_h", None)
@@ -375,3 +398,44 @@ def matmat(code: Code, A, parity, Bt, survivors: int, Ct=None, C=None, status=No
                            Ct.data_ptr(), _ld(Ct, "Ct"), survivors, C.data_ptr(),
                            _ld(C, "C"), sp, _stream()), "cm_matmat")
     return Ct, C
+
+
+# ---- runtime model (Sec. III-B, III-C, III-D) ----------------------------------
+
+SCHEMES = {"uncoded": 0, "repetition": 1, "mds": 2}
+
+
+def runtime_mean(scheme: str, n: int, k: int, shift: float = 1.0, rate: float = 1.0) -> float:
+    """Expected overall runtime (exact harmonic form) of an uncoded,
+    n/k-repetition or (n,k)-MDS coded job under the shifted exponential."""
+    out = ctypes.c_double(0.0)
+    _check(lib().cm_runtime_mean(SCHEMES[scheme], n, k, shift, rate, ctypes.byref(out)),
+           "cm_runtime_mean")
+    return float(out.value)
+
+
+def runtime_cdf(scheme: str, n: int, k: int, t, shift: float = 1.0, rate: float = 1.0):
+    """P(T_overall <= t) at the points t."""
+    t = np.ascontiguousarray(np.asarray(t, dtype=np.float64).ravel())
+    F = np.empty_like(t)
+    _check(lib().cm_runtime_cdf(SCHEMES[scheme], n, k, shift, rate,
+                                t.ctypes.data_as(ctypes.c_void_p), t.size,
+                                F.ctypes.data_as(ctypes.c_void_p)), "cm_runtime_cdf")
+    return F
+
+
+def runtime_simulate(scheme: str, n: int, k: int, count: int, seed: int, counter0: int = 0,
+                     shift: float = 1.0, rate: float = 1.0):
+    """Monte-Carlo overall runtimes from the straggler draws of draw_erasures."""
+    T = np.empty(count, np.float64)
+    _check(lib().cm_runtime_simulate(SCHEMES[scheme], n, k, shift, rate, seed, counter0, count,
+                                     T.ctypes.data_as(ctypes.c_void_p)), "cm_runtime_simulate")
+    return T
+
+
+def optimal_mds_k(n: int, rate: float = 1.0):
+    """(k*, gamma*) of the lemma on optimal MDS-coded algorithms (Lambert W)."""
+    ks, g = ctypes.c_double(0.0), ctypes.c_double(0.0)
+    _check(lib().cm_optimal_mds_k(n, rate, ctypes.byref(ks), ctypes.byref(g)),
+           "cm_optimal_mds_k")
+    return float(ks.value), float(g.value)

@@ -18,13 +18,44 @@ int popcount32(uint32_t x)
 
 cm_status from_cuda(cudaError_t e) { return e == cudaSuccess ? CM_OK : CM_ECUDA; }
 
-// Survivor mask checks shared by the decoders: no bit at or above n, and at
-// least k survivors (Example "MDS codes": any k results are decodable).
-cm_status check_survivors(const cm_code *c, uint32_t survivors)
+// The k workers a decode uses (written to *eff).  A general code decodes
+// from any k results (Example "MDS codes"): the first k set bits.  A
+// repetition code decodes from one result per block (Example "Repetition
+// codes"): the lowest surviving replica of each block.
+cm_status resolve_survivors(const cm_code *c, uint32_t survivors, uint32_t *eff)
 {
     if (c->n < 32 && (survivors >> c->n)) return CM_EINVAL;
+    if (c->kind == CODE_REPETITION) {
+        uint32_t sel = 0;
+        for (int i = 0; i < c->k; ++i) {
+            int pick = -1;
+            for (int j = i; j < c->n; j += c->k)
+                if ((survivors >> j) & 1u) {
+                    pick = j;
+                    break;
+                }
+            if (pick < 0) return CM_ENOTDECODABLE;
+            sel |= 1u << pick;
+        }
+        *eff = sel;
+        return CM_OK;
+    }
     if (popcount32(survivors) < c->k) return CM_ENOTDECODABLE;
+    uint32_t sel = 0;
+    int cnt = 0;
+    for (int j = 0; j < c->n && cnt < c->k; ++j)
+        if ((survivors >> j) & 1u) {
+            sel |= 1u << j;
+            ++cnt;
+        }
+    *eff = sel;
     return CM_OK;
+}
+
+cm_status check_survivors(const cm_code *c, uint32_t survivors)
+{
+    uint32_t eff;
+    return resolve_survivors(c, survivors, &eff);
 }
 
 // Operand layout checks: base 16-byte aligned, leading dimension >= d and a
@@ -69,9 +100,30 @@ cm_status cm_code_create(int32_t n, int32_t k, int64_t m, int64_t d, cm_dtype dt
     c->d = d;
     c->L = (m + k - 1) / k;   // zero rows appended up to k L (Sec. III-A footnote)
     c->dt = dt;
+    c->kind = CODE_GENERAL;
     std::memcpy(c->P, parity_host, sizeof(float) * (n - k) * k);
     *out = c;
     return CM_OK;
+}
+
+cm_status cm_code_create_repetition(int32_t n, int32_t k, int64_t m, int64_t d, cm_dtype dt,
+                                    cm_code **out)
+{
+    if (!out) return CM_EINVAL;
+    *out = nullptr;
+    if (k < 1 || n <= k || n > CM_MAX_N || n % k != 0) return CM_EINVAL;
+    float P[CM_MAX_P];
+    for (int p = 0; p < n - k; ++p)
+        for (int i = 0; i < k; ++i) P[p * k + i] = (i == p % k) ? 1.f : 0.f;
+    cm_status st = cm_code_create(n, k, m, d, dt, P, out);
+    if (st == CM_OK) (*out)->kind = CODE_REPETITION;
+    return st;
+}
+
+cm_status cm_select_decodable(const cm_code *c, uint32_t survivors, uint32_t *selected)
+{
+    if (!c || !selected) return CM_EINVAL;
+    return resolve_survivors(c, survivors, selected);
 }
 
 void cm_code_destroy(cm_code *code) { std::free(code); }
@@ -109,23 +161,25 @@ cm_status cm_matvec_survivors(const cm_code *c, const float *A, int64_t lda, con
                               double *Yt, int32_t *dev_status, cm_stream_t stream)
 {
     if (!c || c->dt != CM_F32) return CM_EINVAL;
-    cm_status st = check_survivors(c, survivors);
+    uint32_t eff;
+    cm_status st = resolve_survivors(c, survivors, &eff);
     if (st != CM_OK) return st;
     if (b < 1 || b > 8 || !X || !Yt) return CM_EINVAL;
     if (!layout_ok(A, lda, c->d, 4) || !layout_ok(par, ldp, c->d, 4)) return CM_EINVAL;
     if (((uintptr_t)X & 3u) || ((uintptr_t)Yt & 7u)) return CM_EINVAL;
     return from_cuda(launch_matvec(code_params(c), A, lda, par, ldp, X, b, Yt, dev_status,
-                                   survivors, (cudaStream_t)stream));
+                                   eff, (cudaStream_t)stream));
 }
 
 cm_status cm_decode(const cm_code *c, const double *Yt, uint32_t survivors, int32_t b,
                     float *Y, int32_t *dev_status, cm_stream_t stream)
 {
     if (!c) return CM_EINVAL;
-    cm_status st = check_survivors(c, survivors);
+    uint32_t eff;
+    cm_status st = resolve_survivors(c, survivors, &eff);
     if (st != CM_OK) return st;
     if (b < 1 || !Yt || !Y || ((uintptr_t)Yt & 7u) || ((uintptr_t)Y & 3u)) return CM_EINVAL;
-    return from_cuda(launch_decode(code_params(c), Yt, survivors, b, Y, dev_status,
+    return from_cuda(launch_decode(code_params(c), Yt, eff, b, Y, dev_status,
                                    DEC_PLAIN, nullptr, 0.f, (cudaStream_t)stream));
 }
 
@@ -149,9 +203,10 @@ cm_status cm_gd_step(const cm_code *cA, const float *A, int64_t lda, const float
 {
     if (!cA || !cAT || cA->dt != CM_F32 || cAT->dt != CM_F32) return CM_EINVAL;
     if (cAT->m != cA->d || cAT->d != cA->m || cAT->n != cA->n) return CM_EINVAL;
-    cm_status st = check_survivors(cA, surv_A);
+    uint32_t effA, effAT;
+    cm_status st = resolve_survivors(cA, surv_A, &effA);
     if (st != CM_OK) return st;
-    st = check_survivors(cAT, surv_AT);
+    st = resolve_survivors(cAT, surv_AT, &effAT);
     if (st != CM_OK) return st;
     if (!layout_ok(A, lda, cA->d, 4) || !layout_ok(PA, ldpa, cA->d, 4) ||
         !layout_ok(AT, ldat, cAT->d, 4) || !layout_ok(PAT, ldpat, cAT->d, 4))
@@ -173,12 +228,12 @@ cm_status cm_gd_step(const cm_code *cA, const float *A, int64_t lda, const float
     if (launch_matvec(pA, A, lda, PA, ldpa, x, 1, ytA, dev_status, 0u, s) != cudaSuccess)
         return CM_ECUDA;
     // ... forms z = A x - y and multicasts it ...
-    if (launch_decode(pA, ytA, surv_A, 1, z, dev_status, DEC_RESIDUAL, y, 0.f, s) != cudaSuccess)
+    if (launch_decode(pA, ytA, effA, 1, z, dev_status, DEC_RESIDUAL, y, 0.f, s) != cudaSuccess)
         return CM_ECUDA;
     // ... decodes A^T z from any k2 results and steps x <- x - eta A^T z.
     if (launch_matvec(pAT, AT, ldat, PAT, ldpat, z, 1, ytAT, dev_status, 0u, s) != cudaSuccess)
         return CM_ECUDA;
-    if (launch_decode(pAT, ytAT, surv_AT, 1, x, dev_status, DEC_DESCENT, nullptr, eta, s) !=
+    if (launch_decode(pAT, ytAT, effAT, 1, x, dev_status, DEC_DESCENT, nullptr, eta, s) !=
         cudaSuccess)
         return CM_ECUDA;
     return CM_OK;
@@ -204,13 +259,14 @@ cm_status cm_decode_mat(const cm_code *c, const float *Ct, int64_t ldc, uint32_t
                         cm_stream_t stream)
 {
     if (!c) return CM_EINVAL;
-    cm_status st = check_survivors(c, survivors);
+    uint32_t eff;
+    cm_status st = resolve_survivors(c, survivors, &eff);
     if (st != CM_OK) return st;
     if (N < 1 || !Ct || !C || ldc < N || ldcc < N || ((uintptr_t)Ct & 3u) ||
         ((uintptr_t)C & 3u))
         return CM_EINVAL;
     if (C == Ct && ldcc != ldc) return CM_EINVAL;
-    return from_cuda(launch_decode_mat(code_params(c), Ct, ldc, survivors, N, C, ldcc,
+    return from_cuda(launch_decode_mat(code_params(c), Ct, ldc, eff, N, C, ldcc,
                                        dev_status, (cudaStream_t)stream));
 }
 

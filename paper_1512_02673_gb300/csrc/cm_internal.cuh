@@ -9,10 +9,13 @@
 #define CM_MAX_N 32
 #define CM_MAX_P 256   // (n-k) k <= 16 * 16 for n <= 32
 
+enum CodeKind { CODE_GENERAL = 0, CODE_REPETITION = 1 };
+
 struct cm_code {
     int32_t n, k;
     int64_t m, d, L;
     cm_dtype dt;
+    int32_t kind;        // CodeKind
     float P[CM_MAX_P];   // (n-k) x k, row-major
 };
 

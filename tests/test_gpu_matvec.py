@@ -382,3 +382,39 @@ def test_survivors_only_products(cm, orc, n, k, m, d, b):
                 assert torch.all(Yt[blk] == 12345.0), j        # never written
         want = orc.matmul(r["A_cpu"].numpy(), r["X_cpu"].numpy())
         assert rel_l2_cols(Y.cpu().numpy(), want).max() <= 1e-4
+
+
+@pytest.mark.parametrize("n,k,m,d,b", [(12, 4, 1001, 300, 2), (10, 5, 2000, 512, 8), (6, 3, 77, 33, 1)])
+def test_repetition_code_end_to_end(cm, orc, n, k, m, d, b):
+    """n/k-repetition code (Example "Repetition codes"): parity blocks are
+    exact copies, a decode from one replica per block reproduces the product
+    of the systematic blocks exactly, and a set missing a block is refused."""
+    code = cm.Code(n, k, m, d, "repetition")
+    L = code.L
+    A = padded(m, d, (d + 3) // 4 * 4, 31)
+    X_cpu = synth.gaussian((d, b), 32)
+    X = X_cpu.to(DEV)
+    par = cm.encode(code, A)
+    for p in range(n - k):                     # worker k + p copies block p mod k
+        i = p % k
+        rows = min(L, m - i * L)
+        assert torch.equal(par[p * L:p * L + rows], A[i * L:i * L + rows])
+    Yt = cm.matvec(code, A, par, X)
+    Y_sys = cm.decode(code, Yt, (1 << k) - 1)  # all systematic workers
+    rng = np.random.default_rng(7)
+    tried = 0
+    while tried < 12:
+        mask = int(rng.integers(1, 1 << n))
+        try:
+            want_sel = orc.repetition_select(n, k, mask)
+        except orc.OracleError:
+            with pytest.raises(cm.CodedError) as e:
+                cm.decode(code, Yt, mask)
+            assert e.value.status == cm.CM_ENOTDECODABLE
+            continue
+        assert code.select_decodable(mask) == want_sel
+        Y = cm.decode(code, Yt, mask)
+        assert torch.equal(Y, Y_sys), hex(mask)
+        tried += 1
+    want = orc.matmul(A.cpu().numpy(), X_cpu.numpy())
+    assert rel_l2_cols(Y_sys.cpu().numpy(), want).max() <= 1e-4

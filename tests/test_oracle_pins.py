@@ -282,3 +282,41 @@ def test_seeded_parity_is_mds(n, k):
                 blk = sub[:, cols[c0:c0 + 200000]].transpose(1, 0, 2)
                 worst = min(worst, np.abs(np.linalg.det(blk)).min())
     assert worst > 1e-9, worst
+
+
+# ---- runtime model and repetition codes (Sec. III-B, III-C, III-D) --------------
+
+@pytest.mark.parametrize("scheme,n,k", [("uncoded", 8, 8), ("repetition", 8, 4), ("mds", 8, 4)])
+def test_oracle_runtime_simulator_matches_paper_forms(orc, scheme, n, k):
+    # the simulated overall runtime follows the paper's distributions (eqs. for
+    # F_uncoded, F_rep and the integral F_MDS, by quadrature) and their means
+    from scipy import stats
+    import oracle.runtime_model as rm
+    T = orc.runtime_simulate(scheme, n, k, 1.0, 1.0, 4242, 0, 20000)
+    cdf = {"uncoded": lambda t: rm.cdf_uncoded(t, n),
+           "repetition": lambda t: rm.cdf_repetition(t, n, k),
+           "mds": lambda t: rm.cdf_mds(t, n, k)}[scheme]
+    assert stats.kstest(T[:3000], cdf).pvalue > 1e-3
+    upper = 60.0 / (k if scheme != "uncoded" else n)
+    mean = rm.mean_from_cdf(cdf, upper)
+    assert abs(T.mean() - mean) < 5 * T.std() / math.sqrt(T.size)
+
+
+def test_repetition_select_brute_force(orc):
+    # Example "Repetition codes": a survivor set is decodable iff some k of its
+    # members give a nonsingular G_S; the selection must be such a set, and
+    # must fail exactly when none exists (brute force over all k-subsets)
+    for n, k in [(6, 3), (8, 4), (6, 2)]:
+        G = np.vstack([np.eye(k), orc.repetition_parity(n, k)])
+        for mask in range(1 << n):
+            surv = [j for j in range(n) if mask >> j & 1]
+            ok = any(np.linalg.matrix_rank(G[list(S)]) == k
+                     for S in itertools.combinations(surv, k)) if len(surv) >= k else False
+            if ok:
+                sel = orc.repetition_select(n, k, mask)
+                S = [j for j in range(n) if sel >> j & 1]
+                assert len(S) == k and set(S) <= set(surv)
+                assert np.linalg.matrix_rank(G[S]) == k
+            else:
+                with pytest.raises(orc.OracleError):
+                    orc.repetition_select(n, k, mask)

@@ -269,6 +269,130 @@ cm_status cm_runtime_simulate(cm_scheme scheme, int32_t n, int32_t k, double shi
  * the Lambert W function). */
 cm_status cm_optimal_mds_k(int32_t n, double rate, double *k_star, double *gamma_star);
 
+/* ---- coded shuffling (Sec. IV) --------------------------------------------
+ * q data rows of r 4-byte words are reshuffled across n workers before every
+ * iteration: a uniformly random partition into sets S_i of q/n rows (Sec.
+ * IV-A).  Worker i has a cache of s rows (q/n <= s <= q) holding S_i plus
+ * s - q/n rows kept by the cache update rule: drawn without replacement from
+ * its previous cache outside the new S_i (Sec. IV-B).  For the transition
+ * t -> t+1 the master sends, for every worker set I with |I| >= 2, the sum of
+ * the zero-padded blocks A(S_i^{t+1} & C~_{I\{i}}), i in I, where C~_J is the
+ * set of rows cached at every worker of J and at no other (Alg. 1); each
+ * worker recovers its missing rows by subtracting the rows it caches (the
+ * decoding algorithm of Sec. IV-B).
+ *
+ * A cm_shuffle is a host object: the master's planner.  It holds the
+ * partition, the caches (as n x s slot tables: slot c of worker i holds data
+ * row slot_row[i s + c]) and the row programs of the last transition.  The
+ * data plane runs on the device on caller-owned buffers:
+ *   A       q x r data rows (leading dimension lda words)
+ *   caches  n s x r: slot c of worker i is row i s + c (leading dimension ldc)
+ *   M       coded message rows, >= coded_rows x r (leading dimension ldm)
+ *   Rx      received rows, >= uncoded_rows x r (leading dimension ldr): the
+ *           rows of S_i^{t+1} missing from cache i, for worker 0, 1, ... in
+ *           ascending data-row order (cm_shuffle_received lists them).
+ * Every device buffer starts on a 16-byte boundary and its leading dimension
+ * is a multiple of 4 words; any r >= 1.  Nothing runs in place: M, Rx and
+ * the caches are distinct buffers.
+ *
+ * Sums: CM_SHUFFLE_ADD adds and subtracts the rows as fp32 reals, the
+ * arithmetic of the paper (decoded rows then carry fp32 rounding of the sum);
+ * CM_SHUFFLE_XOR combines the 32-bit words by exclusive or, a sum in which
+ * every element is its own negative, so decoding is exact for any data.
+ *
+ * Random draws are SplitMix64 outputs (state = seed + index
+ * 0x9E3779B97F4A7C15, then the standard finaliser): iteration t's partition
+ * orders rows by (key(partition_seed, t q + r), r) and gives the positions
+ * [i q/n, (i+1) q/n) to worker i; a cache refill of worker i at iteration t
+ * keeps the s - q/n candidates with the smallest (key(cache_seed,
+ * (t n + i) q + r), r).  Iteration 0's caches refill from all rows outside
+ * S_i^0. */
+typedef struct cm_shuffle cm_shuffle;
+
+typedef enum { CM_SHUFFLE_ADD = 0, CM_SHUFFLE_XOR = 1 } cm_shuffle_op;
+
+typedef struct {
+    int64_t iteration;      /* t of the current partition and caches */
+    int64_t message_sets;   /* sets I with a non-empty message in the last transition */
+    int64_t coded_rows;     /* rows the coded scheme sends (the realised R_c) */
+    int64_t uncoded_rows;   /* rows missing from their new owner's cache (realised R_u) */
+    int64_t subtractions;   /* cached rows the workers subtract while decoding */
+} cm_shuffle_stats;
+
+/* Draws iteration 0 (partition and caches).  2 <= n <= 64, q % n == 0,
+ * q/n <= s <= q and n q < 2^31; else CM_EINVAL.  CM_ENOMEM if the host tables
+ * (about 4 n q + 16 q bytes) cannot be allocated. */
+cm_status cm_shuffle_create(int32_t n, int64_t q, int64_t s, uint64_t partition_seed,
+                            uint64_t cache_seed, cm_shuffle **out);
+void cm_shuffle_destroy(cm_shuffle *shuffle);
+
+/* Host planning of the transition t -> t+1: draws the next partition, plans
+ * Alg. 1's messages and the decoding, applies the cache update rule and
+ * assigns the received rows to the freed cache slots.  stats is nullable. */
+cm_status cm_shuffle_next(cm_shuffle *shuffle, cm_shuffle_stats *stats);
+
+/* Statistics of the last transition (zeros before the first). */
+cm_status cm_shuffle_query(const cm_shuffle *shuffle, cm_shuffle_stats *stats);
+
+/* The messages of the last transition: message row m sums data rows
+ * msg_src[msg_ptr[m] .. msg_ptr[m+1]) (coded_rows + 1 offsets; uncoded_rows
+ * rows), row x needed by worker msg_worker[x]; msg_set[m] is the bit mask of
+ * its I.  Any output may be NULL.  CM_EINVAL before the first transition. */
+cm_status cm_shuffle_plan(const cm_shuffle *shuffle, int32_t *msg_ptr, int32_t *msg_src,
+                          int32_t *msg_worker, uint64_t *msg_set);
+
+/* Layout of Rx: worker i's received rows are rows [recv_ptr[i], recv_ptr[i+1])
+ * (n + 1 offsets), holding data rows recv_row[...] in ascending order. */
+cm_status cm_shuffle_received(const cm_shuffle *shuffle, int32_t *recv_ptr, int32_t *recv_row);
+
+/* The current partition (owner[r] = i for r in S_i, q entries) and cache
+ * slot tables (n s entries).  Either output may be NULL. */
+cm_status cm_shuffle_caches(const cm_shuffle *shuffle, int32_t *owner, int32_t *slot_row);
+
+/* Communication rates of the coded shuffling rate theorem, in data rows per
+ * iteration: R_c = sum_{i=2}^{n} C(n,i) (q/n) ((i-1)/n) p^{i-2} (1-p)^{n-i+1},
+ * p = (s - q/n)/(q - q/n) (the sum its proof evaluates; equal to the closed
+ * form q/(np)^2 ((1-p)^{n+1} + (n-1) p (1-p) - (1-p)^2)), and the uncoded
+ * rate R_u = q (1 - s/q) (eq. for R_u).  Host only. */
+cm_status cm_shuffle_rates(int32_t n, double q, double s, double *coded, double *uncoded);
+
+/* Bytes of device workspace for the row programs of any transition of this
+ * instance (about 4 q (n + 5) + 4 n s). */
+size_t cm_shuffle_workspace_bytes(const cm_shuffle *shuffle);
+
+/* Copies the current row programs (and slot tables) into `workspace` (16-byte
+ * aligned, >= cm_shuffle_workspace_bytes) on `stream`.  The host tables may
+ * change once this returns.  Every data-plane call below checks that the
+ * workspace it is given holds the programs of the current transition and
+ * returns CM_EINVAL otherwise. */
+cm_status cm_shuffle_upload(cm_shuffle *shuffle, void *workspace, size_t bytes,
+                            cm_stream_t stream);
+
+/* Loads every cache from A by its slot table: caches[i s + c] = A[slot_row[i s + c]]. */
+cm_status cm_shuffle_fill(const cm_shuffle *shuffle, const void *workspace, const void *A,
+                          int64_t lda, int64_t r, void *caches, int64_t ldc,
+                          cm_stream_t stream);
+
+/* Alg. 1 (master): M[m] = sum of the data rows of message row m (zero-padded
+ * blocks contribute nothing).  Needs a planned transition. */
+cm_status cm_shuffle_encode(const cm_shuffle *shuffle, const void *workspace, cm_shuffle_op op,
+                            const void *A, int64_t lda, int64_t r, void *M, int64_t ldm,
+                            cm_stream_t stream);
+
+/* Decoding by subtraction (workers): every received row = its message row
+ * minus the other rows of that message row, read from the receiving
+ * worker's cache before the transition (the caches must still hold C^t). */
+cm_status cm_shuffle_decode(const cm_shuffle *shuffle, const void *workspace, cm_shuffle_op op,
+                            const void *M, int64_t ldm, const void *caches, int64_t ldc,
+                            int64_t r, void *Rx, int64_t ldr, cm_stream_t stream);
+
+/* Cache update (workers): writes every received row into the cache slot it
+ * takes over, turning the caches C^t into C^{t+1}.  Run after the decode of
+ * the same transition. */
+cm_status cm_shuffle_commit(const cm_shuffle *shuffle, const void *workspace, const void *Rx,
+                            int64_t ldr, int64_t r, void *caches, int64_t ldc,
+                            cm_stream_t stream);
+
 /* Static description of a status code. */
 const char *cm_status_string(cm_status s);
 

@@ -76,6 +76,20 @@ def lib() -> ctypes.CDLL:
             "cm_runtime_cdf": (st, [st, i32, i32, f64, f64, vp, i64, vp]),
             "cm_runtime_simulate": (st, [st, i32, i32, f64, f64, u64, u64, i64, vp]),
             "cm_optimal_mds_k": (st, [i32, f64, ctypes.POINTER(f64), ctypes.POINTER(f64)]),
+            "cm_shuffle_create": (st, [i32, i64, i64, u64, u64, ctypes.POINTER(vp)]),
+            "cm_shuffle_destroy": (None, [vp]),
+            "cm_shuffle_next": (st, [vp, vp]),
+            "cm_shuffle_query": (st, [vp, vp]),
+            "cm_shuffle_plan": (st, [vp, vp, vp, vp, vp]),
+            "cm_shuffle_received": (st, [vp, vp, vp]),
+            "cm_shuffle_caches": (st, [vp, vp, vp]),
+            "cm_shuffle_rates": (st, [i32, f64, f64, ctypes.POINTER(f64), ctypes.POINTER(f64)]),
+            "cm_shuffle_workspace_bytes": (sz, [vp]),
+            "cm_shuffle_upload": (st, [vp, vp, sz, vp]),
+            "cm_shuffle_fill": (st, [vp, vp, vp, i64, i64, vp, i64, vp]),
+            "cm_shuffle_encode": (st, [vp, vp, st, vp, i64, i64, vp, i64, vp]),
+            "cm_shuffle_decode": (st, [vp, vp, st, vp, i64, vp, i64, i64, vp, i64, vp]),
+            "cm_shuffle_commit": (st, [vp, vp, vp, i64, i64, vp, i64, vp]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -439,3 +453,144 @@ def optimal_mds_k(n: int, rate: float = 1.0):
     _check(lib().cm_optimal_mds_k(n, rate, ctypes.byref(ks), ctypes.byref(g)),
            "cm_optimal_mds_k")
     return float(ks.value), float(g.value)
+
+
+# ---- coded shuffling (Sec. IV) --------------------------------------------------
+
+SHUFFLE_OPS = {"add": 0, "xor": 1}
+
+
+class _ShuffleStats(ctypes.Structure):
+    _fields_ = [("iteration", ctypes.c_int64), ("message_sets", ctypes.c_int64),
+                ("coded_rows", ctypes.c_int64), ("uncoded_rows", ctypes.c_int64),
+                ("subtractions", ctypes.c_int64)]
+
+
+def _rows(t: torch.Tensor, name: str) -> int:
+    """Pointer of a CUDA matrix of 4-byte words (fp32 or int32), row-major."""
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError("%s must be a CUDA tensor" % name)
+    if t.dtype not in (torch.float32, torch.int32):
+        raise TypeError("%s must hold 4-byte words (float32 or int32)" % name)
+    _ld(t, name)
+    return t.data_ptr()
+
+
+def _np(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.c_void_p)
+
+
+def shuffle_rates(n: int, q: float, s: float):
+    """(R_c, R_u) of the coded shuffling rate theorem and eq. for R_u."""
+    c, u = ctypes.c_double(0.0), ctypes.c_double(0.0)
+    _check(lib().cm_shuffle_rates(n, q, s, ctypes.byref(c), ctypes.byref(u)),
+           "cm_shuffle_rates")
+    return float(c.value), float(u.value)
+
+
+class Shuffle:
+    """Coded shuffling of q rows over n workers with caches of s rows.
+
+    The planner is host state in libcm; the device workspace for its row
+    programs is a torch byte tensor owned by this object."""
+
+    def __init__(self, n: int, q: int, s: int, partition_seed: int, cache_seed: int):
+        out = ctypes.c_void_p()
+        _check(lib().cm_shuffle_create(n, q, s, partition_seed, cache_seed, ctypes.byref(out)),
+               "cm_shuffle_create")
+        self._h = out
+        self.n, self.q, self.s = n, q, s
+        self._ws = None
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h and _lib is not None:
+            _lib.cm_shuffle_destroy(h)
+            self._h = None
+
+    def next(self) -> dict:
+        """Plans the next transition; returns its statistics."""
+        st = _ShuffleStats()
+        _check(lib().cm_shuffle_next(self._h, ctypes.byref(st)), "cm_shuffle_next")
+        return {f: int(getattr(st, f)) for f, _ in _ShuffleStats._fields_}
+
+    def stats(self) -> dict:
+        st = _ShuffleStats()
+        _check(lib().cm_shuffle_query(self._h, ctypes.byref(st)), "cm_shuffle_query")
+        return {f: int(getattr(st, f)) for f, _ in _ShuffleStats._fields_}
+
+    def plan(self):
+        """(msg_ptr, msg_src, msg_worker, msg_set) of the last transition."""
+        st = self.stats()
+        ptr = np.empty(st["coded_rows"] + 1, np.int32)
+        src = np.empty(st["uncoded_rows"], np.int32)
+        wk = np.empty(st["uncoded_rows"], np.int32)
+        sets = np.empty(st["coded_rows"], np.uint64)
+        _check(lib().cm_shuffle_plan(self._h, _np(ptr), _np(src), _np(wk), _np(sets)),
+               "cm_shuffle_plan")
+        return ptr, src, wk, sets
+
+    def received(self):
+        """(recv_ptr, recv_row): the layout of the received rows Rx."""
+        st = self.stats()
+        ptr = np.empty(self.n + 1, np.int32)
+        rows = np.empty(st["uncoded_rows"], np.int32)
+        _check(lib().cm_shuffle_received(self._h, _np(ptr), _np(rows)), "cm_shuffle_received")
+        return ptr, rows
+
+    def caches(self):
+        """(owner, slot_row): the current partition and cache slot tables."""
+        owner = np.empty(self.q, np.int32)
+        slots = np.empty(self.n * self.s, np.int32)
+        _check(lib().cm_shuffle_caches(self._h, _np(owner), _np(slots)), "cm_shuffle_caches")
+        return owner, slots.reshape(self.n, self.s)
+
+    def workspace_bytes(self) -> int:
+        return int(lib().cm_shuffle_workspace_bytes(self._h))
+
+    def upload(self, device=None):
+        """Copies the current row programs to the device workspace."""
+        nb = self.workspace_bytes()
+        if self._ws is None:
+            self._ws = torch.empty(nb, dtype=torch.uint8,
+                                   device=device or torch.device("cuda"))
+        _check(lib().cm_shuffle_upload(self._h, ctypes.c_void_p(self._ws.data_ptr()), nb,
+                                       _stream()), "cm_shuffle_upload")
+
+    def _wsp(self):
+        return ctypes.c_void_p(self._ws.data_ptr() if self._ws is not None else 0)
+
+    def fill(self, A: torch.Tensor, caches: torch.Tensor | None = None) -> torch.Tensor:
+        r = A.shape[1]
+        if caches is None:
+            caches = torch.empty((self.n * self.s, r), dtype=A.dtype, device=A.device)
+        _check(lib().cm_shuffle_fill(self._h, self._wsp(), _rows(A, "A"), _ld(A, "A"), r,
+                                     _rows(caches, "caches"), _ld(caches, "caches"), _stream()),
+               "cm_shuffle_fill")
+        return caches
+
+    def encode(self, op: str, A: torch.Tensor, M: torch.Tensor | None = None) -> torch.Tensor:
+        r = A.shape[1]
+        if M is None:
+            M = torch.empty((max(1, self.stats()["coded_rows"]), r), dtype=A.dtype,
+                            device=A.device)
+        _check(lib().cm_shuffle_encode(self._h, self._wsp(), SHUFFLE_OPS[op], _rows(A, "A"),
+                                       _ld(A, "A"), r, _rows(M, "M"), _ld(M, "M"), _stream()),
+               "cm_shuffle_encode")
+        return M
+
+    def decode(self, op: str, M: torch.Tensor, caches: torch.Tensor, r: int,
+               Rx: torch.Tensor | None = None) -> torch.Tensor:
+        if Rx is None:
+            Rx = torch.empty((max(1, self.stats()["uncoded_rows"]), r), dtype=M.dtype,
+                             device=M.device)
+        _check(lib().cm_shuffle_decode(self._h, self._wsp(), SHUFFLE_OPS[op], _rows(M, "M"),
+                                       _ld(M, "M"), _rows(caches, "caches"),
+                                       _ld(caches, "caches"), r, _rows(Rx, "Rx"), _ld(Rx, "Rx"),
+                                       _stream()), "cm_shuffle_decode")
+        return Rx
+
+    def commit(self, Rx: torch.Tensor, caches: torch.Tensor, r: int) -> None:
+        _check(lib().cm_shuffle_commit(self._h, self._wsp(), _rows(Rx, "Rx"), _ld(Rx, "Rx"), r,
+                                       _rows(caches, "caches"), _ld(caches, "caches"),
+                                       _stream()), "cm_shuffle_commit")

@@ -25,6 +25,8 @@ import torch
 DATA_SEED = 1512
 CODE_SEED = 2673
 ERASURE_SEED = 3
+SHUFFLE_PARTITION_SEED = 4   # coded shuffling: partitions of [q]
+SHUFFLE_CACHE_SEED = 5       # coded shuffling: cache refills
 STRAGGLE_SHIFT = 1.0   # shifted-exponential model, Sec. III-D: shift 1
 STRAGGLE_RATE = 1.0    # straggling parameter mu
 
@@ -72,6 +74,32 @@ BANDWIDTH = Workload("coded mat-multi-vec (32,24) 65536x65536 b=8", m=65536,
                      d=65536, b=8, n=32, k=24, data_device="cuda")
 GEMM = Workload("coded GEMM bf16 (16,12) 32768x8192x4096", m=32768, d=8192,
                 b=0, n=16, k=12, dtype="bf16", gemm_n=4096)
+
+
+@dataclasses.dataclass(frozen=True)
+class ShuffleWorkload:
+    """Coded shuffling (Sec. IV): q data rows of r fp32 words, n workers with
+    caches of s rows, `transitions` reshuffles."""
+    name: str
+    n: int
+    q: int
+    s: int
+    r: int
+    transitions: int = 1
+
+
+# the setting of the rate figure of Sec. IV-D (n = 50, q = 1000, s/q = 0.1) is
+# a rate example; the data-plane workload keeps rows of 1 KiB and fewer
+# workers so that every block of Alg. 1 holds thousands of rows
+SHUFFLE = ShuffleWorkload("coded shuffling n=8 q=2097152 s=q/4 r=256", n=8, q=1 << 21,
+                          s=1 << 19, r=256, transitions=4)
+SHUFFLE_SMALL = ShuffleWorkload("coded shuffling n=4 q=4000 s=1700 r=67", n=4, q=4000,
+                                s=1700, r=67, transitions=3)
+
+
+def shuffle_rows(w: ShuffleWorkload, device="cpu", seed: int = DATA_SEED + 7) -> torch.Tensor:
+    """The q x r data rows (i.i.d. N(0,1) fp32)."""
+    return gaussian((w.q, w.r), seed, device)
 
 
 def parity_coefficients(n: int, k: int, seed: int = CODE_SEED) -> np.ndarray:

@@ -250,6 +250,9 @@ PROFILE = synth.Workload("coded mat-multi-vec (32,24) 14592x16384 b=8 (profiling
 PROFILE_GEMM = synth.Workload("coded GEMM bf16 (16,12) 16384x8192x4096 (profiling case)",
                               m=16384, d=8192, b=0, n=16, k=12, dtype="bf16", gemm_n=4096,
                               data_device="cuda")
+PROFILE_SHUFFLE = synth.ShuffleWorkload("coded shuffling n=8 q=524288 s=q/4 r=256 "
+                                        "(profiling case)", n=8, q=1 << 19, s=1 << 17,
+                                        r=256, transitions=3)
 WORKLOADS = {"bandwidth": synth.BANDWIDTH, "profile": PROFILE}
 
 
@@ -326,10 +329,12 @@ def run_ours(args, world, rank, local):
         del A, parity
         torch.cuda.empty_cache()
         gm = bench_gemm(cm, dev, PROFILE_GEMM, args.steps, args.warmup)
+        torch.cuda.empty_cache()
+        shf = bench_shuffle(cm, dev, PROFILE_SHUFFLE)
         if rank == 0:
             print(json.dumps({"workload": w.name, "ms_per_step": ms / args.steps,
                               "kernels_us": {k: v * 1e3 for k, v in avg.items()},
-                              "gemm": gm}), flush=True)
+                              "gemm": gm, "coded_shuffling": shf}), flush=True)
         return
 
     # end to end through the public API with host buffers: pinned X in, Y out
@@ -366,6 +371,8 @@ def run_ours(args, world, rank, local):
     mv100 = bench_repeats(cm, dev, synth.MATVEC)
     tiny = bench_repeats(cm, dev, synth.TINY, repeats=20)
     torch.cuda.empty_cache()
+    shuffle = bench_shuffle(cm, dev, synth.SHUFFLE)
+    torch.cuda.empty_cache()
 
     peaks = measured_peaks()
     achieved = nbytes["matvec"] / (avg["matvec"] * 1e-3) / 1e9
@@ -400,6 +407,7 @@ def run_ours(args, world, rank, local):
         "clocks": clk.summary(),
         "secondary": {"survivors_only": so, "gemm": gemm, "gd": gd,
                       "matvec_100_repeats": mv100, "tiny": tiny,
+                      "coded_shuffling": shuffle,
                       "runtime_model": runtime_model_report(cm)},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -431,6 +439,80 @@ def bench_survivors_only(cm, code, A, parity, X, Yt, Y, status, w, args) -> dict
     read = w.k * L * w.d * 4 + w.d * w.b * 4 + w.k * L * w.b * 8
     return {"matvec_ms": mv, "decode_ms": dec, "matvec_gbs": read / (mv * 1e-3) / 1e9,
             "bytes_read": read, "status": int(status.item())}
+
+
+def shuffle_bytes(st: dict, r: int) -> dict:
+    """Algorithmic HBM bytes of one transition's kernels: data rows of r fp32
+    words plus the int32 row programs.  encode reads every summed row once and
+    writes every message row; decode reads every message row once (one
+    multicast for all of I), every subtracted cached row, and writes every
+    received row; commit copies every received row into its cache slot."""
+    R, C, X = st["uncoded_rows"], st["coded_rows"], st["subtractions"]
+    rb = 4 * r
+    return {"encode": (R + C) * rb + 4 * (C + 1 + R),
+            "decode": (C + X + R) * rb + 4 * (3 * R + 1 + X),
+            "commit": 2 * R * rb + 4 * R}
+
+
+def bench_shuffle(cm, dev, w: synth.ShuffleWorkload) -> dict:
+    """Coded shuffling (Sec. IV) on the GPU: per transition the host plans
+    Alg. 1 and the cache update, then encode, decode by subtraction and the
+    cache commit run on the device (xor sums: exact, the same bytes as real
+    sums).  Checks after the last transition that every cache slot holds its
+    data row exactly."""
+    peaks = measured_peaks()
+    A = synth.shuffle_rows(w, dev)
+    sh = cm.Shuffle(w.n, w.q, w.s, synth.SHUFFLE_PARTITION_SEED, synth.SHUFFLE_CACHE_SEED)
+    sh.upload()
+    caches = sh.fill(A)
+    M = torch.empty((w.q, w.r), device=dev)
+    Rx = torch.empty((w.q, w.r), device=dev)
+    rows = {"coded": [], "uncoded": []}
+    t_plan, t_up, ms = [], [], {"encode": [], "decode": [], "commit": []}
+    nb = {"encode": 0, "decode": 0, "commit": 0}
+    for t in range(w.transitions):
+        t0 = time.perf_counter()
+        st = sh.next()
+        t1 = time.perf_counter()
+        sh.upload()
+        torch.cuda.synchronize()
+        t2 = time.perf_counter()
+        t_plan.append(t1 - t0)
+        t_up.append(t2 - t1)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        ev[0].record()
+        sh.encode("xor", A, M)
+        ev[1].record()
+        sh.decode("xor", M, caches, w.r, Rx)
+        ev[2].record()
+        sh.commit(Rx, caches, w.r)
+        ev[3].record()
+        torch.cuda.synchronize()
+        if t > 0:      # the first transition warms the kernels up
+            for j, k in enumerate(("encode", "decode", "commit")):
+                ms[k].append(ev[j].elapsed_time(ev[j + 1]))
+            for k, v in shuffle_bytes(st, w.r).items():
+                nb[k] += v
+        rows["coded"].append(st["coded_rows"])
+        rows["uncoded"].append(st["uncoded_rows"])
+    _, slots = sh.caches()
+    exact = bool(torch.equal(caches, A[torch.from_numpy(slots.reshape(-1)).long().to(dev)]))
+    rc, ru = cm.shuffle_rates(w.n, w.q, w.s)
+    kern = {}
+    for k in ms:
+        tot = sum(ms[k])
+        gbs = nb[k] / (tot * 1e-3) / 1e9
+        kern[k] = {"ms": tot / len(ms[k]), "gbs": gbs, "frac": gbs / peaks["hbm_gbs"]}
+    dev_ms = sum(kern[k]["ms"] for k in kern)
+    return {"workload": w.name, "transitions_timed": w.transitions - 1,
+            "kernels": kern, "device_ms_per_transition": dev_ms,
+            "device_gbs": sum(nb.values()) / (sum(sum(v) for v in ms.values()) * 1e-3) / 1e9,
+            "host_plan_ms": 1e3 * float(np.mean(t_plan[1:])),
+            "upload_ms": 1e3 * float(np.mean(t_up[1:])),
+            "rows": {"coded_mean": float(np.mean(rows["coded"][1:])),
+                     "uncoded_mean": float(np.mean(rows["uncoded"][1:])),
+                     "theorem_R_c": rc, "R_u": ru},
+            "roofline_peak_gbs": peaks["hbm_gbs"], "caches_exact": exact}
 
 
 def runtime_model_report(cm) -> dict:

@@ -9,8 +9,9 @@
 // zero-padded block contributes no term, so a padded row of Alg. 1 costs
 // nothing.  Rows are r 4-byte words with 16-byte aligned starts.
 //
-// Mapping: one warp per output row, persistent grid (a multiple of the SM
-// count), rows taken in a warp-strided loop.  Each lane owns U float4 columns
+// Mapping: persistent grid (the resident blocks of every SM); row o goes to
+// warp o mod W, which batches the program words of its next 32 rows.  Each
+// lane owns U float4 columns
 // of a column block of 32 U float4 and issues the U loads of a term together,
 // so every warp keeps U x 512 bytes per term in flight.  Term row indices are
 // read once per row by the lanes and broadcast by shuffles.  Every data byte
@@ -83,51 +84,84 @@ __global__ void __launch_bounds__(kThreads) row_program_kernel(
     RowProgram p, const float *__restrict__ in0, int64_t ld0, const float *__restrict__ in1,
     int64_t ld1, float *__restrict__ out, int64_t ldo, int64_t r)
 {
+    constexpr unsigned kAll = 0xffffffffu;
     const int lane = threadIdx.x & 31;
+    const int64_t warp = (((int64_t)blockIdx.x * kThreads) + threadIdx.x) >> 5;
     const int64_t nwarps = ((int64_t)gridDim.x * kThreads) >> 5;
     const int64_t r4 = r >> 2;
-    for (int64_t o = (((int64_t)blockIdx.x * kThreads) + threadIdx.x) >> 5; o < p.rows;
-         o += nwarps) {
-        int beg = 0, nt = 0;
+    // Rows are dealt to warps round-robin (row o to warp o mod W), so that
+    // neighbouring rows, which touch neighbouring messages and data rows,
+    // are in flight together.  A warp reads the program words of its next 32
+    // rows in one go (lane l: its l-th next row) and broadcasts them by
+    // shuffles, and fetches the term indices of the next row while the
+    // current row's data moves: a row waits on one memory latency, not three.
+    for (int64_t base = warp; base < p.rows; base += 32 * nwarps) {
+        const int64_t mine = base + lane * nwarps;
+        const bool valid = mine < p.rows;
+        const int cnt = (int)min((int64_t)32, (p.rows - base + nwarps - 1) / nwarps);
+        int beg_l = 0, end_l = 0, first_l = 0, dst_l = 0;
+        if (valid) {
+            if (p.ptr) {
+                beg_l = p.ptr[mine];
+                end_l = p.ptr[mine + 1];
+            }
+            if (FIRST) first_l = p.first ? p.first[mine] : (int)mine;
+            dst_l = p.dst ? p.dst[mine] : (int)mine;
+        }
+        // terms of row j: lane l holds terms l and 32 + l (nt <= 64)
+        int next0 = 0, next1 = 0;
         if (p.ptr) {
-            beg = p.ptr[o];
-            nt = p.ptr[o + 1] - beg;    // <= n - 1 <= 63 (decode) or <= n (encode)
+            const int b = __shfl_sync(kAll, beg_l, 0);
+            const int nj = __shfl_sync(kAll, end_l, 0) - b;
+            next0 = lane < nj ? p.term[b + lane] : 0;
+            next1 = 32 + lane < nj ? p.term[b + 32 + lane] : 0;
         }
-        // term rows: lane l holds terms l and 32 + l, broadcast by shuffles
-        const int t0 = lane < nt ? p.term[beg + lane] : 0;
-        const int t1 = 32 + lane < nt ? p.term[beg + 32 + lane] : 0;
-        const float *src0 = nullptr;
-        if constexpr (FIRST) src0 = in0 + (int64_t)(p.first ? p.first[o] : o) * ld0;
-        float *dst = out + (int64_t)(p.dst ? p.dst[o] : o) * ldo;
-        const int e_begin = FIRST ? 0 : 1;
-        for (int64_t c0 = 0; c0 < r4; c0 += 32 * kU) {
-            float4 acc[kU];
-            if constexpr (FIRST) {
-                load_block(acc, src0, c0, r4, lane, true);
-            } else {   // a sum without in0 starts from its first term
-                const int row = __shfl_sync(0xffffffffu, t0, 0);
-                load_block(acc, in1 + (int64_t)row * ld1, c0, r4, lane, false);
+        for (int j = 0; j < cnt; ++j) {
+            const int t0 = next0, t1 = next1;
+            const int beg = __shfl_sync(kAll, beg_l, j);
+            const int nt = __shfl_sync(kAll, end_l, j) - beg;
+            // j + 1 < cnt <= 32 keeps the shuffle source in range; lanes of an
+            // out-of-range j + 1 read nothing (their nj comes out <= 0)
+            const int jn = j + 1 < cnt ? j + 1 : j;
+            const int bn = __shfl_sync(kAll, beg_l, jn);
+            const int nn = j + 1 < cnt ? __shfl_sync(kAll, end_l, jn) - bn : 0;
+            if (p.ptr) {
+                next0 = lane < nn ? p.term[bn + lane] : 0;
+                next1 = 32 + lane < nn ? p.term[bn + 32 + lane] : 0;
             }
+            const float *src0 = nullptr;
+            if constexpr (FIRST) src0 = in0 + (int64_t)__shfl_sync(kAll, first_l, j) * ld0;
+            float *dst = out + (int64_t)__shfl_sync(kAll, dst_l, j) * ldo;
+            const int e_begin = FIRST ? 0 : 1;
+            for (int64_t c0 = 0; c0 < r4; c0 += 32 * kU) {
+                float4 acc[kU];
+                if constexpr (FIRST) {
+                    load_block(acc, src0, c0, r4, lane, true);
+                } else {   // a sum without in0 starts from its first term
+                    const int row = __shfl_sync(kAll, t0, 0);
+                    load_block(acc, in1 + (int64_t)row * ld1, c0, r4, lane, false);
+                }
 #pragma unroll 4
-            for (int e = e_begin; e < nt; ++e) {
-                const int row = __shfl_sync(0xffffffffu, e < 32 ? t0 : t1, e & 31);
-                float4 v[kU];
-                load_block(v, in1 + (int64_t)row * ld1, c0, r4, lane, false);
+                for (int e = e_begin; e < nt; ++e) {
+                    const int row = __shfl_sync(kAll, e < 32 ? t0 : t1, e & 31);
+                    float4 v[kU];
+                    load_block(v, in1 + (int64_t)row * ld1, c0, r4, lane, false);
 #pragma unroll
-                for (int u = 0; u < kU; ++u) combine4<OP>(acc[u], v[u]);
-            }
+                    for (int u = 0; u < kU; ++u) combine4<OP>(acc[u], v[u]);
+                }
 #pragma unroll
-            for (int u = 0; u < kU; ++u) {
-                const int64_t c = c0 + u * 32 + lane;
-                if (c < r4) __stcs(reinterpret_cast<float4 *>(dst + 4 * c), acc[u]);
+                for (int u = 0; u < kU; ++u) {
+                    const int64_t c = c0 + u * 32 + lane;
+                    if (c < r4) __stcs(reinterpret_cast<float4 *>(dst + 4 * c), acc[u]);
+                }
             }
-        }
-        // ragged tail of r % 4 words
-        for (int64_t c = 4 * r4 + lane; c < r; c += 32) {
-            float a = FIRST ? src0[c] : in1[(int64_t)p.term[beg] * ld1 + c];
-            for (int e = e_begin; e < nt; ++e)
-                a = combine<OP>(a, in1[(int64_t)p.term[beg + e] * ld1 + c]);
-            dst[c] = a;
+            // ragged tail of r % 4 words
+            for (int64_t c = 4 * r4 + lane; c < r; c += 32) {
+                float a = FIRST ? src0[c] : in1[(int64_t)p.term[beg] * ld1 + c];
+                for (int e = e_begin; e < nt; ++e)
+                    a = combine<OP>(a, in1[(int64_t)p.term[beg + e] * ld1 + c]);
+                dst[c] = a;
+            }
         }
     }
 }

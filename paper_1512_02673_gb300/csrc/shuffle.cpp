@@ -35,10 +35,13 @@
 // outside S_i^0, so C_i^0 \ S_i^0 is uniform without replacement (the
 // marginal law the rule maintains).
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
 #include <new>
+#include <thread>
+#include <unordered_map>
 #include <vector>
 
 #include "shuffle_internal.h"
@@ -56,7 +59,64 @@ inline uint64_t mix64(uint64_t seed, uint64_t index)
     return z;
 }
 
-using Keyed = std::pair<uint64_t, int32_t>;   // (key, row): ties broken by row
+// Runs body(j) for j = 0 .. count-1 on up to hardware_concurrency threads.
+// Returns false if a body ran out of memory.
+template <class Body>
+bool parallel_for(int count, Body body)
+{
+    const int hw = std::max(1u, std::thread::hardware_concurrency());
+    const int T = std::min(count, hw);
+    std::atomic<bool> ok{true};
+    auto run = [&](int tid) {
+        try {
+            for (int j = tid; j < count; j += T) body(j);
+        } catch (const std::bad_alloc &) {
+            ok = false;
+        }
+    };
+    if (T <= 1) {
+        run(0);
+        return ok;
+    }
+    std::vector<std::thread> th;
+    th.reserve(T - 1);
+    for (int tid = 1; tid < T; ++tid) th.emplace_back(run, tid);
+    run(0);
+    for (auto &x : th) x.join();
+    return ok;
+}
+
+struct Keyed {
+    uint64_t key;
+    int32_t row;
+};
+
+// Sorts by (key, row): one counting pass on the top 11 bits of the key, then
+// every bucket (about 2^-11 of the rows, cache resident) sorted on its own,
+// the buckets spread over threads.
+void sort_keyed(std::vector<Keyed> &a)
+{
+    constexpr int kBits = 11;
+    const size_t B = (size_t)1 << kBits;
+    std::vector<int64_t> start(B + 1, 0);
+    for (const Keyed &k : a) ++start[(k.key >> (64 - kBits)) + 1];
+    for (size_t b = 0; b < B; ++b) start[b + 1] += start[b];
+    std::vector<Keyed> out(a.size());
+    {
+        std::vector<int64_t> at(start.begin(), start.end() - 1);
+        for (const Keyed &k : a) out[at[k.key >> (64 - kBits)]++] = k;
+    }
+    auto less = [](const Keyed &x, const Keyed &y) {
+        return x.key != y.key ? x.key < y.key : x.row < y.row;
+    };
+    const int T = (int)std::max(1u, std::thread::hardware_concurrency());
+    if (!parallel_for(T, [&](int tid) {
+            for (size_t b = (size_t)tid; b < B; b += (size_t)T)
+                std::sort(out.begin() + start[b], out.begin() + start[b + 1], less);
+        }))
+        throw std::bad_alloc();
+    a.swap(out);
+}
 
 void draw_partition(const cm_shuffle &S, int64_t t, std::vector<int32_t> &owner)
 {
@@ -64,161 +124,244 @@ void draw_partition(const cm_shuffle &S, int64_t t, std::vector<int32_t> &owner)
     for (int64_t r = 0; r < S.q; ++r)
         keys[r] = {mix64(S.partition_seed, (uint64_t)t * (uint64_t)S.q + (uint64_t)r),
                    (int32_t)r};
-    std::sort(keys.begin(), keys.end());
+    sort_keyed(keys);
     owner.assign(S.q, 0);
-    for (int64_t pos = 0; pos < S.q; ++pos) owner[keys[pos].second] = (int32_t)(pos / S.per);
+    for (int64_t pos = 0; pos < S.q; ++pos) owner[keys[pos].row] = (int32_t)(pos / S.per);
 }
 
-// Sets bit i of next[r] for every r in S_i (owner[r] == i) and for the
-// s - q/n rows with candidate[r] != 0 whose keys are smallest.
-void refill(const cm_shuffle &S, int64_t t, int32_t i, const std::vector<int32_t> &owner,
-            const std::vector<char> &candidate, std::vector<uint64_t> &next)
+// The s - q/n rows kept by cache i at iteration t: among the rows r with
+// is_candidate(r), those with the smallest (key, r).
+template <class Pred>
+std::vector<int32_t> draw_kept(const cm_shuffle &S, int64_t t, int32_t i, Pred is_candidate)
 {
-    const uint64_t bit = 1ull << i;
     std::vector<Keyed> cand;
-    for (int64_t r = 0; r < S.q; ++r) {
-        if (owner[r] == i) {
-            next[r] |= bit;
-        } else if (candidate[r]) {
-            const uint64_t idx = ((uint64_t)t * (uint64_t)S.n + (uint64_t)i) * (uint64_t)S.q + (uint64_t)r;
-            cand.push_back({mix64(S.cache_seed, idx), (int32_t)r});
-        }
-    }
-    const size_t keep = (size_t)(S.s - S.per);
-    if (cand.size() > keep) std::nth_element(cand.begin(), cand.begin() + keep, cand.end());
-    for (size_t c = 0; c < std::min(keep, cand.size()); ++c) next[cand[c].second] |= bit;
+    cand.reserve((size_t)S.s);
+    const uint64_t base = ((uint64_t)t * (uint64_t)S.n + (uint64_t)i) * (uint64_t)S.q;
+    for (int64_t r = 0; r < S.q; ++r)
+        if (is_candidate(r)) cand.push_back({mix64(S.cache_seed, base + (uint64_t)r), (int32_t)r});
+    const size_t keep = std::min((size_t)(S.s - S.per), cand.size());
+    auto less = [](const Keyed &a, const Keyed &b) {
+        return a.key != b.key ? a.key < b.key : a.row < b.row;
+    };
+    if (cand.size() > keep) std::nth_element(cand.begin(), cand.begin() + keep, cand.end(), less);
+    std::vector<int32_t> rows(keep);
+    for (size_t c = 0; c < keep; ++c) rows[c] = cand[c].row;
+    return rows;
 }
 
-struct Needed {
-    uint64_t set;     // I = workers caching r, plus i
-    int32_t worker;   // i: new owner of r
-    int32_t row;      // r
-    int32_t msg;      // message row carrying r
-    int32_t entry;    // index of r among the summed rows (message order)
-};
+// Cache masks of iteration t: S_i plus the kept rows of every worker.
+std::vector<uint64_t> cache_masks(const cm_shuffle &S, const std::vector<int32_t> &owner,
+                                  const std::vector<std::vector<int32_t>> &kept)
+{
+    std::vector<uint64_t> mask(S.q, 0);
+    for (int64_t r = 0; r < S.q; ++r) mask[r] = 1ull << owner[r];
+    for (int32_t i = 0; i < S.n; ++i)
+        for (int32_t r : kept[i]) mask[r] |= 1ull << i;
+    return mask;
+}
+
+// Stable counting sort of `idx` by key(idx[u]) in [0, buckets).
+template <class Key>
+void counting_sort(std::vector<int32_t> &idx, size_t buckets, Key key)
+{
+    std::vector<int64_t> start(buckets + 1, 0);
+    for (int32_t u : idx) ++start[key(u) + 1];
+    for (size_t b = 0; b < buckets; ++b) start[b + 1] += start[b];
+    std::vector<int32_t> out(idx.size());
+    for (int32_t u : idx) out[start[key(u)]++] = u;
+    idx.swap(out);
+}
 
 cm_status plan_transition(cm_shuffle &S)
 {
     const int32_t n = S.n;
     const int64_t q = S.q, s = S.s;
     const int64_t t1 = S.t + 1;
+    S.planned = false;   // no program of this transition is usable until it is complete
     std::vector<int32_t> owner1;
     draw_partition(S, t1, owner1);
 
-    // rows of S_i^{t+1} missing from cache i, grouped by (I, i, r)
-    std::vector<Needed> need;
+    // rows of S_i^{t+1} missing from cache i, scanned in ascending row order
+    std::vector<int32_t> row, worker;
+    std::vector<uint64_t> set;
     for (int64_t r = 0; r < q; ++r) {
         const int32_t i = owner1[r];
         const uint64_t have = S.cached[r];
         if (have & (1ull << i)) continue;
-        need.push_back({have | (1ull << i), i, (int32_t)r, -1, -1});
+        row.push_back((int32_t)r);
+        worker.push_back(i);
+        set.push_back(have | (1ull << i));   // I = workers caching r, plus i
     }
-    std::sort(need.begin(), need.end(), [](const Needed &a, const Needed &b) {
-        if (a.set != b.set) return a.set < b.set;
-        if (a.worker != b.worker) return a.worker < b.worker;
-        return a.row < b.row;
-    });
+    const int64_t R = (int64_t)row.size();
+
+    // received-row order: (worker, row), a stable sort by worker
+    std::vector<int32_t> byw(R);
+    for (int64_t u = 0; u < R; ++u) byw[u] = (int32_t)u;
+    counting_sort(byw, (size_t)n, [&](int32_t u) { return (size_t)worker[u]; });
+    // message order: (I, worker, row), a stable sort of that by the rank of I
+    // among the distinct sets (ids by first appearance, then ranked)
+    std::vector<int32_t> rank(R);
+    std::vector<uint64_t> masks;
+    if (n <= 20) {
+        std::vector<int32_t> id((size_t)1 << n, -1);
+        for (int64_t u = 0; u < R; ++u) {
+            int32_t &v = id[set[u]];
+            if (v < 0) {
+                v = (int32_t)masks.size();
+                masks.push_back(set[u]);
+            }
+            rank[u] = v;
+        }
+    } else {
+        std::unordered_map<uint64_t, int32_t> id;
+        for (int64_t u = 0; u < R; ++u) {
+            auto it = id.emplace(set[u], (int32_t)masks.size());
+            if (it.second) masks.push_back(set[u]);
+            rank[u] = it.first->second;
+        }
+    }
+    {
+        std::vector<int32_t> order(masks.size());
+        for (size_t d = 0; d < masks.size(); ++d) order[d] = (int32_t)d;
+        std::sort(order.begin(), order.end(),
+                  [&](int32_t x, int32_t y) { return masks[x] < masks[y]; });
+        std::vector<int32_t> to_rank(masks.size());
+        for (size_t d = 0; d < order.size(); ++d) to_rank[order[d]] = (int32_t)d;
+        for (int64_t u = 0; u < R; ++u) rank[u] = to_rank[rank[u]];
+    }
+    std::vector<int32_t> byset(byw);
+    counting_sort(byset, masks.size(), [&](int32_t u) { return (size_t)rank[u]; });
+    // the needed rows in message order, as contiguous arrays
+    std::vector<int32_t> krow(R), kworker(R), krank(R);
+    for (int64_t k = 0; k < R; ++k) {
+        const int32_t u = byset[k];
+        krow[k] = row[u];
+        kworker[k] = worker[u];
+        krank[k] = rank[u];
+    }
 
     // Alg. 1: one zero-padded block sum per I, as rows of a CSR program
+    std::vector<int32_t> msg_of(R), entry_of(R);    // indexed by position k
     S.enc_ptr.assign(1, 0);
-    S.enc_src.clear();
-    S.msg_worker.clear();
+    S.enc_src.resize(R);
+    S.msg_worker.resize(R);
     S.msg_set.clear();
-    S.message_sets = 0;
-    std::vector<size_t> run_begin, run_len;
-    for (size_t g = 0; g < need.size();) {
-        size_t h = g;
-        while (h < need.size() && need[h].set == need[g].set) ++h;
+    S.message_sets = (int64_t)masks.size();
+    std::vector<int64_t> run_begin, run_len;
+    int32_t x = 0;
+    for (int64_t g = 0; g < R;) {
+        int64_t h = g;
+        while (h < R && krank[h] == krank[g]) ++h;
         run_begin.clear();
         run_len.clear();
-        size_t ell = 0;
-        for (size_t a = g; a < h;) {           // one run per worker of I
-            size_t b = a;
-            while (b < h && need[b].worker == need[a].worker) ++b;
+        int64_t ell = 0;
+        for (int64_t a = g; a < h;) {          // one run per worker of I
+            int64_t b = a;
+            while (b < h && kworker[b] == kworker[a]) ++b;
             run_begin.push_back(a);
             run_len.push_back(b - a);
             ell = std::max(ell, b - a);
             a = b;
         }
-        for (size_t j = 0; j < ell; ++j) {
+        const uint64_t I = set[byset[g]];
+        for (int64_t j = 0; j < ell; ++j) {
             const int32_t m = (int32_t)S.msg_set.size();
             for (size_t w = 0; w < run_begin.size(); ++w) {
                 if (j >= run_len[w]) continue;          // shorter block: zero row
-                Needed &e = need[run_begin[w] + j];
-                e.msg = m;
-                e.entry = (int32_t)S.enc_src.size();
-                S.enc_src.push_back(e.row);
-                S.msg_worker.push_back(e.worker);
+                const int64_t k = run_begin[w] + j;
+                msg_of[k] = m;
+                entry_of[k] = x;
+                S.enc_src[x] = krow[k];
+                S.msg_worker[x] = kworker[k];
+                ++x;
             }
-            S.enc_ptr.push_back((int32_t)S.enc_src.size());
-            S.msg_set.push_back(need[g].set);
+            S.enc_ptr.push_back(x);
+            S.msg_set.push_back(I);
         }
-        ++S.message_sets;
         g = h;
     }
+    // position k of every needed row u
+    std::vector<int32_t> pos(R);
+    for (int64_t k = 0; k < R; ++k) pos[byset[k]] = (int32_t)k;
 
-    // received rows in (worker, row) order; decode program in entry order
-    std::sort(need.begin(), need.end(), [](const Needed &a, const Needed &b) {
-        if (a.worker != b.worker) return a.worker < b.worker;
-        return a.row < b.row;
-    });
-    const int64_t R = (int64_t)need.size();
+    // received rows, and the decode program in entry order
     S.recv_row.resize(R);
     S.recv_ptr.assign(n + 1, 0);
     S.dec_msg.resize(R);
     S.dec_dst.resize(R);
-    for (int64_t u = 0; u < R; ++u) {
-        const Needed &e = need[u];
-        S.recv_row[u] = e.row;
-        ++S.recv_ptr[e.worker + 1];
-        S.dec_msg[e.entry] = e.msg;
-        S.dec_dst[e.entry] = (int32_t)u;
+    S.dec_ptr.resize(R + 1);
+    std::vector<int32_t> entry_w(R);     // entry of the v-th received row
+    for (int64_t v = 0; v < R; ++v) {
+        const int32_t u = byw[v], k = pos[u];
+        S.recv_row[v] = row[u];
+        ++S.recv_ptr[worker[u] + 1];
+        entry_w[v] = entry_of[k];
+        S.dec_msg[entry_of[k]] = msg_of[k];
+        S.dec_dst[entry_of[k]] = (int32_t)v;
     }
     for (int32_t i = 0; i < n; ++i) S.recv_ptr[i + 1] += S.recv_ptr[i];
-    S.dec_ptr.assign(1, 0);
-    S.dec_slot.clear();
+    S.dec_ptr[0] = 0;
     for (int64_t x = 0; x < R; ++x) {
-        const int32_t i = S.msg_worker[x], m = S.dec_msg[x];
-        for (int32_t y = S.enc_ptr[m]; y < S.enc_ptr[m + 1]; ++y) {
-            if (y == x) continue;
-            const int32_t slot = S.slot_of[(int64_t)i * q + S.enc_src[y]];
-            if (slot < 0) return CM_EINVAL;   // unreachable: every other row of I is cached at i
-            S.dec_slot.push_back((int32_t)(i * s + slot));
-        }
-        S.dec_ptr.push_back((int32_t)S.dec_slot.size());
+        const int32_t m = S.dec_msg[x];
+        S.dec_ptr[x + 1] = S.dec_ptr[x] + (S.enc_ptr[m + 1] - S.enc_ptr[m] - 1);
     }
+    S.dec_slot.resize(S.dec_ptr[R]);
+    // slots of the subtracted rows, one worker per thread (its slot table only)
+    std::atomic<bool> consistent{true};
+    bool ok = parallel_for(n, [&](int32_t i) {
+        const int32_t *slot_of = S.slot_of.data() + (int64_t)i * q;
+        for (int64_t v = S.recv_ptr[i]; v < S.recv_ptr[i + 1]; ++v) {
+            const int32_t x = entry_w[v], m = S.dec_msg[x];
+            int32_t at = S.dec_ptr[x];
+            for (int32_t y = S.enc_ptr[m]; y < S.enc_ptr[m + 1]; ++y) {
+                if (y == x) continue;
+                const int32_t slot = slot_of[S.enc_src[y]];
+                if (slot < 0) consistent = false;   // unreachable: the rows of I \ {i} are cached at i
+                S.dec_slot[at++] = (int32_t)(i * s + slot);
+            }
+        }
+    });
+    if (!ok) return CM_ENOMEM;
+    if (!consistent) return CM_EINVAL;
 
     // cache update rule: S_i^{t+1} plus s - q/n rows of C_i^t \ S_i^{t+1}
-    std::vector<uint64_t> next(q, 0);
-    std::vector<char> keepable(q);
-    for (int32_t i = 0; i < n; ++i) {
+    std::vector<std::vector<int32_t>> kept(n);
+    ok = parallel_for(n, [&](int32_t i) {
         const uint64_t bit = 1ull << i;
-        for (int64_t r = 0; r < q; ++r) keepable[r] = (S.cached[r] & bit) && owner1[r] != i;
-        refill(S, t1, i, owner1, keepable, next);
-    }
+        kept[i] = draw_kept(S, t1, i, [&](int64_t r) {
+            return (S.cached[r] & bit) && owner1[r] != i;
+        });
+    });
+    if (!ok) return CM_ENOMEM;
+    std::vector<uint64_t> next = cache_masks(S, owner1, kept);
 
     // commit: received rows of worker i fill, in order, the slots of cache i
     // whose rows were dropped (as many as rows received: both caches hold s)
     S.com_dst.resize(R);
-    for (int32_t i = 0; i < n; ++i) {
+    ok = parallel_for(n, [&](int32_t i) {
         const uint64_t bit = 1ull << i;
-        int64_t u = S.recv_ptr[i];
+        int32_t *slot_of = S.slot_of.data() + (int64_t)i * q;
+        int64_t v = S.recv_ptr[i];
         for (int64_t c = 0; c < s; ++c) {
             const int64_t g = (int64_t)i * s + c;
             const int32_t old = S.slot_row[g];
             if (next[old] & bit) continue;
-            if (u >= S.recv_ptr[i + 1]) return CM_EINVAL;   // unreachable
-            S.slot_of[(int64_t)i * q + old] = -1;
-            S.com_dst[u] = (int32_t)g;
-            ++u;
+            if (v >= S.recv_ptr[i + 1]) {      // unreachable
+                consistent = false;
+                return;
+            }
+            slot_of[old] = -1;
+            S.com_dst[v++] = (int32_t)g;
         }
-        if (u != S.recv_ptr[i + 1]) return CM_EINVAL;       // unreachable
-        for (u = S.recv_ptr[i]; u < S.recv_ptr[i + 1]; ++u) {
-            const int32_t g = S.com_dst[u];
-            S.slot_row[g] = S.recv_row[u];
-            S.slot_of[(int64_t)i * q + S.recv_row[u]] = (int32_t)(g - i * s);
+        if (v != S.recv_ptr[i + 1]) consistent = false;   // unreachable
+        for (v = S.recv_ptr[i]; v < S.recv_ptr[i + 1]; ++v) {
+            const int32_t g = S.com_dst[v];
+            S.slot_row[g] = S.recv_row[v];
+            slot_of[S.recv_row[v]] = (int32_t)(g - i * s);
         }
-    }
+    });
+    if (!ok) return CM_ENOMEM;
+    if (!consistent) return CM_EINVAL;
     S.cached.swap(next);
     S.owner.swap(owner1);
     S.t = t1;
@@ -275,12 +418,13 @@ cm_status cm_shuffle_create(int32_t n, int64_t q, int64_t s, uint64_t partition_
         S->cache_seed = cache_seed;
         S->t = 0;
         draw_partition(*S, 0, S->owner);
-        S->cached.assign(q, 0);
-        std::vector<char> outside(q);
-        for (int32_t i = 0; i < n; ++i) {
-            for (int64_t r = 0; r < q; ++r) outside[r] = S->owner[r] != i;
-            refill(*S, 0, i, S->owner, outside, S->cached);
-        }
+        std::vector<std::vector<int32_t>> kept(n);
+        const cm_shuffle &C = *S;
+        if (!parallel_for(n, [&](int32_t i) {
+                kept[i] = draw_kept(C, 0, i, [&](int64_t r) { return C.owner[r] != i; });
+            }))
+            throw std::bad_alloc();
+        S->cached = cache_masks(*S, S->owner, kept);
         // slots of cache i hold its rows in ascending order
         S->slot_row.resize((size_t)n * s);
         S->slot_of.assign((size_t)n * q, -1);

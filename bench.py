@@ -480,6 +480,9 @@ def bench_shuffle(cm, dev, w: synth.ShuffleWorkload) -> dict:
         t_plan.append(t1 - t0)
         t_up.append(t2 - t1)
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        # queue the three launches behind a short device sleep, so that the
+        # events time the kernels and not the host's launch gap
+        torch.cuda._sleep(2_000_000)
         ev[0].record()
         sh.encode("xor", A, M)
         ev[1].record()

@@ -47,6 +47,9 @@ cudaError_t launch_encode_f32(const CodeParams &cp, const float *A, int64_t lda,
                               float *par, int64_t ldp, int32_t *status, cudaStream_t s);
 cudaError_t launch_encode_bf16(const CodeParams &cp, const uint16_t *A, int64_t lda,
                                uint16_t *par, int64_t ldp, int32_t *status, cudaStream_t s);
+// Rows per K2 work unit for b = 1 (8 or 4) given L, the computed workers
+// and the warps of the persistent grid.
+int matvec_rows_per_unit(int64_t L, int nw, int64_t warps);
 // `only` = 0: all n workers; otherwise the workers of the first k set bits.
 cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda,
                           const float *par, int64_t ldp, const float *X, int b,

@@ -381,6 +381,23 @@ cudaError_t launch_bp(MatvecArgs a, const float *A, int64_t lda, const float *pa
 
 }  // namespace
 
+// Rows per work unit for b = 1.  The persistent grid takes units in rounds of
+// `warps`; a partly filled last round leaves the other warps idle, which on a
+// small problem (a few rounds) costs up to a fifth of the time.  4-row units
+// (with a ring twice as deep, the same bytes in flight) fill the rounds more
+// evenly but add a round's X staging and ring start-up each time; measured on
+// this part, they pay off when they fill the rounds at least 2 points better.
+// (2-row units ran at two thirds of the bandwidth: per-step costs dominate.)
+int matvec_rows_per_unit(int64_t L, int nw, int64_t warps)
+{
+    auto fill = [&](int R) {
+        const int64_t units = (L + R - 1) / R * nw;
+        const int64_t rounds = (units + warps - 1) / warps;
+        return (double)units / (double)(rounds * warps);
+    };
+    return fill(4) >= fill(8) + 0.02 ? 4 : 8;
+}
+
 cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, const float *par,
                           int64_t ldp, const float *X, int b, double *Yt, int32_t *status,
                           uint32_t only, cudaStream_t s)
@@ -401,7 +418,11 @@ cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, con
     a.b = b;
     a.groups = 0;
     a.fast16 = b == 1 && ((uintptr_t)X & 15u) == 0;
-    if (b == 1) return launch_bp<1, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
+    if (b == 1) {
+        if (matvec_rows_per_unit(a.L, a.nw, (int64_t)cm_sm_count() * 8) == 4)
+            return launch_bp<1, 4, 12, 16, 8>(a, A, lda, par, ldp, s);
+        return launch_bp<1, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
+    }
     if (b <= 4) return launch_bp<4, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
     return launch_bp<8, 8, 6, 64, 8>(a, A, lda, par, ldp, s);
 }

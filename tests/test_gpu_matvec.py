@@ -140,6 +140,41 @@ def test_path_matches_oracle(cm, orc, n, k, m, d, b, lda):
     assert rel_l2_cols(r["Y"].cpu().numpy(), want).max() <= 1e-4
 
 
+def _rows_per_unit(L, nw, warps):
+    """The unit height rule of the b = 1 launch, restated: 4-row units when
+    they fill the grid's rounds at least 2 points better than 8-row ones."""
+    def fill(R):
+        units = -(-L // R) * nw
+        rounds = -(-units // warps)
+        return units / (rounds * warps)
+    return 4 if fill(4) >= fill(8) + 0.02 else 8
+
+
+@pytest.mark.parametrize("n,k,m,d,want_R", [(32, 24, 65536, 64, 8), (10, 5, 12000, 256, 4),
+                                            (20, 10, 8000, 128, 8), (6, 3, 1201, 300, 4)])
+def test_unit_heights_at_b1(cm, orc, n, k, m, d, want_R):
+    # b = 1 products run 8- or 4-row units depending on how the units fill the
+    # persistent grid; both heights must give the same results
+    warps = torch.cuda.get_device_properties(0).multi_processor_count * 8
+    L = -(-m // k)
+    if _rows_per_unit(L, n, warps) != want_R:
+        pytest.skip("this GPU's SM count selects another height for the shape")
+    r = run_path(cm, orc, n, k, m, d, 1, seed=31)
+    check_workers(orc, n, k, r["A_cpu"], r["par"], r["X_cpu"], r["Yt"], r["code"].L)
+    want = orc.matmul(r["A_cpu"].numpy(), r["X_cpu"].numpy())
+    assert rel_l2_cols(r["Y"].cpu().numpy(), want).max() <= 1e-4
+    # survivors only: the rule over nw = k workers may pick another height;
+    # the blocks agree to the fp32 partial rounding
+    Yt2 = cm.matvec_survivors(r["code"], r["A"], r["par"], r["X"], r["mask"])
+    torch.cuda.synchronize()
+    sel = r["code"].select_decodable(r["mask"])
+    got, ref = Yt2.cpu().numpy(), r["Yt"].cpu().numpy()
+    for j in range(n):
+        if (sel >> j) & 1:
+            blk = slice(j * L, (j + 1) * L)
+            assert rel_l2_cols(got[blk], ref[blk]).max() <= 1e-6
+
+
 @pytest.mark.parametrize("b", [1, 4, 8, 3])
 def test_misaligned_x_uses_general_staging(cm, orc, b):
     n, k, m, d = 6, 3, 500, 301

@@ -88,6 +88,7 @@ def check_encode_bf16(orc, n, k, A, P, par):
     (5, 4, 517, 200, 80),        # d not a multiple of 64, N not of 256, L not of 128
     (16, 12, 1537, 512, 512),    # several row and column tiles
     (4, 3, 40, 64, 16),          # tiny
+    (6, 3, 900, 128, 300),       # 3 row tiles per block, ragged last tile and columns
 ])
 def test_coded_gemm_matches_oracle(cm, orc, n, k, m, d, N):
     r = run(cm, n, k, m, d, N)

@@ -568,9 +568,17 @@ def bench_gd(cm, dev, steps: int) -> dict:
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / w.iters
     nb = gd_iter_bytes(w, cA.L, cAT.L)
+    # the same 50 iterations as plain (uncoded) fp64 gradient descent on the
+    # device: the coded iterate must follow it (Sec. III-E: decoding is exact)
+    A64, y64 = A.double(), y.double()
+    x64 = torch.zeros(w.d, dtype=torch.float64, device=dev)
+    for t in range(w.iters):
+        x64 -= w.eta * (A64.t() @ (A64 @ x64 - y64))
+    rel = float(torch.linalg.norm(x.double() - x64) / torch.linalg.norm(x64))
+    del A64
     return {"workload": w.name, "iters": w.iters, "ms_per_iter": ms,
             "gbs": nb / (ms * 1e-3) / 1e9, "launches_per_iter": 4,
-            "status": int(status.item())}
+            "x50_rel_err_vs_fp64_gd": rel, "status": int(status.item())}
 
 
 def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
@@ -642,10 +650,16 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
     torch.cuda.synchronize()
     enc_us = e0.elapsed_time(e1) * 1e3
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(reps)]
+    # inputs that fit in L2 are flushed from it before every repeat (a write of
+    # a buffer larger than L2, outside the timed events)
+    flush = (torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+             if step_bytes(w, code.L)["matvec"] < (200 << 20) else None)
     # keep the device queue ahead of the host: the per-call events then time
     # the kernels, not the host's launch gaps
     torch.cuda._sleep(int(2e6 + reps * 4e5))
     for r in range(reps):
+        if flush is not None:
+            flush.fill_(r & 255)
         ev[r][0].record()
         cm.matvec(code, A, parity, X, Yt, status=status)
         ev[r][1].record()
@@ -655,7 +669,8 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
     mv = np.array([e[0].elapsed_time(e[1]) * 1e3 for e in ev])
     dec = np.array([e[1].elapsed_time(e[2]) * 1e3 for e in ev])
     nb = step_bytes(w, code.L)
-    return {"workload": w.name, "repeats": reps, "encode_us": enc_us,
+    return {"workload": w.name, "repeats": reps, "l2_flushed": flush is not None,
+            "encode_us": enc_us,
             "encode_gbs": nb["encode"] / (enc_us * 1e-6) / 1e9,
             "matvec_us_median": float(np.median(mv)), "matvec_us_p95": float(np.percentile(mv, 95)),
             "matvec_gbs_median": nb["matvec"] / (np.median(mv) * 1e-6) / 1e9,

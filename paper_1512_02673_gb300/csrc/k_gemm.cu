@@ -6,38 +6,56 @@
 // j >= k rows of the bf16 parity buffer (both K-major, i.e. row-major); B is
 // given transposed (N x d, K-major).
 //
-// Tiles.  128 x 256 output tiles that never straddle a worker block: worker j
-// has ceil(L / 128) row tiles; the last one reads past the block (zeros past
-// m or the parity buffer, or the next block's rows) and stores only rows < L.
-// Tile order: column tile fastest, so the 16 column tiles of one row tile run
-// at the same time on different SMs and the 2 MB row slab of A~ comes from
-// HBM once and from L2 after that; Bt (64 MB) stays L2-resident.
+// Two-SM tiles.  A cluster of two CTAs on a pair of SMs computes one 256 x 256
+// output tile with tcgen05.mma.cta_group::2 (M = 256 over the pair, N = 256,
+// K = 16): CTA r stages rows [128 r, 128 r + 128) of the A~ tile and rows
+// [128 r, 128 r + 128) of the Bt tile, and accumulates its 128 output rows in
+// its own tensor memory.  Per K block of 64 each SM thus stages 32 KB (instead
+// of 48 KB for a one-SM 128 x 256 tile), which leaves six stages in shared
+// memory and halves the Bt bytes every SM reads per MMA: the one-SM version
+// was held near 0.8 of peak by shared-memory traffic (TMA fills plus tensor-
+// core operand reads).
 //
-// One persistent CTA per SM, warp-specialised:
-//   warp 0 lane 0  TMA producer: 128B-swizzled boxes of A~ (128 x 64) and Bt
-//                  (256 x 64) into a 4-stage shared-memory ring (48 KB per stage);
-//   warp 1         allocates 512 TMEM columns (two 128 x 256 fp32 accumulators);
-//                  lane 0 issues tcgen05.mma.cta_group::1.kind::f16 (M=128,
-//                  N=256, K=16, four per stage) and tcgen05.commit to free a
-//                  stage / publish an accumulator;
+// Tiles never straddle a worker block: worker j has ceil(L / 128) row tiles,
+// paired as (2 i, 2 i + 1) (the second one virtual past the block when the
+// count is odd: it loads zeros or foreign rows, and stores nothing); a tile's
+// last rows may read past the block and are not stored.  Pair order: column
+// tile fastest, so the 16 column tiles of one row pair run together and the
+// A~ row slab comes from HBM once; Bt (64 MB) stays L2-resident.
+//
+// One persistent CTA per SM, warp-specialised, in both CTAs of a pair:
+//   warp 0 lane 0  TMA producer of the CTA's halves (128B-swizzled 128 x 64
+//                  boxes) into a 6-stage ring; every load completes on the
+//                  leader CTA's stage barrier, which the leader's producer
+//                  arms with the bytes of both CTAs;
+//   warp 1         allocates 512 TMEM columns together with the peer
+//                  (cta_group::2: two 128 x 256 fp32 accumulators per CTA);
+//                  in the leader (rank 0), lane 0 issues the MMAs and
+//                  tcgen05.commit, multicast to both CTAs, to free a stage or
+//                  publish an accumulator;
 //   warps 2..5     epilogue: tcgen05.ld (32 lanes x 32 columns per load) from
-//                  the accumulator of their TMEM lane quarter, fp32 stores to Ct,
-//                  then release the accumulator, so the epilogue of one tile
+//                  the CTA's accumulator, fp32 stores to Ct, then release of
+//                  the accumulator on the leader's barrier (the peer's
+//                  threads arrive remotely), so the epilogue of one tile
 //                  overlaps the MMAs of the next.
 // Every wait is bounded (about 2 s); on a time-out the kernel writes
 // CM_ETIMEOUT to the status word, every role stops, outstanding work is
-// drained with bounded waits and the TMEM is freed before the CTA exits.
+// drained with bounded waits, and both CTAs meet at a cluster barrier before
+// the TMEM is freed and they exit, so neither touches the other's shared
+// memory while it is not live.
 #include "cm_internal.cuh"
 #include "tma.cuh"
 
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4, ACCS = 2;
+constexpr int BM = 128;              // rows per CTA (256 per pair)
+constexpr int BN = 256, BK = 64, STAGES = 6, ACCS = 2;
+constexpr int BNH = BN / 2;          // Bt rows staged per CTA
 constexpr int TMEM_COLS = ACCS * BN;   // 512
 constexpr int kThreads = 192;
 constexpr uint32_t A_BYTES = BM * BK * 2;
-constexpr uint32_t B_BYTES = BN * BK * 2;
-constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr uint32_t B_BYTES = BNH * BK * 2;
+constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;   // 32 KB per CTA
 constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
 
 struct GemmArgs {
@@ -46,13 +64,14 @@ struct GemmArgs {
     int32_t *status;
     int64_t L;
     int32_t n, k, N;
-    int32_t mtiles;    // row tiles per worker block
+    int32_t mtiles;    // 128-row tiles per worker block
+    int32_t mpairs;    // row-tile pairs per worker block (ceil(mtiles / 2))
     int32_t ntiles;    // column tiles
     int32_t kblocks;   // 64-wide K blocks
-    int64_t tiles;
+    int64_t pairs;     // (worker, row pair, column tile) work items
 };
 
-// ---- tcgen05 helpers (inline PTX) ---------------------------------------------------
+// ---- tcgen05 / cluster helpers (inline PTX) ------------------------------------------
 
 // Shared-memory matrix descriptor of a K-major operand tile written by TMA with
 // 128-byte swizzling: 8-row groups 1024 bytes apart (stride byte offset), the
@@ -65,31 +84,98 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr)
 }
 
 // Instruction descriptor for kind::f16: fp32 accumulator, bf16 A and B, both
-// K-major, N = BN, M = BM.
+// K-major, N = BN, M = 256 (the pair).
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                            ((uint32_t)(BM >> 4) << 24);
+                            ((uint32_t)((2 * BM) >> 4) << 24);
 
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                         uint32_t accumulate)
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                              uint32_t accumulate)
 {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
         "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
         : "memory");
 }
 
-__device__ __forceinline__ void mma_commit(uint64_t *bar)
+// Arrive on the mbarrier at this offset in both CTAs of the pair once the
+// MMAs issued so far have completed.
+__device__ __forceinline__ void mma_commit_pair(uint64_t *bar)
 {
     asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster"
+        ".b64 [%0], %1;\n" ::"r"(cm_smem_u32(bar)),
+        "h"((uint16_t)0x3)
+        : "memory");
+}
+
+// Arrive on a local mbarrier once this thread's MMAs have completed.
+__device__ __forceinline__ void mma_commit_local(uint64_t *bar)
+{
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];\n" ::"r"(
             cm_smem_u32(bar))
         : "memory");
 }
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory"); }
+
+__device__ __forceinline__ uint32_t cluster_ctarank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;\n" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_id()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%clusterid.x;\n" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_count()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%nclusterid.x;\n" : "=r"(r));
+    return r;
+}
+
+// Shared::cluster address of the same shared-memory location in CTA `rank`.
+__device__ __forceinline__ uint32_t map_to_rank(const void *p, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(r) : "r"(cm_smem_u32(p)), "r"(rank));
+    return r;
+}
+
+// Every thread of both CTAs: release its earlier writes, wait for the others.
+__device__ __forceinline__ void cluster_sync()
+{
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;\n" ::: "memory");
+}
+
+// Arrive (release, cluster scope) on an mbarrier given by its shared::cluster
+// address, possibly in the peer CTA.
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cl_addr)
+{
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];\n" ::"r"(cl_addr)
+                 : "memory");
+}
+
+// 2-D TMA load into this CTA's shared memory whose completion is counted on an
+// mbarrier of either CTA of the pair (shared::cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(void *smem_dst, const CUtensorMap *map, int32_t x,
+                                                 int32_t y, uint32_t bar_cl)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];\n" ::"r"(cm_smem_u32(smem_dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar_cl)
+        : "memory");
+}
 
 // 32 lanes x 32 consecutive fp32 columns of TMEM into 32 registers per thread.
 __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32])
@@ -114,19 +200,20 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32])
 
 struct Tile {
     int j;          // worker
-    int mt;         // row tile within the worker block
+    int mt;         // 128-row tile within the worker block (may be virtual)
     int n0;         // first output column
     bool parity;    // rows come from the parity buffer
     int32_t y;      // row coordinate in A or in the parity buffer
 };
 
-__device__ __forceinline__ Tile tile_of(const GemmArgs &g, int64_t t)
+// CTA `rank`'s half of work item p: row tile 2 (p's row pair) + rank.
+__device__ __forceinline__ Tile tile_of(const GemmArgs &g, int64_t p, int rank)
 {
     Tile x;
-    const int nt = (int)(t % g.ntiles);
-    const int64_t rest = t / g.ntiles;
-    x.mt = (int)(rest % g.mtiles);
-    x.j = (int)(rest / g.mtiles);
+    const int nt = (int)(p % g.ntiles);
+    const int64_t rest = p / g.ntiles;
+    x.mt = 2 * (int)(rest % g.mpairs) + rank;
+    x.j = (int)(rest / g.mpairs);
     x.n0 = nt * BN;
     x.parity = x.j >= g.k;
     const int64_t r0 = (int64_t)x.mt * BM;
@@ -149,30 +236,34 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int rank = (int)cluster_ctarank();
+    const bool leader = rank == 0;
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
-            cm_mbar_init(&full[s], 1);
-            cm_mbar_init(&empty[s], 1);
+            cm_mbar_init(&full[s], 1);    // leader: its producer's arrive (+ both CTAs' bytes)
+            cm_mbar_init(&empty[s], 1);   // the leader's MMA commit
         }
         for (int a = 0; a < ACCS; ++a) {
-            cm_mbar_init(&tfull[a], 1);
-            cm_mbar_init(&tempty[a], 128);
+            cm_mbar_init(&tfull[a], 1);                // the leader's MMA commit
+            cm_mbar_init(&tempty[a], 2 * 4 * 32);      // leader: both CTAs' epilogue threads
         }
         cm_mbar_init(drain, 1);
         *abort_flag = 0;
         cm_fence_mbar_init();
     }
-    if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
+    if (warp == 1) {   // with the peer's warp 1: the same columns in both CTAs
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(
                          cm_smem_u32(tmem_slot)),
                      "r"(TMEM_COLS)
                      : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;\n" ::: "memory");
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    const int64_t first = cluster_id(), stride = cluster_count();
+    cluster_sync();   // both CTAs' barriers exist before either signals the other
 
     auto fail = [&]() {
         *abort_flag = 1;
@@ -180,12 +271,12 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
     };
 
     if (warp == 0 && lane == 0) {
-        // ---- TMA producer ----
+        // ---- TMA producer (both CTAs) ----
         int s = 0;
         uint32_t ph = 0;
         int64_t issued = 0;
-        for (int64_t t = blockIdx.x; t < g.tiles && !*abort_flag; t += gridDim.x) {
-            const Tile x = tile_of(g, t);
+        for (int64_t p = first; p < g.pairs && !*abort_flag; p += stride) {
+            const Tile x = tile_of(g, p, rank);
             const CUtensorMap *ma = x.parity ? &tmP : &tmA;
             for (int kb = 0; kb < g.kblocks; ++kb) {
                 if (*abort_flag || !cm_mbar_wait(&empty[s], ph ^ 1u)) {
@@ -193,9 +284,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                     break;
                 }
                 unsigned char *sa = base + s * STAGE_BYTES;
-                cm_mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
-                cm_tma_load_2d(sa, ma, kb * BK, x.y, &full[s]);
-                cm_tma_load_2d(sa + A_BYTES, &tmB, kb * BK, x.n0, &full[s]);
+                const uint32_t bar = map_to_rank(&full[s], 0);   // the leader's stage barrier
+                if (leader) cm_mbar_arrive_expect_tx(&full[s], 2 * STAGE_BYTES);
+                tma_load_2d_pair(sa, ma, kb * BK, x.y, bar);
+                tma_load_2d_pair(sa + A_BYTES, &tmB, kb * BK, x.n0 + rank * BNH, bar);
                 ++issued;
                 if (++s == STAGES) {
                     s = 0;
@@ -203,7 +295,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                 }
             }
         }
-        if (*abort_flag) {
+        if (*abort_flag && leader) {
             // drain: wait (bounded) for the last phase of every stage in flight
             for (int i = 0; i < STAGES && i < issued; ++i) {
                 if (--s < 0) {
@@ -213,11 +305,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                 cm_mbar_wait(&full[s], ph, 100000000ull);
             }
         }
-    } else if (warp == 1 && lane == 0) {
-        // ---- MMA issuer ----
+    } else if (warp == 1 && lane == 0 && leader) {
+        // ---- MMA issuer (leader only) ----
         int s = 0, acc = 0;
         uint32_t ph = 0, aph = 0;
-        for (int64_t t = blockIdx.x; t < g.tiles && !*abort_flag; t += gridDim.x) {
+        for (int64_t p = first; p < g.pairs && !*abort_flag; p += stride) {
             if (!cm_mbar_wait(&tempty[acc], aph ^ 1u)) {
                 fail();
                 break;
@@ -236,31 +328,31 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                 const uint32_t sb = sa + A_BYTES;
 #pragma unroll
                 for (int kk = 0; kk < BK / 16; ++kk)
-                    mma_bf16(d_tmem, smem_desc_sw128(sa + kk * 32), smem_desc_sw128(sb + kk * 32),
-                             (kb | kk) != 0);
-                mma_commit(&empty[s]);   // the stage is free once these MMAs finish
+                    mma_bf16_pair(d_tmem, smem_desc_sw128(sa + kk * 32),
+                                  smem_desc_sw128(sb + kk * 32), (kb | kk) != 0);
+                mma_commit_pair(&empty[s]);   // the stage is free in both CTAs
                 if (++s == STAGES) {
                     s = 0;
                     ph ^= 1u;
                 }
             }
             if (!ok) break;
-            mma_commit(&tfull[acc]);     // accumulator ready for the epilogue
+            mma_commit_pair(&tfull[acc]);     // both halves of the accumulator are ready
             if (++acc == ACCS) {
                 acc = 0;
                 aph ^= 1u;
             }
         }
         // all MMAs issued by this thread have completed once `drain` fires
-        mma_commit(drain);
+        mma_commit_local(drain);
         cm_mbar_wait(drain, 0, 100000000ull);
     } else if (warp >= 2) {
-        // ---- epilogue: TMEM -> registers -> Ct ----
+        // ---- epilogue (both CTAs): TMEM -> registers -> Ct ----
         const int q = warp & 3;                  // TMEM lane quarter of this warp
-        const int row = q * 32 + lane;           // row of the tile
+        const int row = q * 32 + lane;           // row of the CTA's tile
         int acc = 0;
         uint32_t aph = 0;
-        for (int64_t t = blockIdx.x; t < g.tiles; t += gridDim.x) {
+        for (int64_t p = first; p < g.pairs; p += stride) {
             // warp-uniform decisions: tcgen05.ld below is .sync.aligned
             if (__shfl_sync(0xffffffffu, *abort_flag, 0)) break;
             const bool ok = cm_mbar_wait(&tfull[acc], aph);
@@ -269,7 +361,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                 break;
             }
             tc_fence_after();
-            const Tile x = tile_of(g, t);
+            const Tile x = tile_of(g, p, rank);
             const int64_t r = (int64_t)x.mt * BM + row;
             const bool valid = r < g.L;
             float *dst = g.Ct + ((int64_t)x.j * g.L + r) * g.ldc + x.n0;
@@ -280,21 +372,21 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
                 tmem_load32(taddr + c * 32, v);
                 const int col = x.n0 + c * 32;
                 if (valid && col < g.N) {
-                    float *p = dst + c * 32;
+                    float *o = dst + c * 32;
                     if (col + 32 <= g.N && ((g.ldc & 3) == 0)) {
 #pragma unroll
                         for (int i = 0; i < 32; i += 4)
-                            *reinterpret_cast<float4 *>(p + i) =
+                            *reinterpret_cast<float4 *>(o + i) =
                                 make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
                     } else {
 #pragma unroll
                         for (int i = 0; i < 32; ++i)
-                            if (col + i < g.N) p[i] = v[i];
+                            if (col + i < g.N) o[i] = v[i];
                     }
                 }
             }
             tc_fence_before();
-            cm_mbar_arrive(&tempty[acc]);
+            mbar_arrive_cluster(map_to_rank(&tempty[acc], 0));   // release on the leader
             if (++acc == ACCS) {
                 acc = 0;
                 aph ^= 1u;
@@ -303,10 +395,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
     }
     tc_fence_before();
     __syncthreads();
+    cluster_sync();   // neither CTA has a copy, commit or arrival left for the other
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base),
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;\n" ::"r"(tmem_base),
                      "r"(TMEM_COLS)
                      : "memory");
     }
@@ -326,7 +419,7 @@ cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t l
                          (uint64_t)(cp.n - cp.k) * cp.L, (uint64_t)ldp * 2, BK, BM,
                          CU_TENSOR_MAP_SWIZZLE_128B) ||
         !cm_make_tmap_2d(&tmB, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, Bt, d, (uint64_t)N,
-                         (uint64_t)ldb * 2, BK, BN, CU_TENSOR_MAP_SWIZZLE_128B))
+                         (uint64_t)ldb * 2, BK, BNH, CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
     GemmArgs g;
     g.Ct = Ct;
@@ -337,15 +430,33 @@ cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t l
     g.k = cp.k;
     g.N = N;
     g.mtiles = (int)((cp.L + BM - 1) / BM);
+    g.mpairs = (g.mtiles + 1) / 2;
     g.ntiles = (N + BN - 1) / BN;
     g.kblocks = (int)((cp.d + BK - 1) / BK);
-    g.tiles = (int64_t)cp.n * g.mtiles * g.ntiles;
+    g.pairs = (int64_t)cp.n * g.mpairs * g.ntiles;
     cudaError_t e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    int64_t grid = cm_sm_count();
-    if (grid < 1) grid = 1;
-    if (grid > g.tiles) grid = g.tiles;
-    gemm_kernel<<<(unsigned)grid, kThreads, SMEM_BYTES, s>>>(tmA, tmP, tmB, g);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(2 * (unsigned)((cm_sm_count() + 1) / 2));
+    // persistent: as many pairs as can be resident at once
+    int clusters = 0;
+    e = cudaOccupancyMaxActiveClusters(&clusters, gemm_kernel, &cfg);
+    if (e != cudaSuccess) return e;
+    if (clusters < 1) return cudaErrorInvalidConfiguration;
+    if (clusters > g.pairs) clusters = (int)g.pairs;
+    cfg.gridDim = dim3(2 * (unsigned)clusters);
+    e = cudaLaunchKernelEx(&cfg, gemm_kernel, tmA, tmP, tmB, g);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

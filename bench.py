@@ -247,8 +247,8 @@ def run_reference(args, world, rank):
 # the 152-SM mat-vec grid exactly two rounds of 8-row units.
 PROFILE = synth.Workload("coded mat-multi-vec (32,24) 14592x16384 b=8 (profiling case)",
                          m=14592, d=16384, b=8, n=32, k=24, data_device="cuda")
-PROFILE_GEMM = synth.Workload("coded GEMM bf16 (16,12) 16384x8192x4096 (profiling case)",
-                              m=16384, d=8192, b=0, n=16, k=12, dtype="bf16", gemm_n=4096,
+PROFILE_GEMM = synth.Workload("coded GEMM bf16 (16,12) 18432x8192x4096 (profiling case)",
+                              m=18432, d=8192, b=0, n=16, k=12, dtype="bf16", gemm_n=4096,
                               data_device="cuda")
 PROFILE_SHUFFLE = synth.ShuffleWorkload("coded shuffling n=8 q=524288 s=q/4 r=256 "
                                         "(profiling case)", n=8, q=1 << 19, s=1 << 17,

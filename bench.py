@@ -458,8 +458,9 @@ def bench_shuffle(cm, dev, w: synth.ShuffleWorkload) -> dict:
     """Coded shuffling (Sec. IV) on the GPU: per transition the host plans
     Alg. 1 and the cache update, then encode, decode by subtraction and the
     cache commit run on the device (xor sums: exact, the same bytes as real
-    sums).  Checks after the last transition that every cache slot holds its
-    data row exactly."""
+    sums).  Then the same transitions with the planner on the device.  Checks
+    after the last transition of each that every cache slot holds its data
+    row exactly."""
     peaks = measured_peaks()
     A = synth.shuffle_rows(w, dev)
     sh = cm.Shuffle(w.n, w.q, w.s, synth.SHUFFLE_PARTITION_SEED, synth.SHUFFLE_CACHE_SEED)
@@ -500,6 +501,33 @@ def bench_shuffle(cm, dev, w: synth.ShuffleWorkload) -> dict:
         rows["uncoded"].append(st["uncoded_rows"])
     _, slots = sh.caches()
     exact = bool(torch.equal(caches, A[torch.from_numpy(slots.reshape(-1)).long().to(dev)]))
+    del sh
+    # the same transitions planned on the device: plan time (CUDA events on
+    # the planner's stream, and wall time including the read-back of the
+    # counts) and the wall time of a whole transition (plan + data plane)
+    shd = cm.Shuffle(w.n, w.q, w.s, synth.SHUFFLE_PARTITION_SEED, synth.SHUFFLE_CACHE_SEED)
+    shd.device_init()
+    caches = shd.fill(A, caches)
+    d_plan_ev, d_plan_wall, d_trans_wall = [], [], []
+    for t in range(w.transitions):
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0 = time.perf_counter()
+        e0.record()
+        shd.device_next()
+        e1.record()
+        t1 = time.perf_counter()
+        shd.encode("xor", A, M)
+        shd.decode("xor", M, caches, w.r, Rx)
+        shd.commit(Rx, caches, w.r)
+        torch.cuda.synchronize()
+        t2 = time.perf_counter()
+        if t > 0:
+            d_plan_ev.append(e0.elapsed_time(e1))
+            d_plan_wall.append(1e3 * (t1 - t0))
+            d_trans_wall.append(1e3 * (t2 - t0))
+    _, slots = shd.caches()
+    exact_d = bool(torch.equal(caches, A[torch.from_numpy(slots.reshape(-1)).long().to(dev)]))
     rc, ru = cm.shuffle_rates(w.n, w.q, w.s)
     kern = {}
     for k in ms:
@@ -515,6 +543,10 @@ def bench_shuffle(cm, dev, w: synth.ShuffleWorkload) -> dict:
             "rows": {"coded_mean": float(np.mean(rows["coded"][1:])),
                      "uncoded_mean": float(np.mean(rows["uncoded"][1:])),
                      "theorem_R_c": rc, "R_u": ru},
+            "device_planner": {"plan_ms": float(np.mean(d_plan_ev)),
+                               "plan_wall_ms": float(np.mean(d_plan_wall)),
+                               "transition_wall_ms": float(np.mean(d_trans_wall)),
+                               "caches_exact": exact_d},
             "roofline_peak_gbs": peaks["hbm_gbs"], "caches_exact": exact}
 
 

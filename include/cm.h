@@ -386,6 +386,34 @@ cm_status cm_shuffle_decode(const cm_shuffle *shuffle, const void *workspace, cm
                             const void *M, int64_t ldm, const void *caches, int64_t ldc,
                             int64_t r, void *Rx, int64_t ldr, cm_stream_t stream);
 
+/* ---- the planner on the device ---------------------------------------------
+ * The same plan as cm_shuffle_next (bit for bit: partition, messages,
+ * programs, cache update, slot tables), computed on the GPU with the state
+ * resident in a caller-owned workspace, for n <= 16.  After
+ * cm_shuffle_device_init the instance is in device mode: cm_shuffle_next and
+ * cm_shuffle_upload return CM_EINVAL, cm_shuffle_device_next plans each
+ * transition, the data-plane calls take this workspace, and cm_shuffle_plan,
+ * cm_shuffle_received and cm_shuffle_caches copy their tables out of it
+ * (synchronously). */
+
+/* Bytes of device workspace for the device planner (0 if n > 16): the row
+ * programs of cm_shuffle_workspace_bytes first, then the resident state and
+ * scratch (about 4 q (n + 5) + 4 n s + 100 q + 24 max(q, n s) bytes). */
+size_t cm_shuffle_device_workspace_bytes(const cm_shuffle *shuffle);
+
+/* Moves the current host state (and, after a transition, its programs) into
+ * `workspace` (16-byte aligned, >= cm_shuffle_device_workspace_bytes) and
+ * switches the instance to device mode.  Synchronises `stream`. */
+cm_status cm_shuffle_device_init(cm_shuffle *shuffle, void *workspace, size_t bytes,
+                                 cm_stream_t stream);
+
+/* Plans the transition t -> t+1 on the device (about 40 launches on
+ * `stream`), then reads back its counts (synchronising `stream`); stats is
+ * nullable.  The programs are then in place for cm_shuffle_encode, _decode
+ * and _commit. */
+cm_status cm_shuffle_device_next(cm_shuffle *shuffle, void *workspace, size_t bytes,
+                                 cm_shuffle_stats *stats, cm_stream_t stream);
+
 /* Cache update (workers): writes every received row into the cache slot it
  * takes over, turning the caches C^t into C^{t+1}.  Run after the decode of
  * the same transition. */

@@ -90,6 +90,9 @@ def lib() -> ctypes.CDLL:
             "cm_shuffle_encode": (st, [vp, vp, st, vp, i64, i64, vp, i64, vp]),
             "cm_shuffle_decode": (st, [vp, vp, st, vp, i64, vp, i64, i64, vp, i64, vp]),
             "cm_shuffle_commit": (st, [vp, vp, vp, i64, i64, vp, i64, vp]),
+            "cm_shuffle_device_workspace_bytes": (sz, [vp]),
+            "cm_shuffle_device_init": (st, [vp, vp, sz, vp]),
+            "cm_shuffle_device_next": (st, [vp, vp, sz, vp, vp]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -559,6 +562,30 @@ class Shuffle:
 
     def _wsp(self):
         return ctypes.c_void_p(self._ws.data_ptr() if self._ws is not None else 0)
+
+    # ---- the planner on the device ----
+
+    def device_workspace_bytes(self) -> int:
+        return int(lib().cm_shuffle_device_workspace_bytes(self._h))
+
+    def device_init(self, device=None):
+        """Moves the state to a device workspace; later transitions are planned
+        on the GPU (device_next) and the data plane uses that workspace."""
+        nb = self.device_workspace_bytes()
+        if nb == 0:
+            raise ValueError("the device planner handles n <= 16")
+        ws = torch.empty(nb, dtype=torch.uint8, device=device or torch.device("cuda"))
+        _check(lib().cm_shuffle_device_init(self._h, ctypes.c_void_p(ws.data_ptr()), nb,
+                                            _stream()), "cm_shuffle_device_init")
+        self._ws = ws
+
+    def device_next(self) -> dict:
+        """Plans the next transition on the device; returns its statistics."""
+        st = _ShuffleStats()
+        _check(lib().cm_shuffle_device_next(self._h, self._wsp(), self._ws.numel(),
+                                            ctypes.byref(st), _stream()),
+               "cm_shuffle_device_next")
+        return {f: int(getattr(st, f)) for f, _ in _ShuffleStats._fields_}
 
     def fill(self, A: torch.Tensor, caches: torch.Tensor | None = None) -> torch.Tensor:
         r = A.shape[1]

@@ -215,6 +215,7 @@ size_t cm_shuffle_workspace_bytes(const cm_shuffle *S)
 cm_status cm_shuffle_upload(cm_shuffle *S, void *ws, size_t bytes, cm_stream_t stream)
 {
     if (!S || !ws || !aligned16(ws) || bytes < cm_shuffle_workspace_bytes(S)) return CM_EINVAL;
+    if (S->device_ws) return CM_EINVAL;   // the device planner keeps its programs in place
     const ShuffleLayout L = shuffle_layout(S->n, S->q, S->s);
     cudaStream_t st = (cudaStream_t)stream;
     int32_t *w = static_cast<int32_t *>(ws);
@@ -258,7 +259,7 @@ cm_status cm_shuffle_encode(const cm_shuffle *S, const void *ws, cm_shuffle_op o
         !rows_ok(M, ldm, r))
         return CM_EINVAL;
     const ShuffleLayout L = shuffle_layout(S->n, S->q, S->s);
-    RowProgram p{(int64_t)S->msg_set.size(), at(ws, L.enc_ptr), at(ws, L.enc_src), nullptr,
+    RowProgram p{S->n_coded, at(ws, L.enc_ptr), at(ws, L.enc_src), nullptr,
                  nullptr};
     cudaStream_t st = (cudaStream_t)stream;
     if (op == CM_SHUFFLE_ADD)
@@ -278,7 +279,7 @@ cm_status cm_shuffle_decode(const cm_shuffle *S, const void *ws, cm_shuffle_op o
         !rows_ok(caches, ldc, r) || !rows_ok(Rx, ldr, r))
         return CM_EINVAL;
     const ShuffleLayout L = shuffle_layout(S->n, S->q, S->s);
-    RowProgram p{(int64_t)S->dec_msg.size(), at(ws, L.dec_ptr), at(ws, L.dec_slot),
+    RowProgram p{S->n_recv, at(ws, L.dec_ptr), at(ws, L.dec_slot),
                  at(ws, L.dec_msg), at(ws, L.dec_dst)};
     cudaStream_t st = (cudaStream_t)stream;
     if (op == CM_SHUFFLE_ADD)
@@ -297,7 +298,7 @@ cm_status cm_shuffle_commit(const cm_shuffle *S, const void *ws, const void *Rx,
         !rows_ok(caches, ldc, r))
         return CM_EINVAL;
     const ShuffleLayout L = shuffle_layout(S->n, S->q, S->s);
-    RowProgram p{(int64_t)S->com_dst.size(), nullptr, nullptr, nullptr, at(ws, L.com_dst)};
+    RowProgram p{S->n_recv, nullptr, nullptr, nullptr, at(ws, L.com_dst)};
     return from_cuda(run<ROW_SUM, true>(p, (const float *)Rx, ldr, nullptr, 0,
                                         (float *)caches, ldc, r, (cudaStream_t)stream));
 }

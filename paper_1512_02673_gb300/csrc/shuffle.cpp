@@ -365,6 +365,9 @@ cm_status plan_transition(cm_shuffle &S)
     S.cached.swap(next);
     S.owner.swap(owner1);
     S.t = t1;
+    S.n_coded = (int64_t)S.msg_set.size();
+    S.n_recv = R;
+    S.n_sub = (int64_t)S.dec_slot.size();
     S.planned = true;
     return CM_OK;
 }
@@ -373,9 +376,9 @@ void fill_stats(const cm_shuffle &S, cm_shuffle_stats *st)
 {
     st->iteration = S.t;
     st->message_sets = S.planned ? S.message_sets : 0;
-    st->coded_rows = S.planned ? (int64_t)S.msg_set.size() : 0;
-    st->uncoded_rows = S.planned ? (int64_t)S.recv_row.size() : 0;
-    st->subtractions = S.planned ? (int64_t)S.dec_slot.size() : 0;
+    st->coded_rows = S.planned ? S.n_coded : 0;
+    st->uncoded_rows = S.planned ? S.n_recv : 0;
+    st->subtractions = S.planned ? S.n_sub : 0;
 }
 
 int64_t up64(int64_t x) { return (x + 63) & ~(int64_t)63; }
@@ -449,7 +452,7 @@ void cm_shuffle_destroy(cm_shuffle *S) { delete S; }
 
 cm_status cm_shuffle_next(cm_shuffle *S, cm_shuffle_stats *stats)
 {
-    if (!S) return CM_EINVAL;
+    if (!S || S->device_ws) return CM_EINVAL;   // device-planned instances plan on the device
     cm_status st;
     try {
         st = plan_transition(*S);
@@ -472,6 +475,7 @@ cm_status cm_shuffle_plan(const cm_shuffle *S, int32_t *msg_ptr, int32_t *msg_sr
 {
     if (!S) return CM_EINVAL;
     if (!S->planned) return CM_EINVAL;
+    if (S->device_ws) return shuffle_device_plan(S, msg_ptr, msg_src, msg_worker, msg_set);
     auto put = [](void *dst, const void *src, size_t bytes) {
         if (dst && bytes) std::memcpy(dst, src, bytes);
     };
@@ -485,6 +489,7 @@ cm_status cm_shuffle_plan(const cm_shuffle *S, int32_t *msg_ptr, int32_t *msg_sr
 cm_status cm_shuffle_received(const cm_shuffle *S, int32_t *recv_ptr, int32_t *recv_row)
 {
     if (!S || !S->planned) return CM_EINVAL;
+    if (S->device_ws) return shuffle_device_received(S, recv_ptr, recv_row);
     if (recv_ptr) std::memcpy(recv_ptr, S->recv_ptr.data(), sizeof(int32_t) * (S->n + 1));
     if (recv_row && !S->recv_row.empty())
         std::memcpy(recv_row, S->recv_row.data(), sizeof(int32_t) * S->recv_row.size());
@@ -494,6 +499,7 @@ cm_status cm_shuffle_received(const cm_shuffle *S, int32_t *recv_ptr, int32_t *r
 cm_status cm_shuffle_caches(const cm_shuffle *S, int32_t *owner, int32_t *slot_row)
 {
     if (!S) return CM_EINVAL;
+    if (S->device_ws) return shuffle_device_caches(S, owner, slot_row);
     if (owner) std::memcpy(owner, S->owner.data(), sizeof(int32_t) * S->q);
     if (slot_row) std::memcpy(slot_row, S->slot_row.data(), sizeof(int32_t) * S->slot_row.size());
     return CM_OK;

@@ -36,9 +36,23 @@ struct cm_shuffle {
     std::vector<int32_t> dec_msg, dec_ptr, dec_slot, dec_dst, com_dst;
     std::vector<int32_t> recv_ptr, recv_row;
     int64_t message_sets = 0;
+    // Sizes of the current programs: coded rows, received rows, subtracted rows
+    int64_t n_coded = 0, n_recv = 0, n_sub = 0;
     // Workspace the current programs were last copied to, and for which t.
     const void *uploaded_ws = nullptr;
     int64_t uploaded_t = -1;
+    // Device planning: once set, the partition, caches and programs live in
+    // this workspace (the host tables above are stale), and dev_cur selects
+    // the current copy of the double-buffered partition and cache masks.
+    void *device_ws = nullptr;
+    int dev_cur = 0;
 };
 
 ShuffleLayout shuffle_layout(int32_t n, int64_t q, int64_t s);
+
+// Device-mode queries (k_shuffle_plan.cu): copy the current tables out of
+// the device workspace (synchronous).
+cm_status shuffle_device_plan(const cm_shuffle *S, int32_t *msg_ptr, int32_t *msg_src,
+                              int32_t *msg_worker, uint64_t *msg_set);
+cm_status shuffle_device_received(const cm_shuffle *S, int32_t *recv_ptr, int32_t *recv_row);
+cm_status shuffle_device_caches(const cm_shuffle *S, int32_t *owner, int32_t *slot_row);

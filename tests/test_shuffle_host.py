@@ -127,3 +127,17 @@ def test_data_plane_needs_an_uploaded_plan(cm):
         lib.plan()                         # no transition planned yet
     assert L.cm_shuffle_upload(lib._h, nul, 0, nul) == cm.CM_EINVAL
     assert lib.workspace_bytes() >= 4 * (30 * (3 + 5) + 3 * 15)
+
+
+def test_device_planner_refuses_without_workspace(cm):
+    # argument checks only (no GPU): device planning needs an initialised
+    # workspace, and the dense set tables limit it to n <= 16
+    import ctypes
+    L = cm.lib()
+    nul = ctypes.c_void_p(0)
+    small = cm.Shuffle(4, 40, 20, 1, 2)
+    assert L.cm_shuffle_device_next(small._h, nul, 0, nul, nul) == cm.CM_EINVAL
+    assert L.cm_shuffle_device_init(small._h, nul, 0, nul) == cm.CM_EINVAL
+    assert small.device_workspace_bytes() >= small.workspace_bytes()
+    big = cm.Shuffle(17, 17 * 4, 8, 1, 2)
+    assert big.device_workspace_bytes() == 0

@@ -165,11 +165,18 @@ def dist_setup():
     return world, rank, local
 
 
+def _reduce_device():
+    """Tensors for collectives live where the process group's backend wants
+    them: on the GPU for NCCL, on the host for gloo."""
+    import torch.distributed as dist
+    return "cpu" if dist.get_backend() == "gloo" else "cuda"
+
+
 def max_over_ranks(x: float, world: int) -> float:
     if world == 1:
         return x
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    t = torch.tensor([x], dtype=torch.float64, device=_reduce_device())
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
 
@@ -178,6 +185,15 @@ def barrier(world: int):
     if world > 1:
         import torch.distributed as dist
         dist.barrier()
+
+
+def whole_job_value(bytes_per_step_per_rank: int, steps: int, ms_local: float,
+                    world: int) -> tuple:
+    """(value in GB/s, ms): weak scaling, every rank runs its own replica of
+    the workload; the job moves world x the bytes of one replica in the time
+    of the slowest rank."""
+    ms = max_over_ranks(ms_local, world)
+    return world * bytes_per_step_per_rank * steps / (ms * 1e-3) / 1e9, ms
 
 
 # ---- CPU oracle on a bounded sample (the baseline / reference arm) ---------------------
@@ -316,7 +332,7 @@ def run_ours(args, world, rank, local):
     ms_local = t_start.elapsed_time(t_end)
     if int(status.item()) != 0:
         raise RuntimeError("device status %d during the timed steps" % int(status.item()))
-    ms = max_over_ranks(ms_local, world)
+    value, ms = whole_job_value(nbytes["step"], args.steps, ms_local, world)
     per = {"encode": [], "matvec": [], "decode": []}
     for e in evs:
         per["encode"].append(e[0].elapsed_time(e[1]))
@@ -378,7 +394,6 @@ def run_ours(args, world, rank, local):
     achieved = nbytes["matvec"] / (avg["matvec"] * 1e-3) / 1e9
     traffic = recorded_traffic("matvec",
                                os.path.join(ROOT, "paper_1512_02673_gb300", "csrc", "k_matvec.cu"))
-    value = world * nbytes["step"] * args.steps / (ms * 1e-3) / 1e9
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,

@@ -684,6 +684,7 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     parity = cm.encode(code, A)
     torch.cuda.synchronize()
+    torch.cuda._sleep(1_000_000)   # the event times the kernel, not the host's call
     e0.record()
     cm.encode(code, A, parity)
     e1.record()

@@ -18,11 +18,13 @@
 //                 worker: the first s - q/n of each worker are kept;
 //   commit        dropped slots of each worker, ascending, take its received
 //                 rows in order.
-// Radix passes: one warp per tile of 2048 items, 8-bit digits; a tile's
+// Radix passes: one warp per tile of 1024 items, 8-bit digits; a tile's
 // histogram by shared-memory atomics, global offsets by an exclusive scan of
 // the (digit, tile) matrix, and a stable scatter that ranks equal digits
-// within each 32-item step by __match_any_sync.  Device scans: 4096 items
-// per 1024-thread block, block sums scanned recursively.
+// within each 32-item step by __match_any_sync, reorders the tile by digit in
+// shared memory and writes each digit's run to consecutive addresses.
+// Device scans: 4096 items per 1024-thread block, block sums scanned
+// recursively.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -34,8 +36,11 @@
 
 namespace {
 
-constexpr int kTile = 2048;        // items per warp in a radix pass
-constexpr int kRadixWarps = 8;     // warps (tiles) per radix block
+constexpr int kTile = 1024;        // items per warp in a radix pass
+constexpr int kRadixWarps = 4;     // warps (tiles) per radix block
+// shared memory of one warp's scatter: its tile's keys and values in digit
+// order, and three 256-entry tables (local starts, running counts, global bases)
+constexpr int kScatterWarpBytes = kTile * 12 + 3 * 256 * 4;
 constexpr int kScanBlock = 1024;
 constexpr int kScanItems = 4 * kScanBlock;
 constexpr int kMaxDeviceN = 16;    // dense tables over all 2^n worker sets
@@ -158,39 +163,100 @@ __global__ void radix_hist_kernel(const uint64_t *keys, const int32_t *countp, i
     if (tile >= tiles) return;
     const int64_t count = countp ? (int64_t)*countp : cap;
     const int64_t beg = tile * kTile, end = std::min(count, beg + kTile);
+#pragma unroll 8
     for (int64_t i = beg + lane; i < end; i += 32) atomicAdd(&cnt[warp][(keys[i] >> shift) & 255], 1);
     __syncwarp();
     for (int d = lane; d < 256; d += 32) hist[(int64_t)d * tiles + tile] = cnt[warp][d];
 }
 
-__global__ void radix_scatter_kernel(const uint64_t *kin, const int32_t *vin, uint64_t *kout,
-                                     int32_t *vout, const int32_t *countp, int64_t cap, int shift,
-                                     const int32_t *offsets, int64_t tiles)
+// One warp per tile of 32 x 32 items: (1) the tile loaded into registers
+// (lane l holds items l, 32 + l, ...; all loads in flight together), its digit
+// counts and their exclusive scan (local starts); (2) every item placed,
+// stably, at its digit's local start plus its rank in shared memory (equal
+// digits of a 32-item step ranked by lane with __match_any_sync); (3) the
+// tile written out in that digit order: a run of equal digits goes to
+// consecutive global positions, so the writes coalesce.
+__global__ void __launch_bounds__(32 * kRadixWarps)
+radix_scatter_kernel(const uint64_t *kin, const int32_t *vin, uint64_t *kout, int32_t *vout,
+                     const int32_t *countp, int64_t cap, int shift, const int32_t *offsets,
+                     int64_t tiles)
 {
-    __shared__ int32_t base[kRadixWarps][256];
+    static_assert(kTile == 32 * 32, "a tile is 32 steps of 32 items");
+    extern __shared__ __align__(16) unsigned char smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    unsigned char *mine = smem + warp * kScatterWarpBytes;
+    uint64_t *sk = reinterpret_cast<uint64_t *>(mine);
+    int32_t *sv = reinterpret_cast<int32_t *>(mine + kTile * 8);
+    int32_t *start = reinterpret_cast<int32_t *>(mine + kTile * 12);
+    int32_t *run = start + 256;
+    int32_t *base = run + 256;
     const int64_t tile = (int64_t)blockIdx.x * kRadixWarps + warp;
     if (tile >= tiles) return;
-    for (int d = lane; d < 256; d += 32) base[warp][d] = offsets[(int64_t)d * tiles + tile];
-    __syncwarp();
     const int64_t count = countp ? (int64_t)*countp : cap;
     const int64_t beg = tile * kTile, end = std::min(count, beg + kTile);
+    const int nt = end > beg ? (int)(end - beg) : 0;
+    for (int d = lane; d < 256; d += 32) {
+        run[d] = 0;
+        base[d] = offsets[(int64_t)d * tiles + tile];
+    }
+    uint64_t k[32];
+    int32_t v[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+        const int p = 32 * j + lane;
+        k[j] = p < nt ? kin[beg + p] : 0;
+        v[j] = p < nt ? vin[beg + p] : 0;
+    }
+    __syncwarp();
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+        if (32 * j + lane < nt) atomicAdd(&run[(k[j] >> shift) & 255], 1);
+    __syncwarp();
+    {   // exclusive scan of the 256 counts: 8 per lane
+        int32_t c[8], sum = 0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            c[q] = run[8 * lane + q];
+            sum += c[q];
+        }
+        int32_t x = sum;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        int32_t at = x - sum;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            start[8 * lane + q] = at;
+            at += c[q];
+        }
+    }
+    __syncwarp();
+    for (int d = lane; d < 256; d += 32) run[d] = 0;
+    __syncwarp();
     const unsigned below = (1u << lane) - 1u;
-    for (int64_t i0 = beg; i0 < end; i0 += 32) {
-        const int64_t i = i0 + lane;
-        const bool valid = i < end;
-        const uint64_t k = valid ? kin[i] : 0;
-        const int32_t v = valid ? vin[i] : 0;
-        const int d = valid ? (int)((k >> shift) & 255) : 256;   // 256: not an item
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+        if (32 * j >= nt) break;   // warp-uniform
+        const bool valid = 32 * j + lane < nt;
+        const int d = valid ? (int)((k[j] >> shift) & 255) : 256;   // 256: not an item
         const unsigned peers = __match_any_sync(0xffffffffu, d);
         if (valid) {
-            const int pos = base[warp][d] + __popc(peers & below);
-            kout[pos] = k;
-            vout[pos] = v;
+            const int pos = start[d] + run[d] + __popc(peers & below);
+            sk[pos] = k[j];
+            sv[pos] = v[j];
         }
         __syncwarp();
-        if (valid && (peers & below) == 0) base[warp][d] += __popc(peers);
+        if (valid && (peers & below) == 0) run[d] += __popc(peers);
         __syncwarp();
+    }
+    for (int p = lane; p < nt; p += 32) {
+        const uint64_t kk = sk[p];
+        const int d = (int)((kk >> shift) & 255);
+        const int g = base[d] + (p - start[d]);
+        kout[g] = kk;
+        vout[g] = sv[p];
     }
 }
 
@@ -210,12 +276,16 @@ cudaError_t radix_sort(const SortBufs &b, const int32_t *countp, int64_t cap, in
     const unsigned blocks = (unsigned)((tiles + kRadixWarps - 1) / kRadixWarps);
     uint64_t *ki = b.kA, *ko = b.kB;
     int32_t *vi = b.vA, *vo = b.vB;
+    cudaError_t ea = cudaFuncSetAttribute(radix_scatter_kernel,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          kRadixWarps * kScatterWarpBytes);
+    if (ea != cudaSuccess) return ea;
     for (int shift = lo; shift < hi; shift += 8) {
         radix_hist_kernel<<<blocks, 32 * kRadixWarps, 0, s>>>(ki, countp, cap, shift, b.hist, tiles);
         cudaError_t e = scan_exclusive(b.hist, b.hist, 256 * tiles, b.scan, nullptr, s);
         if (e != cudaSuccess) return e;
-        radix_scatter_kernel<<<blocks, 32 * kRadixWarps, 0, s>>>(ki, vi, ko, vo, countp, cap, shift,
-                                                                 b.hist, tiles);
+        radix_scatter_kernel<<<blocks, 32 * kRadixWarps, kRadixWarps * kScatterWarpBytes, s>>>(
+            ki, vi, ko, vo, countp, cap, shift, b.hist, tiles);
         std::swap(ki, ko);
         std::swap(vi, vo);
     }

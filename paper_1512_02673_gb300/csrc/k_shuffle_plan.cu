@@ -314,15 +314,22 @@ __global__ void owner_kernel(const int32_t *order, int64_t q, int64_t per, int32
 // Per row: missing from its new owner's cache?  Its set I, its candidate
 // bits for the cache refill; counts per (I, worker), per worker and per
 // candidate worker.  Counters of n bins are aggregated in shared memory.
+// Per row: missing from its new owner's cache?  Its set I, its candidate
+// bits for the cache refill; counts per (I, worker), per worker and per
+// candidate worker.  The per-worker counters are aggregated in shared memory
+// per block, and so are the (I, worker) counters when their table fits
+// (`local` = 2^n n entries, else 0: global atomics).
 __global__ void need_kernel(int64_t q, int n, const int32_t *owner1, const uint64_t *cached0,
                             uint64_t *rmask, int32_t *needflag, int32_t *ccnt_row, uint64_t *next,
-                            int32_t *counts, int32_t *wcount, int32_t *ccount)
+                            int32_t *counts, int32_t *wcount, int32_t *ccount, int local)
 {
+    extern __shared__ int32_t sl[];
     __shared__ int32_t sw[kMaxDeviceN], sc[kMaxDeviceN];
     if (threadIdx.x < kMaxDeviceN) {
         sw[threadIdx.x] = 0;
         sc[threadIdx.x] = 0;
     }
+    for (int i = threadIdx.x; i < local; i += blockDim.x) sl[i] = 0;
     __syncthreads();
     GS_LOOP(r, q)
     {
@@ -335,7 +342,9 @@ __global__ void need_kernel(int64_t q, int n, const int32_t *owner1, const uint6
         next[r] = bit;
         ccnt_row[r] = __popcll(cand);
         if (nf) {
-            atomicAdd(&counts[(int64_t)(have | bit) * n + i], 1);
+            const int64_t slot = (int64_t)(have | bit) * n + i;
+            if (local) atomicAdd(&sl[slot], 1);
+            else atomicAdd(&counts[slot], 1);
             atomicAdd(&sw[i], 1);
         }
         for (uint64_t b = cand; b; b &= b - 1) atomicAdd(&sc[__ffsll((long long)b) - 1], 1);
@@ -345,6 +354,8 @@ __global__ void need_kernel(int64_t q, int n, const int32_t *owner1, const uint6
         atomicAdd(&wcount[threadIdx.x], sw[threadIdx.x]);
         atomicAdd(&ccount[threadIdx.x], sc[threadIdx.x]);
     }
+    for (int i = threadIdx.x; i < local; i += blockDim.x)
+        if (sl[i]) atomicAdd(&counts[i], sl[i]);
 }
 
 __global__ void compact_kernel(int64_t q, const int32_t *flag, const int32_t *idx, int32_t *items)
@@ -689,8 +700,9 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     uint64_t *rmask = ptr<uint64_t>(ws, D.rmask);
     int32_t *needflag = ptr<int32_t>(ws, D.needflag), *idx = ptr<int32_t>(ws, D.idx);
     int32_t *ccnt_row = ptr<int32_t>(ws, D.ccnt_row), *cbase = ptr<int32_t>(ws, D.cbase);
-    need_kernel<<<grid_for(q), 256, 0, s>>>(q, n, owner1, cached0, rmask, needflag, ccnt_row,
-                                            next, counts, wcount, ccount);
+    const int local = nm * n <= 8192 ? (int)(nm * n) : 0;   // 32 KB of shared counters
+    need_kernel<<<grid_for(q), 256, sizeof(int32_t) * local, s>>>(
+        q, n, owner1, cached0, rmask, needflag, ccnt_row, next, counts, wcount, ccount, local);
     LAUNCHED();
     CK(scan_exclusive(needflag, idx, q, scan, totals + T_R, s));
     int32_t *items = ptr<int32_t>(ws, D.items);

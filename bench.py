@@ -225,7 +225,26 @@ def cpu_baseline(w: synth.Workload, target_s: float = 12.0) -> dict:
     return {"value": nb / dt / 1e9, "unit": "GB/s", "cores": oracle.num_threads(),
             "kind": "oracle",
             "sample": "%d of %d block rows of every worker (%.1f%% of the step), one step, "
-                      "%.1f s" % (s, w.L, 100.0 * s / w.L, dt)}
+                      "%.1f s" % (s, w.L, 100.0 * s / w.L, dt),
+            "small_configs": oracle_small_configs()}
+
+
+def oracle_small_configs() -> dict:
+    """The oracle's full step (encode, all worker products, decode) on the
+    tiny and the (10,5) mat-vec configurations, on every host thread and on
+    one, in ms."""
+    import oracle
+    threads = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    out = {"threads": threads}
+    for w in (synth.TINY, synth.MATVEC):
+        r = {}
+        for label, t in (("all_threads_ms", threads), ("one_thread_ms", 1)):
+            oracle.set_threads(t)
+            dt, _ = oracle_sample_step(w, w.L, 80, 0)
+            r[label] = 1e3 * dt
+        out[w.name] = r
+    oracle.set_threads(threads)
+    return out
 
 
 def run_reference(args, world, rank):

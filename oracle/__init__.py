@@ -56,6 +56,7 @@ def _load():
         vp = ctypes.c_void_p
         sig = {
             "or_num_threads": (ctypes.c_int, []),
+            "or_set_threads": (None, [ctypes.c_int]),
             "or_block_rows": (i64, [i64, i32]),
             "or_encode": (ctypes.c_int, [i32, i32, i64, i64, vp, vp, i64, vp, vp]),
             "or_encode_bf16": (ctypes.c_int, [i32, i32, i64, i64, vp, vp, i64, vp, vp]),
@@ -109,6 +110,11 @@ def _check(status: int):
 
 def num_threads() -> int:
     return int(_load().or_num_threads())
+
+
+def set_threads(threads: int) -> None:
+    """Threads of the OpenMP loops (timing only)."""
+    _load().or_set_threads(threads)
 
 
 def block_rows(m: int, k: int) -> int:

@@ -38,6 +38,17 @@ int or_num_threads(void)
 #endif
 }
 
+/* Threads for the parallel loops that follow (timing only; no arithmetic
+ * depends on it: every loop splits independent outputs). */
+void or_set_threads(int threads)
+{
+#ifdef _OPENMP
+    if (threads > 0) omp_set_num_threads(threads);
+#else
+    (void)threads;
+#endif
+}
+
 /* Sec. III-A, footnote on zero padding: when m is not a multiple of k, zero
  * rows are appended so that A splits into k equal blocks of L = ceil(m/k). */
 int64_t or_block_rows(int64_t m, int32_t k)

@@ -74,6 +74,9 @@ def gd_iter_bytes(w: synth.GDWorkload, LA: int, LAT: int) -> int:
 
 # ---- helpers -----------------------------------------------------------------------------
 
+NOMINAL_HBM_GBS = 7900.0   # GB300 HBM3e, nominal
+
+
 def measured_peaks() -> dict:
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -688,6 +691,7 @@ def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
             "roofline": {"bound": "tensor", "kernel": "coded GEMM (tcgen05, bf16 -> fp32)",
                          "achieved": tflops, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                          "frac": tflops / peaks["bf16_tflops"],
+                         "frac_of_sustained": tflops / peaks["bf16_tflops_sustained"],
                          "peak_source": peaks["source"] + " bf16 burst"},
             "decode_mat_ms": d_ms, "decode_mat_gbs": dec_bytes / (d_ms * 1e-3) / 1e9,
             "encode_bf16_ms": enc_ms, "status": int(status.item())}
@@ -736,7 +740,11 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
     mv = np.array([e[0].elapsed_time(e[1]) * 1e3 for e in ev])
     dec = np.array([e[1].elapsed_time(e[2]) * 1e3 for e in ev])
     nb = step_bytes(w, code.L)
+    peaks = measured_peaks()
+    mv_gbs = nb["matvec"] / (np.median(mv) * 1e-6) / 1e9
     return {"workload": w.name, "repeats": reps, "l2_flushed": flush is not None,
+            "matvec_pct_of_measured_hbm": 100.0 * mv_gbs / peaks["hbm_gbs"],
+            "matvec_pct_of_nominal_hbm": 100.0 * mv_gbs / NOMINAL_HBM_GBS,
             "encode_us": enc_us,
             "encode_gbs": nb["encode"] / (enc_us * 1e-6) / 1e9,
             "matvec_us_median": float(np.median(mv)), "matvec_us_p95": float(np.percentile(mv, 95)),

@@ -482,7 +482,7 @@ __global__ void decslot_kernel(const int32_t *Rp, int64_t q, int64_t s, const in
 
 __global__ void cand_kernel(int64_t q, int n, int64_t t1, uint64_t seed, const int32_t *owner1,
                             const uint64_t *cached0, const int32_t *cbase, int32_t *cw,
-                            int32_t *cr, uint64_t *keys, int32_t *vals)
+                            int32_t *cr, uint64_t *ckey, uint64_t *keys, int32_t *vals)
 {
     GS_LOOP(r, q)
     {
@@ -494,6 +494,7 @@ __global__ void cand_kernel(int64_t q, int n, int64_t t1, uint64_t seed, const i
             cr[c] = (int32_t)r;
             keys[c] = mix64(seed, ((uint64_t)t1 * (uint64_t)n + (uint64_t)i) * (uint64_t)q +
                                       (uint64_t)r);
+            ckey[c] = keys[c];
             vals[c] = c;
         }
     }
@@ -504,6 +505,52 @@ __global__ void cand_worker_keys_kernel(const int32_t *Kp, const int32_t *vals, 
 {
     const int64_t K = *Kp;
     GS_LOOP(p, K) keys[p] = (uint64_t)cw[vals[p]];
+}
+
+// After a stable sort on the top 24 bits of the keys only, items whose top
+// bits tie are adjacent and in their original order; each such run (short:
+// keys are uniform 64-bit values) is put in full (key, row) order by the
+// thread at its start.  `grp` (nullable) adds a group that must also tie
+// (the worker of a candidate); keys and rows are read through the values
+// (`key_of`, `row_of`: item id -> key / row; null: the sorted key array and
+// the value itself).
+__global__ void fixup_runs_kernel(const int32_t *countp, int64_t cap, const uint64_t *skeys,
+                                  int32_t *vals, const uint64_t *key_of, const int32_t *row_of,
+                                  const int32_t *grp)
+{
+    const int64_t count = countp ? (int64_t)*countp : cap;
+    auto key = [&](int32_t v, int64_t p) { return key_of ? key_of[v] : skeys[p]; };
+    auto row = [&](int32_t v) { return row_of ? row_of[v] : v; };
+    auto top = [&](int32_t v, int64_t p) {
+        return ((key(v, p) >> 40) << 8) | (uint64_t)(grp ? grp[v] : 0);
+    };
+    GS_LOOP(p, count)
+    {
+        const int32_t v0 = vals[p];
+        const uint64_t t0 = top(v0, p);
+        if (p > 0 && top(vals[p - 1], p - 1) == t0) continue;   // not a run start
+        int64_t e = p + 1;
+        while (e < count && top(vals[e], e) == t0) ++e;
+        if (e - p < 2) continue;
+        // insertion sort of vals[p, e) by (key, row); with key_of null the
+        // keys move with the values
+        for (int64_t i = p + 1; i < e; ++i) {
+            const int32_t vi = vals[i];
+            const uint64_t ki = key_of ? key_of[vi] : skeys[i];
+            const int32_t ri = row(vi);
+            int64_t j = i - 1;
+            while (j >= p) {
+                const int32_t vj = vals[j];
+                const uint64_t kj = key_of ? key_of[vj] : skeys[j];
+                if (kj < ki || (kj == ki && row(vj) < ri)) break;
+                vals[j + 1] = vj;
+                if (!key_of) const_cast<uint64_t *>(skeys)[j + 1] = kj;
+                --j;
+            }
+            vals[j + 1] = vi;
+            if (!key_of) const_cast<uint64_t *>(skeys)[j + 1] = ki;
+        }
+    }
 }
 
 __global__ void kept_kernel(const int32_t *Kp, int64_t keep, const int32_t *vals,
@@ -570,7 +617,7 @@ struct DevLayout {
     int64_t kA, kB, vA, vB, hist, scan;
     int64_t rmask, needflag, idx, items, recv_row, wcount, recv_ptr;
     int64_t counts, runstart, ell, msgbase, earr, msg_set, msg_worker, dx;
-    int64_t ccnt_row, cbase, cw, cr, ccount, cstart, evflag, evrank, totals;
+    int64_t ccnt_row, cbase, cw, cr, ckey, ccount, cstart, evflag, evrank, totals;
     int64_t bytes;            // total
     int64_t capK, nm;
 };
@@ -620,6 +667,7 @@ DevLayout device_layout(int32_t n, int64_t q, int64_t s)
     D.cbase = take(4 * (q + 1));
     D.cw = take(4 * D.capK);
     D.cr = take(4 * D.capK);
+    D.ckey = take(8 * D.capK);
     D.ccount = take(4 * (n + 1));
     D.cstart = take(4 * (n + 1));
     D.evflag = take(4 * (ns + 1));
@@ -692,7 +740,9 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     LAUNCHED();
     uint64_t *ko;
     int32_t *vo;
-    CK(radix_sort(sb, nullptr, q, 0, 64, s, &ko, &vo));
+    CK(radix_sort(sb, nullptr, q, 40, 64, s, &ko, &vo));   // top 24 bits, then the ties
+    fixup_runs_kernel<<<grid_for(q), 256, 0, s>>>(nullptr, q, ko, vo, nullptr, nullptr, nullptr);
+    LAUNCHED();
     owner_kernel<<<grid_for(q), 256, 0, s>>>(vo, q, S->per, owner1);
     LAUNCHED();
 
@@ -754,14 +804,26 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     // cache update rule: candidates by (worker, key, row); the first s - q/n kept
     CK(scan_exclusive(ccnt_row, cbase, q, scan, totals + T_K, s));
     int32_t *cw = ptr<int32_t>(ws, D.cw), *cr = ptr<int32_t>(ws, D.cr);
+    uint64_t *ckey = ptr<uint64_t>(ws, D.ckey);
     cand_kernel<<<grid_for(q), 256, 0, s>>>(q, n, t1, S->cache_seed, owner1, cached0, cbase, cw,
-                                            cr, sb.kA, sb.vA);
+                                            cr, ckey, sb.kA, sb.vA);
     LAUNCHED();
-    CK(radix_sort(sb, totals + T_K, D.capK, 0, 64, s, &ko, &vo));
-    // the sorted pairs are in A again (8 passes): re-key them by worker
-    cand_worker_keys_kernel<<<grid_for(D.capK), 256, 0, s>>>(totals + T_K, vo, cw, ko);
-    LAUNCHED();
+    // by the top 24 bits of the key, then by worker (both stable), then each
+    // run of equal (worker, top bits) in full (key, row) order
+    CK(radix_sort(sb, totals + T_K, D.capK, 40, 64, s, &ko, &vo));
+    {
+        // the sort leaves its result in A or B: move it to A for the next one
+        if (vo != sb.vA) {
+            copy_i32_counted<<<grid_for(D.capK), 256, 0, s>>>(totals + T_K, vo, sb.vA);
+            LAUNCHED();
+        }
+        cand_worker_keys_kernel<<<grid_for(D.capK), 256, 0, s>>>(totals + T_K, sb.vA, cw, sb.kA);
+        LAUNCHED();
+    }
     CK(radix_sort(sb, totals + T_K, D.capK, 0, 8, s, &ko, &vo));
+    fixup_runs_kernel<<<grid_for(D.capK), 256, 0, s>>>(totals + T_K, D.capK, ko, vo, ckey, cr,
+                                                        cw);
+    LAUNCHED();
     int32_t *cstart = ptr<int32_t>(ws, D.cstart);
     CK(scan_exclusive(ccount, cstart, n + 1, scan, totals + T_DUMMY, s));
     kept_kernel<<<grid_for(D.capK), 256, 0, s>>>(totals + T_K, sz - S->per, vo, cw, cr, cstart,

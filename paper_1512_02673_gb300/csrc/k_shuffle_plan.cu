@@ -8,14 +8,16 @@
 // The definitions are the host planner's (see its header comment); the
 // device version reaches the same order through stable sorts:
 //   partition     rows sorted by (key, row): a stable LSD radix sort of the
-//                 64-bit keys over rows in ascending order;
+//                 rows (ascending) on the top 24 bits of their 64-bit keys,
+//                 then each run of equal top bits sorted by (key, row);
 //   received      missing rows in (worker, row) order: a stable sort by
 //                 worker of the rows in ascending order;
 //   messages      received rows stably sorted by the set I (bit mask), i.e.
 //                 (I, worker, row); row j of a worker's run in I goes to
 //                 message row base(I) + j, entries ordered by worker;
-//   cache update  candidates (worker, row) stably sorted by key, then by
-//                 worker: the first s - q/n of each worker are kept;
+//   cache update  candidates (worker, row) stably sorted on the top key bits,
+//                 then by worker, runs of equal (worker, top bits) by
+//                 (key, row): the first s - q/n of each worker are kept;
 //   commit        dropped slots of each worker, ascending, take its received
 //                 rows in order.
 // Radix passes: one warp per tile of 1024 items, 8-bit digits; a tile's
@@ -708,7 +710,7 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     const int cur = S->dev_cur, nxt = cur ^ 1;
     const int64_t t1 = S->t + 1;
     const int64_t nm = D.nm;
-    int32_t *owner0 = ptr<int32_t>(ws, D.owner[cur]), *owner1 = ptr<int32_t>(ws, D.owner[nxt]);
+    int32_t *owner1 = ptr<int32_t>(ws, D.owner[nxt]);
     uint64_t *cached0 = ptr<uint64_t>(ws, D.cached[cur]), *next = ptr<uint64_t>(ws, D.cached[nxt]);
     int32_t *slot_of = ptr<int32_t>(ws, D.slot_of);
     int32_t *slot_row = prog(ws, D.prog.fill_row);
@@ -719,7 +721,6 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     int32_t *counts = ptr<int32_t>(ws, D.counts), *wcount = ptr<int32_t>(ws, D.wcount);
     int32_t *ccount = ptr<int32_t>(ws, D.ccount), *ell = ptr<int32_t>(ws, D.ell);
     int32_t *dx = ptr<int32_t>(ws, D.dx);
-    (void)owner0;
     cudaError_t e;
 #define CK(x)                                      \
     do {                                           \

@@ -140,11 +140,13 @@ cm_status cm_draw_erasures(uint64_t seed, uint64_t counter, int32_t n, int32_t k
 /* Decoding (Sec. III-A last paragraph; Example "MDS codes").  S = the first
  * k set bits of `survivors` (ascending; extra survivors are ignored, which
  * favours the systematic workers).  The surviving results satisfy
- * Yt_S = G_S Z with Z the uncoded block products; the kernel inverts G_S in
- * fp64 (the k-e unit rows of surviving systematic workers are eliminated
- * first, then Gauss-Jordan with partial pivoting on the e x e block of the
- * missing systematic columns), forms the rows of G_S^-1 for the e missing
- * systematic blocks and applies them to the k surviving results in fp64;
+ * Yt_S = G_S Z with Z the uncoded block products.  The library inverts G_S
+ * on the host in fp64 when the call is made (the master knows the
+ * survivors; the k-e unit rows of surviving systematic workers are
+ * eliminated first, then Gauss-Jordan with partial pivoting on the e x e
+ * block of the missing systematic columns), forms the rows of G_S^-1 for the
+ * e missing systematic blocks, and the kernel applies them to the k surviving
+ * results (double-float arithmetic, about 2^-44 relative per term);
  * surviving systematic blocks pass through.  Y (m x b fp32) is the
  * concatenation of the k decoded blocks without the appended zero rows.
  * Returns CM_ENOTDECODABLE when fewer than k bits are set; a singular G_S

@@ -11,11 +11,14 @@
 // the rows of G_S^-1 for the missing blocks are
 //   coefficient of Yt_s, s in Ps  :  Q^-1[c][pos of s in Ps]
 //   coefficient of Yt_s, s in Ks  : -sum_a Q^-1[c][a] P[Ps[a]][s]
-// Every CTA forms these coefficients itself in shared memory (one warp, fp64),
-// then the CTA's threads apply them: missing block M[c] row r is the
-// combination of the k surviving rows r, surviving systematic blocks pass
-// through.  A zero (or relatively negligible) pivot marks G_S singular: the
-// kernel writes CM_ESINGULAR to the status word and writes no output.
+// The master knows the survivors when it decodes, so the library's host code
+// forms these coefficients once per call (plan_decode, fp64, a few
+// microseconds; formed on the device they cost every CTA ~10 us of
+// latency-bound fp64 work) and passes them to the kernel by value; the
+// kernel's threads apply them: missing block M[c] row r is the combination of
+// the k surviving rows r, surviving systematic blocks pass through.  A zero
+// (or relatively negligible) pivot marks G_S singular: the kernel writes
+// CM_ESINGULAR to the status word and writes no decoded block.
 //
 // fp64 arithmetic runs at about 1/58 of the fp32 rate on this part, so the
 // vector decode applies the fp64 coefficients in double-float arithmetic on
@@ -24,7 +27,10 @@
 // instruction), products are formed exactly with an FMA and the sums are kept
 // as (sum, compensation) pairs (Knuth's TwoSum), about 2^-44 relative per
 // term, far below the rounding of the fp32 output.
+#include <algorithm>
 #include <cfloat>
+#include <cmath>
+#include <cstring>
 
 #include "cm_internal.cuh"
 
@@ -33,167 +39,17 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kMaxE = 16;   // e <= min(k, n - k) <= 16 for n <= 32
 
-struct DecodeShared {
-    int S[CM_MAX_N];       // survivors in ascending order (k of them)
-    int role[CM_MAX_N];    // block i < k: -1 passes through, else its row c in M
-    int M[kMaxE];          // missing systematic blocks, ascending
-    int Ps[kMaxE];         // surviving parity workers, ascending
-    int e;
-    int singular;
-    double W[kMaxE][2 * kMaxE];   // [Q | I] during elimination
-    double Qi[kMaxE][kMaxE];      // Q^-1
-    double D[kMaxE][CM_MAX_N];    // decode rows: D[c][p], p = position in S
-    float Dh[kMaxE][CM_MAX_N];    // D as (high, low) fp32 pairs
-    float Dl[kMaxE][CM_MAX_N];
+// The decode of one survivor mask, formed on the host (plan_decode below) and
+// passed to the kernels by value: the survivors used, the missing systematic
+// blocks, and the rows of G_S^-1 for those blocks as (high, low) fp32 pairs.
+struct DecodePlan {
+    int32_t e;               // missing systematic blocks
+    int32_t singular;        // G_S judged singular: decode nothing
+    int32_t S[CM_MAX_N];     // survivors in ascending order (k of them)
+    int32_t M[kMaxE];        // missing systematic blocks, ascending
+    float Dh[kMaxE][CM_MAX_N];   // D[c][p] (p = position in S), rounded to fp32
+    float Dl[kMaxE][CM_MAX_N];   // D - Dh, rounded to fp32
 };
-
-// Warp 0: the survivor lists (S, role, M, Ps, e) from the mask, by ballots.
-__device__ void decode_select(const CodeParams &cp, uint32_t survivors, DecodeShared &sh)
-{
-    const int lane = threadIdx.x & 31;
-    const int n = cp.n, k = cp.k;
-    const uint32_t below = (1u << lane) - 1u;
-    // the first k set bits of the mask are the survivors used
-    const bool set = lane < n && ((survivors >> lane) & 1u);
-    const bool sel = set && __popc(survivors & below) < k;
-    const uint32_t selm = __ballot_sync(0xffffffffu, sel);
-    const bool miss = lane < k && !sel;
-    const uint32_t missm = __ballot_sync(0xffffffffu, miss);
-    const bool par = sel && lane >= k;
-    const uint32_t parm = __ballot_sync(0xffffffffu, par);
-    if (sel) sh.S[__popc(selm & below)] = lane;
-    if (par) sh.Ps[__popc(parm & below)] = lane;
-    if (miss) sh.M[__popc(missm & below)] = lane;
-    if (lane < k) sh.role[lane] = miss ? __popc(missm & below) : -1;
-    if (lane == 0) {
-        sh.e = __popc(missm);
-        sh.singular = 0;
-    }
-}
-
-// Warp 0: rows of G_S^-1 for the missing blocks (D, and D as fp32 pairs).
-// fp64 instructions have long latency on this part (about 64 cycles for a
-// multiply or FMA, about 440 for a reciprocal), so the elimination is
-// fraction-free: a non-pivot row becomes piv * W[a] - W[a][col] * W[col]
-// (separate products, so duplicated rows cancel to exactly zero), with one
-// reciprocal per row at the end; partial pivoting is unaffected because all
-// non-pivot rows are scaled alike.  G_S counts as singular when a pivot is
-// zero or not finite, or when ||Q||_inf ||Q^-1||_inf exceeds 1 / (64 eps).
-__device__ void decode_coefficients(const CodeParams &cp, DecodeShared &sh)
-{
-    const int lane = threadIdx.x & 31;
-    const int k = cp.k, e = sh.e;
-    if (e == 0) return;
-    const int mc = lane < e ? sh.M[lane] : 0;
-    // W = [Q | I], Q[a][c] = P[Ps[a] - k][M[c]]; lane owns column `lane`.
-    double qnorm = 0.0;   // row sums of |Q| (lane a < e holds row a)
-    for (int a = 0; a < e; ++a) {
-        const int ps = sh.Ps[a];
-        double w = 0.0;
-        if (lane < e) w = (double)cp.P[(ps - k) * k + mc];
-        else if (lane < 2 * e) w = (lane - e == a) ? 1.0 : 0.0;
-        if (lane < 2 * e) sh.W[a][lane] = w;
-    }
-    __syncwarp();
-    if (lane < e)
-        for (int c = 0; c < e; ++c) qnorm += fabs(sh.W[lane][c]);
-    for (int off = 16; off; off >>= 1) qnorm = fmax(qnorm, __shfl_xor_sync(0xffffffffu, qnorm, off));
-    int singular = 0;
-    for (int col = 0; col < e; ++col) {
-        // partial pivoting on the fp32 image of |W[a][col]| (a >= col), lowest
-        // index on ties; any near-largest pivot is as good numerically
-        const double wl = lane >= col && lane < e ? sh.W[lane][col] : 0.0;
-        float best = lane >= col && lane < e ? (float)fabs(wl) : -1.f;
-        int bi = lane;
-        for (int off = 16; off; off >>= 1) {
-            const float ob = __shfl_xor_sync(0xffffffffu, best, off);
-            const int oi = __shfl_xor_sync(0xffffffffu, bi, off);
-            if (ob > best || (ob == best && oi < bi)) {
-                best = ob;
-                bi = oi;
-            }
-        }
-        const double bval = __shfl_sync(0xffffffffu, wl, bi);
-        if (!(fabs(bval) > 0.0) || !isfinite(bval)) {
-            singular = 1;
-            break;
-        }
-        if (bi != col && lane < 2 * e) {
-            const double t = sh.W[col][lane];
-            sh.W[col][lane] = sh.W[bi][lane];
-            sh.W[bi][lane] = t;
-        }
-        __syncwarp();
-        if (lane < 2 * e) {
-            // lane owns column `lane`; column `col` of the non-pivot rows becomes 0
-            const double piv = bval;
-            const double wc = sh.W[col][lane];
-            for (int a = 0; a < e; ++a) {
-                if (a == col) continue;
-                const double fa = sh.W[a][col];      // read before anyone writes it
-                const double wa = sh.W[a][lane];
-                __syncwarp(__activemask());
-                sh.W[a][lane] = lane == col ? 0.0 : piv * wa - fa * wc;
-            }
-        }
-        __syncwarp();
-    }
-    if (!singular) {
-        // Q^-1[c][a] = W[c][e + a] / W[c][c]
-        const double dinv = lane < e ? 1.0 / sh.W[lane][lane] : 0.0;
-        double qimax = 0.0;
-        for (int t = lane; t < 32 * ((e * e + 31) / 32); t += 32) {
-            const int c = t / e, aa = t % e;
-            const double dc = __shfl_sync(0xffffffffu, dinv, t < e * e ? c : 0);
-            if (t < e * e) {
-                const double q = sh.W[c][e + aa] * dc;
-                sh.Qi[c][aa] = q;
-                qimax = fmax(qimax, fabs(q));
-            }
-        }
-        for (int off = 16; off; off >>= 1)
-            qimax = fmax(qimax, __shfl_xor_sync(0xffffffffu, qimax, off));
-        // ||Q^-1||_inf <= e max|Q^-1|
-        if (!(qnorm * qimax * e < 1.0 / (64.0 * DBL_EPSILON))) singular = 1;
-    }
-    if (singular) {
-        if (lane == 0) sh.singular = 1;
-        __syncwarp();
-        return;
-    }
-    __syncwarp();
-    // D[c][p] (p = position in S): independent e-term chains, two per lane
-    auto d_entry = [&](int t, double &v) {
-        const int c = t / k, p = t % k;
-        const int s = sh.S[p];
-        if (s >= k) {
-            int aa = 0;
-            while (sh.Ps[aa] != s) ++aa;
-            v = sh.Qi[c][aa];
-            return;
-        }
-        v = 0.0;
-        for (int aa = 0; aa < e; ++aa)
-            v = fma(-sh.Qi[c][aa], (double)cp.P[(sh.Ps[aa] - k) * k + s], v);
-    };
-    for (int t = lane; t < e * k; t += 64) {
-        double v0 = 0.0, v1 = 0.0;
-        const int t1 = t + 32;
-        d_entry(t, v0);
-        if (t1 < e * k) d_entry(t1, v1);
-        for (int q = 0; q < 2; ++q) {
-            const int tt = q ? t1 : t;
-            if (tt >= e * k) break;
-            const double v = q ? v1 : v0;
-            const int c = tt / k, p = tt % k;
-            sh.D[c][p] = v;
-            const float h = __double2float_rn(v);
-            sh.Dh[c][p] = h;
-            sh.Dl[c][p] = __double2float_rn(v - (double)h);
-        }
-    }
-    __syncwarp();
-}
 
 // ---- double-float helpers (fp32 pipe only) -------------------------------------------
 
@@ -237,8 +93,8 @@ __device__ __forceinline__ void df_fma(float dh, float dl, float yh, float yl, f
 
 struct DecodeArgs {
     CodeParams cp;
+    DecodePlan plan;
     const double *Yt;
-    uint32_t survivors;
     int b;
     float *Y;
     int32_t *status;
@@ -260,25 +116,24 @@ __device__ __forceinline__ void store_out(const DecodeArgs &a, int64_t out, floa
     }
 }
 
-__global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a)
+// The plan stays in the parameter space: every access below is uniform
+// across a warp (one (c, p) at a time; S and M indexed by a block number that
+// changes only at block boundaries), which the constant cache serves by
+// broadcast; copying it to shared memory would read it divergently.
+__global__ void __launch_bounds__(kThreads) decode_kernel(const __grid_constant__ DecodeArgs a)
 {
-    __shared__ DecodeShared sh;
-    const int warp = threadIdx.x >> 5;
-    if (warp == 0) decode_select(a.cp, a.survivors, sh);
-    __syncthreads();
+    const DecodePlan &sh = a.plan;
     const int k = a.cp.k, e = sh.e;
     const int64_t L = a.cp.L, m = a.cp.m;
     const int b = a.b;
     const int64_t per_block = L * b;
-    if (warp == 0) {
-        decode_coefficients(a.cp, sh);
-    } else {
-        // meanwhile the other warps pass the surviving systematic blocks
-        // through (exactly rounded to fp32), four independent loads at a time
+    {
+        // the surviving systematic blocks pass through (exactly rounded to
+        // fp32), four independent loads at a time
         const int64_t npass = (int64_t)(k - e) * per_block;
-        const int64_t stride = (int64_t)gridDim.x * (blockDim.x - 32);
-        for (int64_t it0 = (int64_t)blockIdx.x * (blockDim.x - 32) + threadIdx.x - 32;
-             it0 < npass; it0 += 4 * stride) {
+        const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+        for (int64_t it0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it0 < npass;
+             it0 += 4 * stride) {
             double y[4];
             int64_t out[4];
 #pragma unroll
@@ -307,9 +162,8 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a)
             }
         }
     }
-    __syncthreads();
     if (sh.singular) {
-        if (threadIdx.x == 0 && a.status) *a.status = CM_ESINGULAR;
+        if (blockIdx.x == 0 && threadIdx.x == 0 && a.status) *a.status = CM_ESINGULAR;
         return;
     }
     // missing systematic blocks: up to CG of them per thread, one row position;
@@ -353,24 +207,15 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a)
 // every surviving element is read once.
 template <int EMAX>
 __global__ void __launch_bounds__(kThreads)
-decode_mat_kernel(const CodeParams cp, const float *Ct, int64_t ldc, uint32_t survivors, int N,
-                  float *C, int64_t ldcc, int32_t *status)
+decode_mat_kernel(const CodeParams cp, const __grid_constant__ DecodePlan plan, const float *Ct,
+                  int64_t ldc, int N, float *C, int64_t ldcc, int32_t *status)
 {
-    __shared__ DecodeShared sh;
-    __shared__ float Df[kMaxE][CM_MAX_N];
-    if (threadIdx.x < 32) {
-        decode_select(cp, survivors, sh);
-        __syncwarp();
-        decode_coefficients(cp, sh);
-    }
-    __syncthreads();
+    const DecodePlan &sh = plan;   // read in place (uniform accesses)
     if (sh.singular) {
-        if (threadIdx.x == 0 && status) *status = CM_ESINGULAR;
+        if (blockIdx.x == 0 && threadIdx.x == 0 && status) *status = CM_ESINGULAR;
         return;
     }
     const int k = cp.k, e = sh.e;
-    for (int t = threadIdx.x; t < e * k; t += blockDim.x) Df[t / k][t % k] = (float)sh.D[t / k][t % k];
-    __syncthreads();
     const int64_t L = cp.L, m = cp.m;
     const bool inplace = C == Ct;
     const bool vec = (N % 4 == 0) && (ldc % 4 == 0) && (ldcc % 4 == 0) &&
@@ -379,12 +224,8 @@ decode_mat_kernel(const CodeParams cp, const float *Ct, int64_t ldc, uint32_t su
     const int64_t nw = N / W;
     const int64_t total = L * nw;
     int M[EMAX];
-    {
-        int cnt = 0;
-        for (int i = 0; i < k && cnt < EMAX; ++i)
-            if (sh.role[i] >= 0) M[cnt++] = i;
-        for (; cnt < EMAX; ++cnt) M[cnt] = 0;
-    }
+#pragma unroll
+    for (int c = 0; c < EMAX; ++c) M[c] = c < e ? sh.M[c] : 0;
     for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < total;
          it += (int64_t)gridDim.x * blockDim.x) {
         const int64_t r = it / nw;
@@ -412,7 +253,7 @@ decode_mat_kernel(const CodeParams cp, const float *Ct, int64_t ldc, uint32_t su
 #pragma unroll
             for (int c = 0; c < EMAX; ++c) {
                 if (c < e) {
-                    const float w = Df[c][p];
+                    const float w = sh.Dh[c][p];
                     acc[c].x = fmaf(w, v.x, acc[c].x);
                     acc[c].y = fmaf(w, v.y, acc[c].y);
                     acc[c].z = fmaf(w, v.z, acc[c].z);
@@ -434,9 +275,7 @@ decode_mat_kernel(const CodeParams cp, const float *Ct, int64_t ldc, uint32_t su
     }
 }
 
-// Every CTA inverts the small block of G_S itself, so the grid is capped at
-// `per_sm` CTAs per SM: enough to stream the results, few enough that the
-// (slow on this part) fp64 inverse is not repeated needlessly.
+// CTAs for `items` independent items, at most `per_sm` per SM.
 int grid_for(int64_t items, int per_sm)
 {
     int64_t g = (items + kThreads - 1) / kThreads;
@@ -446,6 +285,99 @@ int grid_for(int64_t items, int per_sm)
     return (int)g;
 }
 
+// The decode of `survivors` (host, fp64): the survivor lists, then
+// Gauss-Jordan on [Q | I], Q = P[Ps][M] (e x e), fraction-free (a non-pivot
+// row becomes piv W[a] - W[a][col] W[col], two separately rounded products),
+// with partial pivoting on the fp32 image of |W[a][col]| (lowest index on
+// ties) and one division per row at the end: Q^-1[c][a] = W[c][e+a] / W[c][c].
+// G_S counts as singular when a pivot is zero or not finite, or when
+// ||Q||_inf ||Q^-1||_inf, bounded by ||Q||_inf e max|Q^-1|, exceeds
+// 1 / (64 eps).  Host code is compiled without floating-point contraction, so
+// the plan is the same on every host.
+void plan_decode(const CodeParams &cp, uint32_t survivors, DecodePlan &pl)
+{
+    const int n = cp.n, k = cp.k;
+    int Ps[kMaxE];
+    int ns = 0, e = 0, np = 0;
+    for (int j = 0; j < n && ns < k; ++j)
+        if ((survivors >> j) & 1u) {
+            pl.S[ns++] = j;
+            if (j >= k) Ps[np++] = j;
+        }
+    for (int i = 0; i < k; ++i) {
+        bool in = false;
+        for (int p = 0; p < ns; ++p) in = in || pl.S[p] == i;
+        if (!in) pl.M[e++] = i;
+    }
+    pl.e = e;
+    pl.singular = 0;
+    if (e == 0) return;
+    double W[kMaxE][2 * kMaxE];
+    double qnorm = 0.0;
+    for (int a = 0; a < e; ++a) {
+        double row = 0.0;
+        for (int c = 0; c < e; ++c) {
+            W[a][c] = (double)cp.P[(Ps[a] - k) * k + pl.M[c]];
+            row += std::fabs(W[a][c]);
+        }
+        for (int c = 0; c < e; ++c) W[a][e + c] = a == c ? 1.0 : 0.0;
+        qnorm = std::max(qnorm, row);
+    }
+    for (int col = 0; col < e; ++col) {
+        int bi = col;
+        float best = -1.f;
+        for (int a = col; a < e; ++a) {
+            const float f = (float)std::fabs(W[a][col]);
+            if (f > best) {
+                best = f;
+                bi = a;
+            }
+        }
+        const double piv = W[bi][col];
+        if (!(std::fabs(piv) > 0.0) || !std::isfinite(piv)) {
+            pl.singular = 1;
+            return;
+        }
+        if (bi != col)
+            for (int j = 0; j < 2 * e; ++j) std::swap(W[col][j], W[bi][j]);
+        for (int a = 0; a < e; ++a) {
+            if (a == col) continue;
+            const double fa = W[a][col];
+            for (int j = 0; j < 2 * e; ++j) {
+                const double p1 = piv * W[a][j], p2 = fa * W[col][j];
+                W[a][j] = j == col ? 0.0 : p1 - p2;
+            }
+        }
+    }
+    double Qi[kMaxE][kMaxE], qimax = 0.0;
+    for (int c = 0; c < e; ++c) {
+        const double dinv = 1.0 / W[c][c];
+        for (int a = 0; a < e; ++a) {
+            Qi[c][a] = W[c][e + a] * dinv;
+            qimax = std::max(qimax, std::fabs(Qi[c][a]));
+        }
+    }
+    if (!(qnorm * qimax * e < 1.0 / (64.0 * DBL_EPSILON))) {
+        pl.singular = 1;
+        return;
+    }
+    for (int c = 0; c < e; ++c)
+        for (int p = 0; p < k; ++p) {
+            const int sp = pl.S[p];
+            double v = 0.0;
+            if (sp >= k) {
+                for (int a = 0; a < e; ++a)
+                    if (Ps[a] == sp) v = Qi[c][a];
+            } else {
+                for (int a = 0; a < e; ++a)
+                    v = std::fma(-Qi[c][a], (double)cp.P[(Ps[a] - k) * k + sp], v);
+            }
+            const float h = (float)v;
+            pl.Dh[c][p] = h;
+            pl.Dl[c][p] = (float)(v - (double)h);
+        }
+}
+
 }  // namespace
 
 cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survivors, int b,
@@ -453,16 +385,17 @@ cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survi
                           cudaStream_t s)
 {
     DecodeArgs a;
+    std::memset(&a.plan, 0, sizeof(a.plan));
+    plan_decode(cp, survivors, a.plan);
     a.cp = cp;
     a.Yt = Yt;
-    a.survivors = survivors;
     a.b = b;
     a.Y = Y;
     a.status = status;
     a.mode = mode;
     a.lab = lab;
     a.eta = eta;
-    decode_kernel<<<grid_for((int64_t)cp.k * cp.L * b / 2 + 1, 2), kThreads, 0, s>>>(a);
+    decode_kernel<<<grid_for((int64_t)cp.k * cp.L * b / 2 + 1, 4), kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -470,20 +403,16 @@ cudaError_t launch_decode_mat(const CodeParams &cp, const float *Ct, int64_t ldc
                               uint32_t survivors, int N, float *C, int64_t ldcc, int32_t *status,
                               cudaStream_t s)
 {
-    // e = number of missing systematic blocks among the first k survivors
-    int e = 0, cnt = 0;
-    for (int j = 0; j < cp.n && cnt < cp.k; ++j)
-        if ((survivors >> j) & 1u) {
-            ++cnt;
-            if (j >= cp.k) ++e;
-        }
+    DecodePlan plan;
+    std::memset(&plan, 0, sizeof(plan));
+    plan_decode(cp, survivors, plan);
     const int64_t items = cp.L * (int64_t)N / 4 + 1;
-    const int g = grid_for(items, 4);
-    if (e <= 4)
-        decode_mat_kernel<4><<<g, kThreads, 0, s>>>(cp, Ct, ldc, survivors, N, C, ldcc, status);
-    else if (e <= 8)
-        decode_mat_kernel<8><<<g, kThreads, 0, s>>>(cp, Ct, ldc, survivors, N, C, ldcc, status);
+    const int g = grid_for(items, 8);
+    if (plan.e <= 4)
+        decode_mat_kernel<4><<<g, kThreads, 0, s>>>(cp, plan, Ct, ldc, N, C, ldcc, status);
+    else if (plan.e <= 8)
+        decode_mat_kernel<8><<<g, kThreads, 0, s>>>(cp, plan, Ct, ldc, N, C, ldcc, status);
     else
-        decode_mat_kernel<16><<<g, kThreads, 0, s>>>(cp, Ct, ldc, survivors, N, C, ldcc, status);
+        decode_mat_kernel<16><<<g, kThreads, 0, s>>>(cp, plan, Ct, ldc, N, C, ldcc, status);
     return cudaGetLastError();
 }

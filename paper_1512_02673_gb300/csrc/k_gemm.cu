@@ -16,12 +16,19 @@
 // was held near 0.8 of peak by shared-memory traffic (TMA fills plus tensor-
 // core operand reads).
 //
-// Tiles never straddle a worker block: worker j has ceil(L / 128) row tiles,
-// paired as (2 i, 2 i + 1) (the second one virtual past the block when the
-// count is odd: it loads zeros or foreign rows, and stores nothing); a tile's
-// last rows may read past the block and are not stored.  Pair order: column
-// tile fastest, so the 16 column tiles of one row pair run together and the
-// A~ row slab comes from HBM once; Bt (64 MB) stays L2-resident.
+// Row tiling.  The coded rows are two contiguous ranges: Ct rows [0, kL) are
+// rows of A in place (worker j < k owns [jL, jL + L)), Ct rows [kL, nL) are
+// rows of the parity buffer.  Each range is cut into 256-row pairs of its
+// own, A's over its m real rows only, so no tile computes the virtual zero
+// rows of every block's ragged end or reads a neighbour's rows: at (16,12)
+// with m = 32768 this gives 128 + 43 row pairs x 16 column tiles = 2736 work
+// items, 36 full waves of 76 pairs (per-worker tiles needed 2816, 38 waves
+// with a 4-item tail).  Rows past a range's end load as zeros (TMA
+// out-of-bounds fill) and are not stored; the pad rows [m, kL) of the last
+// systematic block are stored as zeros, by the last A pair's tiles where they
+// cover them and by its rank-1 CTA's epilogue past its end.  Pair order:
+// column tile fastest, so the 16 column tiles of one row pair run together
+// and the A~ row slab comes from HBM once; Bt (64 MB) stays L2-resident.
 //
 // One persistent CTA per SM, warp-specialised, in both CTAs of a pair:
 //   warp 0 lane 0  TMA producer of the CTA's halves (128B-swizzled 128 x 64
@@ -62,13 +69,14 @@ struct GemmArgs {
     float *Ct;
     int64_t ldc;
     int32_t *status;
-    int64_t L;
-    int32_t n, k, N;
-    int32_t mtiles;    // 128-row tiles per worker block
-    int32_t mpairs;    // row-tile pairs per worker block (ceil(mtiles / 2))
+    int64_t kL;        // Ct rows from A (systematic blocks, pad rows included)
+    int64_t pL;        // Ct rows from the parity buffer, (n - k) L
+    int32_t N;
+    int32_t psys;      // 256-row pairs over A's m rows
+    int32_t ppar;      // 256-row pairs over the parity rows
     int32_t ntiles;    // column tiles
     int32_t kblocks;   // 64-wide K blocks
-    int64_t pairs;     // (worker, row pair, column tile) work items
+    int64_t pairs;     // (row pair, column tile) work items
 };
 
 // ---- tcgen05 / cluster helpers (inline PTX) ------------------------------------------
@@ -199,25 +207,30 @@ __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32])
 }
 
 struct Tile {
-    int j;          // worker
-    int mt;         // 128-row tile within the worker block (may be virtual)
-    int n0;         // first output column
     bool parity;    // rows come from the parity buffer
-    int32_t y;      // row coordinate in A or in the parity buffer
+    int32_t y;      // first row in A or in the parity buffer
+    int n0;         // first output column
+    int64_t crow;   // Ct row of the tile's first row
+    int32_t rows;   // rows of the tile that exist in Ct (may be <= 0)
+    int32_t pad;    // pad rows [crow + BM, crow + BM + pad) to store as zeros
 };
 
-// CTA `rank`'s half of work item p: row tile 2 (p's row pair) + rank.
+// CTA `rank`'s half of work item p: rows [128 rank, 128 rank + 128) of p's
+// row pair.
 __device__ __forceinline__ Tile tile_of(const GemmArgs &g, int64_t p, int rank)
 {
     Tile x;
     const int nt = (int)(p % g.ntiles);
-    const int64_t rest = p / g.ntiles;
-    x.mt = 2 * (int)(rest % g.mpairs) + rank;
-    x.j = (int)(rest / g.mpairs);
+    const int rp = (int)(p / g.ntiles);
     x.n0 = nt * BN;
-    x.parity = x.j >= g.k;
-    const int64_t r0 = (int64_t)x.mt * BM;
-    x.y = (int32_t)(x.parity ? (int64_t)(x.j - g.k) * g.L + r0 : (int64_t)x.j * g.L + r0);
+    x.parity = rp >= g.psys;
+    const int64_t y = (int64_t)(x.parity ? rp - g.psys : rp) * (2 * BM) + rank * BM;
+    x.y = (int32_t)y;
+    const int64_t end = x.parity ? g.pL : g.kL;
+    x.crow = x.parity ? g.kL + y : y;
+    x.rows = (int32_t)(end - y < BM ? end - y : BM);
+    x.pad = (!x.parity && rank == 1 && rp == g.psys - 1 && y + BM < g.kL) ? (int32_t)(g.kL - y - BM)
+                                                                          : 0;
     return x;
 }
 
@@ -362,9 +375,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
             }
             tc_fence_after();
             const Tile x = tile_of(g, p, rank);
-            const int64_t r = (int64_t)x.mt * BM + row;
-            const bool valid = r < g.L;
-            float *dst = g.Ct + ((int64_t)x.j * g.L + r) * g.ldc + x.n0;
+            const bool valid = row < x.rows;
+            float *dst = g.Ct + (x.crow + row) * g.ldc + x.n0;
             const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
 #pragma unroll 1
             for (int c = 0; c < BN / 32; ++c) {
@@ -387,6 +399,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
             }
             tc_fence_before();
             mbar_arrive_cluster(map_to_rank(&tempty[acc], 0));   // release on the leader
+            if (row < x.pad) {   // pad rows of the last systematic block past the tile
+                float *z = dst + (int64_t)BM * g.ldc;
+                for (int c = 0; c < BN && x.n0 + c < g.N; ++c) z[c] = 0.0f;
+            }
             if (++acc == ACCS) {
                 acc = 0;
                 aph ^= 1u;
@@ -425,15 +441,14 @@ cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t l
     g.Ct = Ct;
     g.ldc = ldc;
     g.status = status;
-    g.L = cp.L;
-    g.n = cp.n;
-    g.k = cp.k;
+    g.kL = (int64_t)cp.k * cp.L;
+    g.pL = (int64_t)(cp.n - cp.k) * cp.L;
     g.N = N;
-    g.mtiles = (int)((cp.L + BM - 1) / BM);
-    g.mpairs = (g.mtiles + 1) / 2;
+    g.psys = (int)((cp.m + 2 * BM - 1) / (2 * BM));
+    g.ppar = (int)((g.pL + 2 * BM - 1) / (2 * BM));
     g.ntiles = (N + BN - 1) / BN;
     g.kblocks = (int)((cp.d + BK - 1) / BK);
-    g.pairs = (int64_t)cp.n * g.mpairs * g.ntiles;
+    g.pairs = (int64_t)(g.psys + g.ppar) * g.ntiles;
     cudaError_t e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          SMEM_BYTES);
     if (e != cudaSuccess) return e;

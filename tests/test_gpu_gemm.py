@@ -162,3 +162,29 @@ def test_gemm_config_sampled(cm, orc):
     assert err.max() <= 1e-2, err.max()
     del A, B, Bt, par, Ct, C
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("n,k,m,d,N", [
+    (4, 3, 512, 128, 64),        # kL = 513: the pad row lies past the last A tile pair
+    (4, 3, 1000, 64, 96),        # kL = 1002 < 1024: the last A pair overhangs the parity rows
+    (24, 20, 762, 64, 300),      # 12 pad rows past the last A pair, ragged column tile
+])
+def test_coded_gemm_writes_every_row_and_nothing_else(cm, orc, n, k, m, d, N):
+    P = synth.parity_coefficients(n, k)
+    code = cm.Code(n, k, m, d, P, dtype="bf16")
+    L = code.L
+    A = synth.gaussian((m, d), 11, dtype=torch.bfloat16).to(DEV)
+    B = synth.gaussian((d, N), 12, dtype=torch.bfloat16)
+    par = cm.encode(code, A)
+    guard = 7
+    buf = torch.full((n * L + guard, N), float("nan"), dtype=torch.float32, device=DEV)
+    Ct = cm.coded_gemm(code, A, par, B.t().contiguous().to(DEV), Ct=buf[:n * L])
+    torch.cuda.synchronize()
+    got = buf.double().cpu().numpy()
+    assert np.isnan(got[n * L:]).all()                       # rows past Ct untouched
+    assert not np.isnan(got[:n * L]).any()                   # every Ct row written
+    assert (got[m:k * L] == 0).all()                         # pad rows of the last block
+    want = orc.worker_outputs_bf16(n, k, bits(A), bits(par), bits(B))
+    for j in range(n):
+        err = rel_cols(got[j * L:(j + 1) * L], want[j * L:(j + 1) * L])
+        assert err.max() <= worker_tol(d), (j, err.max())

@@ -92,15 +92,19 @@ __device__ __forceinline__ void df_fma(float dh, float dl, float yh, float yl, f
 }
 
 struct DecodeArgs {
-    CodeParams cp;
+    int64_t L, m;
+    int32_t k;
+    int32_t b;
     DecodePlan plan;
     const double *Yt;
-    int b;
     float *Y;
     int32_t *status;
     int mode;
     const float *lab;
     float eta;
+    int32_t dec_ctas;         // CTAs of the decode role: the first ones in the grid
+    int32_t dec_per_group;    // of those, per group of CG missing blocks
+    int32_t pass_per_block;   // pass-through CTAs per surviving systematic block
 };
 
 constexpr int CG = 2;   // missing blocks decoded per thread
@@ -118,86 +122,84 @@ __device__ __forceinline__ void store_out(const DecodeArgs &a, int64_t out, floa
 
 // The plan stays in the parameter space: every access below is uniform
 // across a warp (one (c, p) at a time; S and M indexed by a block number that
-// changes only at block boundaries), which the constant cache serves by
-// broadcast; copying it to shared memory would read it divergently.
+// is fixed per CTA), which the constant cache serves by broadcast; copying it
+// to shared memory would read it divergently.
+//
+// Every CTA has one role, fixed by its index with one division per CTA: the
+// first dec_ctas CTAs form the missing blocks (group g = CTA / dec_per_group
+// of CG blocks, one row position per thread and pass), the others pass one
+// surviving systematic block through (kPassItems positions per thread, loads
+// issued together).  Decode CTAs come first so that their longer chains
+// (k loads, then k CG double-float FMAs) start first.
+constexpr int kPassItems = 4;
+
 __global__ void __launch_bounds__(kThreads) decode_kernel(const __grid_constant__ DecodeArgs a)
 {
     const DecodePlan &sh = a.plan;
-    const int k = a.cp.k, e = sh.e;
-    const int64_t L = a.cp.L, m = a.cp.m;
-    const int b = a.b;
-    const int64_t per_block = L * b;
-    {
-        // the surviving systematic blocks pass through (exactly rounded to
-        // fp32), four independent loads at a time
-        const int64_t npass = (int64_t)(k - e) * per_block;
-        const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-        for (int64_t it0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it0 < npass;
-             it0 += 4 * stride) {
-            double y[4];
-            int64_t out[4];
+    const int k = a.k, e = sh.e;
+    const int64_t per_block = a.L * a.b;
+    const int64_t mb = a.m * a.b;
+    int bx = (int)blockIdx.x;
+    if (bx < a.dec_ctas) {
+        if (sh.singular) {
+            if (bx == 0 && threadIdx.x == 0 && a.status) *a.status = CM_ESINGULAR;
+            return;
+        }
+        const int g = bx / a.dec_per_group;
+        const int c0 = g * CG;
+        const int64_t step = (int64_t)a.dec_per_group * kThreads;
+        for (int64_t rv = (int64_t)(bx - g * a.dec_per_group) * kThreads + threadIdx.x;
+             rv < per_block; rv += step) {
+            double yv[CM_MAX_N];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int64_t it = it0 + u * stride;
-                out[u] = -1;
-                if (it < npass) {
-                    const int t = (int)(it / per_block);
-                    const int64_t o = (int64_t)sh.S[t] * per_block + (it - (int64_t)t * per_block);
-                    if (o < m * b) {
-                        out[u] = o;
-                        y[u] = a.Yt[o];
-                    }
+            for (int p = 0; p < CM_MAX_N; ++p)
+                if (p < k) yv[p] = a.Yt[(int64_t)sh.S[p] * per_block + rv];
+            float sh_[CG], sl_[CG];
+#pragma unroll
+            for (int c = 0; c < CG; ++c) sh_[c] = sl_[c] = 0.f;
+#pragma unroll
+            for (int p = 0; p < CM_MAX_N; ++p) {
+                if (p < k) {
+                    float yh, yl;
+                    split_double(yv[p], yh, yl);
+#pragma unroll
+                    for (int c = 0; c < CG; ++c)
+                        if (c0 + c < e)
+                            df_fma(sh.Dh[c0 + c][p], sh.Dl[c0 + c][p], yh, yl, sh_[c], sl_[c]);
                 }
             }
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                if (out[u] < 0) continue;
-                if (a.mode == DEC_PLAIN) {
-                    a.Y[out[u]] = __double2float_rn(y[u]);
-                } else {
-                    float yh, yl;
-                    split_double(y[u], yh, yl);
-                    store_out(a, out[u], yh, yl);
+            for (int c = 0; c < CG; ++c) {
+                if (c0 + c < e) {
+                    const int64_t out = (int64_t)sh.M[c0 + c] * per_block + rv;
+                    if (out < mb) store_out(a, out, sh_[c], sl_[c]);
                 }
             }
         }
-    }
-    if (sh.singular) {
-        if (blockIdx.x == 0 && threadIdx.x == 0 && a.status) *a.status = CM_ESINGULAR;
         return;
     }
-    // missing systematic blocks: up to CG of them per thread, one row position;
-    // the k surviving values are loaded before any arithmetic
-    const int ngroups = (e + CG - 1) / CG;
-    const int64_t ndec = (int64_t)ngroups * per_block;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < ndec; it += stride) {
-        const int g = (int)(it / per_block);
-        const int64_t rv = it - (int64_t)g * per_block;
-        const int c0 = g * CG;
-        double yv[CM_MAX_N];
+    // a surviving systematic block passes through (exactly rounded to fp32)
+    bx -= a.dec_ctas;
+    const int t = bx / a.pass_per_block;
+    const int64_t base = (int64_t)sh.S[t] * per_block;
+    const int64_t lim = (mb - base < per_block ? mb - base : per_block);
+    const int64_t step = (int64_t)a.pass_per_block * kThreads * kPassItems;
+    for (int64_t i0 = (int64_t)(bx - t * a.pass_per_block) * kThreads * kPassItems + threadIdx.x;
+         i0 < lim; i0 += step) {
+        double y[kPassItems];
 #pragma unroll
-        for (int p = 0; p < CM_MAX_N; ++p)
-            if (p < k) yv[p] = a.Yt[(int64_t)sh.S[p] * per_block + rv];
-        float sh_[CG], sl_[CG];
+        for (int u = 0; u < kPassItems; ++u)
+            if (i0 + u * kThreads < lim) y[u] = a.Yt[base + i0 + u * kThreads];
 #pragma unroll
-        for (int c = 0; c < CG; ++c) sh_[c] = sl_[c] = 0.f;
-#pragma unroll
-        for (int p = 0; p < CM_MAX_N; ++p) {
-            if (p < k) {
+        for (int u = 0; u < kPassItems; ++u) {
+            if (i0 + u * kThreads >= lim) break;
+            const int64_t out = base + i0 + u * kThreads;
+            if (a.mode == DEC_PLAIN) {
+                a.Y[out] = __double2float_rn(y[u]);
+            } else {
                 float yh, yl;
-                split_double(yv[p], yh, yl);
-#pragma unroll
-                for (int c = 0; c < CG; ++c)
-                    if (c0 + c < e)
-                        df_fma(sh.Dh[c0 + c][p], sh.Dl[c0 + c][p], yh, yl, sh_[c], sl_[c]);
-            }
-        }
-#pragma unroll
-        for (int c = 0; c < CG; ++c) {
-            if (c0 + c < e) {
-                const int64_t out = (int64_t)sh.M[c0 + c] * per_block + rv;
-                if (out < m * b) store_out(a, out, sh_[c], sl_[c]);
+                split_double(y[u], yh, yl);
+                store_out(a, out, yh, yl);
             }
         }
     }
@@ -387,15 +389,28 @@ cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survi
     DecodeArgs a;
     std::memset(&a.plan, 0, sizeof(a.plan));
     plan_decode(cp, survivors, a.plan);
-    a.cp = cp;
-    a.Yt = Yt;
+    a.L = cp.L;
+    a.m = cp.m;
+    a.k = cp.k;
     a.b = b;
+    a.Yt = Yt;
     a.Y = Y;
     a.status = status;
     a.mode = mode;
     a.lab = lab;
     a.eta = eta;
-    decode_kernel<<<grid_for((int64_t)cp.k * cp.L * b / 2 + 1, 4), kThreads, 0, s>>>(a);
+    // CTAs per role, capped (threads then loop) so the grid stays well inside
+    // the launch limit for any block size
+    const int64_t per_block = cp.L * (int64_t)b;
+    const int64_t cap = 1 << 20;
+    const int e = a.plan.e, ngroups = (e + CG - 1) / CG;
+    a.dec_per_group = (int32_t)std::min(cap, (per_block + kThreads - 1) / kThreads);
+    a.dec_ctas = a.plan.singular ? 1 : ngroups * a.dec_per_group;
+    a.pass_per_block = (int32_t)std::min(
+        cap, (per_block + kThreads * kPassItems - 1) / (kThreads * kPassItems));
+    const int64_t grid = a.dec_ctas + (int64_t)(cp.k - e) * a.pass_per_block;
+    if (grid < 1) return cudaSuccess;
+    decode_kernel<<<(unsigned)grid, kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -134,7 +134,8 @@ encode_kernel(const __grid_constant__ CUtensorMap tmF, const __grid_constant__ C
         const int64_t r = p_unit / a.nseg;
         const int32_t x = ((int)(p_unit % a.nseg) * SEG + p_s) * STEP;
         unsigned char *dst = ring + p_slot * SLOT;
-        cm_fence_proxy_async();
+        // no proxy fence: the slot is only written by TMA, and the __syncwarp
+        // before every refill orders the lanes' reads of it before the copy
         if (p_c < nfull) {
             cm_mbar_arrive_expect_tx(&bar[p_slot], SLOT);
             cm_tma_load_3d(dst, &tmF, x, (int32_t)r, p_c * KC, &bar[p_slot]);

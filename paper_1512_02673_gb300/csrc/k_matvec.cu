@@ -14,7 +14,11 @@
 // Data movement.  The unit's rows stream through a per-warp ring of ST
 // shared-memory slots, one 2-D TMA box (R rows x 128 columns) per step issued
 // by the warp's lane 0 and counted on the slot's mbarrier, so ST steps are in
-// flight per warp without any per-lane copy work.  The tensor maps zero-fill
+// flight per warp without any per-lane copy work.  Lane 0 refills a slot after
+// a __syncwarp that follows every lane's reads of it: the warp barrier orders
+// those reads before the copy is issued, and the slot is only ever written by
+// TMA, so there is no generic-proxy write for a proxy fence to publish (one
+// per step cost 3 % of the bandwidth at b = 8).  The tensor maps zero-fill
 // whatever lies outside A or the parity buffer: the appended zero rows past m
 // and the ragged column tail cost nothing.  Each coded element is read from
 // HBM exactly once.  X is staged per chunk of columns by cp.async (double
@@ -42,10 +46,10 @@
 namespace {
 
 
-template <int BP>
+template <int BP, int XF = 4096>
 struct XCfg {
-    // columns per staged X chunk (16 KB of X per buffer)
-    static constexpr int CX = 4096 / BP;
+    // columns per staged X chunk (XF floats of X per buffer)
+    static constexpr int CX = XF / BP;
     // floats between the [vector] rows of the smem layout: the 4-float pad
     // makes the staging stores of 32 consecutive (column, vector) elements hit
     // 32 distinct banks.
@@ -53,11 +57,11 @@ struct XCfg {
     static constexpr int FLOATS = BP * GS;
 };
 
-template <int BP, int R, int ST, int W>
+template <int BP, int R, int ST, int W, int XF>
 struct Smem {
     static constexpr int SLOT_FLOATS = R * 128;
     static constexpr int RING_BYTES = W * ST * SLOT_FLOATS * 4;
-    static constexpr int X_BYTES = 2 * XCfg<BP>::FLOATS * 4;
+    static constexpr int X_BYTES = 2 * XCfg<BP, XF>::FLOATS * 4;
     static constexpr int BAR_BYTES = W * ST * 8;
     static constexpr int TOTAL = 1024 + RING_BYTES + X_BYTES + BAR_BYTES;   // + alignment slack
 };
@@ -94,10 +98,10 @@ __device__ __forceinline__ void cp_async_wait_all()
 
 // Stage columns [c0, c0 + CX) of X into smem buffer xs as xs[v * GS + col]
 // (zero past d and for padded vectors v >= b).
-template <int BP, int kThreads>
+template <int BP, int XF, int kThreads>
 __device__ __forceinline__ void stage_x(const MatvecArgs &a, float *xs, int64_t c0)
 {
-    using C = XCfg<BP>;
+    using C = XCfg<BP, XF>;
     const int tid = threadIdx.x;
     const float *X = a.X;
     if (BP == 1 && a.fast16) {
@@ -180,14 +184,15 @@ __device__ __forceinline__ Unit unit_of(const MatvecArgs &a, int64_t g, int R)
     return u;
 }
 
-template <int BP, int R, int ST, int F, int kWarps>
+template <int BP, int R, int ST, int F, int kWarps, int XF>
 __global__ void __launch_bounds__(kWarps * 32, 1)
 matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmP,
               const MatvecArgs a)
 {
     constexpr int kThreads = kWarps * 32;
-    using C = XCfg<BP>;
-    using S = Smem<BP, R, ST, kWarps>;
+    using C = XCfg<BP, XF>;
+    using S = Smem<BP, R, ST, kWarps, XF>;
+    static_assert(S::TOTAL <= 232448, "shared memory per CTA");
     constexpr int V = R * BP;
     constexpr int NH = V >= 32 ? V / 32 : 1;
     constexpr int IPC = C::CX / 128;   // steps per X chunk (a power of two)
@@ -221,7 +226,6 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     int p_slot = 0, p_s = 0, p_round = 0;
     Unit pu = unit_of(a, gw, R);
     auto produce = [&]() {   // lane 0 only; loads step p_idx into slot p_slot
-        cm_fence_proxy_async();
         cm_mbar_arrive_expect_tx(&bar[p_slot], STEP_BYTES);
         cm_tma_load_2d(ring + p_slot * S::SLOT_FLOATS, pu.parity ? &tmP : &tmA, 128 * p_s, pu.y,
                        &bar[p_slot]);
@@ -236,7 +240,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     if (lane == 0)
         while (p_idx < my_steps && p_idx < ST) produce();
 
-    stage_x<BP, kThreads>(a, xs, 0);
+    stage_x<BP, XF, kThreads>(a, xs, 0);
 
     // ---- consumer ----
     int xbuf = 0;             // X buffer of the current chunk
@@ -260,7 +264,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
             cp_async_wait_all();
             __syncthreads();   // X chunk visible; every warp is done with the other buffer
             if (ch + 1 < nchunks || round + 1 < rounds)
-                stage_x<BP, kThreads>(a, xs + (xbuf ^ 1) * C::FLOATS,
+                stage_x<BP, XF, kThreads>(a, xs + (xbuf ^ 1) * C::FLOATS,
                                       ch + 1 < nchunks ? (int64_t)(ch + 1) * C::CX : 0);
             const int ns = steps - ch * IPC < IPC ? steps - ch * IPC : IPC;
             if (has && !failed) {
@@ -354,13 +358,13 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     }
 }
 
-template <int BP, int R, int ST, int F, int kWarps>
+template <int BP, int R, int ST, int F, int kWarps, int XF = 4096>
 cudaError_t launch_bp(MatvecArgs a, const float *A, int64_t lda, const float *par, int64_t ldp,
                       cudaStream_t s)
 {
     constexpr int kThreads = kWarps * 32;
-    using S = Smem<BP, R, ST, kWarps>;
-    auto kern = matvec_kernel<BP, R, ST, F, kWarps>;
+    using S = Smem<BP, R, ST, kWarps, XF>;
+    auto kern = matvec_kernel<BP, R, ST, F, kWarps, XF>;
     CUtensorMap tmA, tmP;
     if (!cm_make_tmap_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, A, a.d, a.m, lda * 4, 128, R,
                          CU_TENSOR_MAP_SWIZZLE_NONE) ||

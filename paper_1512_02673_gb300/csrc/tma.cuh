@@ -43,13 +43,6 @@ __device__ __forceinline__ void cm_fence_mbar_init()
     asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
 }
 
-// Order this thread's earlier generic-proxy shared-memory accesses before
-// later async-proxy (TMA) accesses of the same memory.
-__device__ __forceinline__ void cm_fence_proxy_async()
-{
-    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
-}
-
 __device__ __forceinline__ void cm_mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes)
 {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(cm_smem_u32(bar)),

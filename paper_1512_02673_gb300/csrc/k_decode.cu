@@ -11,14 +11,18 @@
 // the rows of G_S^-1 for the missing blocks are
 //   coefficient of Yt_s, s in Ps  :  Q^-1[c][pos of s in Ps]
 //   coefficient of Yt_s, s in Ks  : -sum_a Q^-1[c][a] P[Ps[a]][s]
-// The master knows the survivors when it decodes, so the library's host code
-// forms these coefficients once per call (plan_decode, fp64, a few
-// microseconds; formed on the device they cost every CTA ~10 us of
-// latency-bound fp64 work) and passes them to the kernel by value; the
-// kernel's threads apply them: missing block M[c] row r is the combination of
-// the k surviving rows r, surviving systematic blocks pass through.  A zero
-// (or relatively negligible) pivot marks G_S singular: the kernel writes
-// CM_ESINGULAR to the status word and writes no decoded block.
+//
+// Two kernels per decode.  A small plan kernel (one CTA) inverts Q in fp64
+// on the device and writes the rows of G_S^-1 for the missing blocks to a
+// plan slot; the apply kernel is launched right behind it as a programmatic
+// dependent launch, so its launch overlaps the inversion: its pass-through
+// CTAs (surviving systematic blocks, which need no inverse) run at once, and
+// its decode CTAs issue the loads of their k surviving values, then wait for
+// the plan (griddepcontrol.wait) and apply it: missing block M[c] row r is
+// the combination of the k surviving rows r.  A zero (or relatively
+// negligible) pivot marks G_S singular: the kernel writes CM_ESINGULAR to
+// the status word and writes no decoded block.  With no missing block there
+// is no plan kernel.
 //
 // fp64 arithmetic runs at about 1/58 of the fp32 rate on this part, so the
 // vector decode applies the fp64 coefficients in double-float arithmetic on
@@ -28,28 +32,65 @@
 // as (sum, compensation) pairs (Knuth's TwoSum), about 2^-44 relative per
 // term, far below the rounding of the fp32 output.
 #include <algorithm>
+#include <atomic>
 #include <cfloat>
 #include <cmath>
-#include <cstring>
 
 #include "cm_internal.cuh"
 
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 256;       // apply kernels
+constexpr int kPlanThreads = 512;   // plan kernel: one entry of [Q | I] per thread
 constexpr int kMaxE = 16;   // e <= min(k, n - k) <= 16 for n <= 32
 
-// The decode of one survivor mask, formed on the host (plan_decode below) and
-// passed to the kernels by value: the survivors used, the missing systematic
-// blocks, and the rows of G_S^-1 for those blocks as (high, low) fp32 pairs.
+// The decode of one survivor mask, formed in shared memory by every CTA that
+// needs it (decode_plan below): the survivors used, the missing systematic
+// blocks, the elimination's working matrix and the rows of G_S^-1 for the
+// missing blocks as (high, low) fp32 pairs.
 struct DecodePlan {
     int32_t e;               // missing systematic blocks
     int32_t singular;        // G_S judged singular: decode nothing
     int32_t S[CM_MAX_N];     // survivors in ascending order (k of them)
+    int32_t Ps[kMaxE];       // surviving parity workers, ascending
     int32_t M[kMaxE];        // missing systematic blocks, ascending
-    float Dh[kMaxE][CM_MAX_N];   // D[c][p] (p = position in S), rounded to fp32
-    float Dl[kMaxE][CM_MAX_N];   // D - Dh, rounded to fp32
+    int32_t bi[kMaxE];       // pivot row (in the current row order) of each column
+    double piv[kMaxE];       // that pivot's value
+    float qmax;              // max |Q| (bounds ||Q||_inf by e max|Q|)
+    unsigned long long qimax;   // max |Q^-1| as a magnitude key
+    // [Q | I | P_K] column-major, W[buf][column][row], ping-pong; P_K holds
+    // P[Ps][s] for the surviving systematic workers s
+    double W[2][kMaxE + CM_MAX_N][kMaxE];
+    double rcp[kMaxE];       // 1 / final pivot of each row
+    float Dh[kMaxE][CM_MAX_N];   // D[c][p] (p = position in S), high part
+    float Dl[kMaxE][CM_MAX_N];   // D - Dh
 };
+
+// What the apply kernels need of a plan: written by the plan kernel into a
+// slot of a ring in static device memory (no allocation per call).
+struct DecodeRows {
+    int32_t e;
+    int32_t singular;
+    int32_t M[kMaxE];
+    float Dh[kMaxE][CM_MAX_N];
+    float Dl[kMaxE][CM_MAX_N];
+};
+
+// Slots in flight at once: a call takes the next slot, so up to this many
+// decodes may be pending at a time across streams.
+constexpr int kPlanSlots = 256;
+__device__ DecodeRows g_decode_rows[kPlanSlots];
+std::atomic<uint32_t> g_next_rows{0};
+
+__device__ __forceinline__ void griddep_wait()
+{
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+}
+
+__device__ __forceinline__ void griddep_launch_dependents()
+{
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
 
 // ---- double-float helpers (fp32 pipe only) -------------------------------------------
 
@@ -91,11 +132,253 @@ __device__ __forceinline__ void df_fma(float dh, float dl, float yh, float yl, f
     sh = s1;
 }
 
+// Magnitude key of an fp64 value for pivot search: the bits of |v|, which
+// order like the values for every finite |v| (integer compares, no fp64
+// instruction); not-a-number counts as the largest, so it is chosen and
+// flagged.
+__device__ __forceinline__ long long mag_key(double v)
+{
+    return __double_as_longlong(v) & 0x7fffffffffffffffll;
+}
+
+constexpr long long kInfKey = 0x7ff0000000000000ll;
+
+// Largest key over the 16 lanes of this half-warp, lowest row on ties; every
+// lane of the half ends with the winner's row.
+__device__ __forceinline__ int half_argmax(long long key, int row)
+{
+#pragma unroll
+    for (int off = 8; off; off >>= 1) {
+        const long long ok = __shfl_xor_sync(0xffffffffu, key, off);
+        const int orow = __shfl_xor_sync(0xffffffffu, row, off);
+        if (ok > key || (ok == key && orow < row)) {
+            key = ok;
+            row = orow;
+        }
+    }
+    return row;
+}
+
+// Largest non-negative float of the CTA into *dst (zero beforehand), by a
+// warp maximum and one atomic per warp (an exact, order-free maximum).
+__device__ __forceinline__ void cta_max(float v, float *dst)
+{
+#pragma unroll
+    for (int off = 16; off; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+    if ((threadIdx.x & 31) == 0 && v > 0.f) atomicMax(reinterpret_cast<int *>(dst), __float_as_int(v));
+}
+
+// The same for magnitude keys.
+__device__ __forceinline__ void cta_max_key(long long v, unsigned long long *dst)
+{
+#pragma unroll
+    for (int off = 16; off; off >>= 1) {
+        const long long o = __shfl_xor_sync(0xffffffffu, v, off);
+        v = o > v ? o : v;
+    }
+    if ((threadIdx.x & 31) == 0 && v > 0) atomicMax(dst, (unsigned long long)v);
+}
+
+// fp64 value of an fp32 value by bit manipulation (exact; no fp64
+// instruction: single fp64 operations have a long latency on this part).
+__device__ __forceinline__ double exact_double(float f)
+{
+    const uint32_t u = __float_as_uint(f);
+    const uint32_t ex = (u >> 23) & 0xFFu, man = u & 0x7FFFFFu;
+    const unsigned long long sign = (unsigned long long)(u >> 31) << 63;
+    if (ex == 0xFFu)   // infinite or not a number
+        return __longlong_as_double((long long)(sign | 0x7FF0000000000000ull |
+                                                ((unsigned long long)man << 29)));
+    if (ex == 0) {     // zero or subnormal: normalise the mantissa
+        if (man == 0) return __longlong_as_double((long long)sign);
+        const int sh = __clz((int)man) - 8;   // shifts that bring the top bit to bit 23
+        const uint32_t m = (man << sh) & 0x7FFFFFu;
+        return __longlong_as_double((long long)(sign | ((unsigned long long)(897 - sh) << 52) |
+                                                ((unsigned long long)m << 29)));
+    }
+    return __longlong_as_double((long long)(sign | ((unsigned long long)(ex + 896) << 52) |
+                                            ((unsigned long long)man << 29)));
+}
+
+// The decode of `survivors` in shared memory, by all kPlanThreads threads of
+// the CTA (call it from every thread; it ends with a CTA barrier).
+//  * Survivor lists by ballots in warp 0: S (the first k set bits), Ps (the
+//    surviving parity workers among them), M (the missing systematic blocks);
+//    the ks = k - e surviving systematic workers are S[0, ks).
+//  * Gauss-Jordan in fp64 on W = [Q | I | P_K], Q = P[Ps][M] (e x e),
+//    P_K = P[Ps][S[0, ks)]; thread t holds entry (row t % 16, column t / 16)
+//    and the one 512 further on.  fp64 latency is long on this part, so the
+//    elimination is fraction-free: at column col with pivot row bi, the pivot
+//    row moves to position col unchanged and every other row r becomes
+//    piv W[r] - W[r][col] W[bi] (two separately rounded products, so
+//    duplicated rows cancel to exactly zero); each row is scaled by its
+//    pivot once at the end, which leaves Q^-1 in the second block and
+//    Q^-1 P_K in the third.  The row swap is part of the update, which reads
+//    one buffer and writes the other: one CTA barrier per column.  The 16
+//    rows of a column sit in one half-warp, which picks the next column's
+//    pivot right after computing it: the largest |W[a][col]|, a >= col
+//    (exact magnitudes compared as integers), lowest row on ties.
+//  * G_S counts as singular when a pivot is zero or not finite, or when
+//    ||Q||_inf ||Q^-1||_inf, bounded by (e max|Q|) (e max|Q^-1|), exceeds
+//    1 / (64 eps) (evaluated in fp32: it is a threshold).
+//  * D[c][p], the coefficient of the p-th survivor in missing block M[c]:
+//    Q^-1[c][a] for the surviving parity worker Ps[a] = S[ks + a], and
+//    -(Q^-1 P_K)[c][p] for the surviving systematic worker S[p], p < ks;
+//    kept as a (high, low) fp32 pair.
+__device__ void decode_plan(const CodeParams &cp, uint32_t survivors, DecodePlan &pl)
+{
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int n = cp.n, k = cp.k;
+    if (tid < 32) {
+        const uint32_t below = (1u << lane) - 1u;
+        const bool set = lane < n && ((survivors >> lane) & 1u);
+        const bool sel = set && __popc(survivors & below) < k;
+        const uint32_t selm = __ballot_sync(0xffffffffu, sel);
+        const bool miss = lane < k && !sel;
+        const uint32_t missm = __ballot_sync(0xffffffffu, miss);
+        const bool par = sel && lane >= k;
+        const uint32_t parm = __ballot_sync(0xffffffffu, par);
+        if (sel) pl.S[__popc(selm & below)] = lane;
+        if (par) pl.Ps[__popc(parm & below)] = lane;
+        if (miss) pl.M[__popc(missm & below)] = lane;
+        if (lane == 0) {
+            pl.e = __popc(missm);
+            pl.singular = 0;
+            pl.qmax = 0.f;
+            pl.qimax = 0ull;
+        }
+    }
+    __syncthreads();
+    const int e = pl.e, ks = k - e;
+    if (e == 0) return;
+    const float *P = cp.P;
+    const int ncol = 2 * e + ks;   // e + k columns
+    {
+        float q0 = 0.f, qm = 0.f;
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int t = tid + u * kPlanThreads;
+            const int j = t >> 4, a = t & 15;
+            if (j < ncol && a < e) {
+                double w;
+                if (j < e) {
+                    const float q = P[(pl.Ps[a] - k) * k + pl.M[j]];
+                    w = exact_double(q);
+                    qm = fmaxf(qm, fabsf(q));
+                    if (j == 0) q0 = q;
+                } else if (j < 2 * e) {
+                    w = j - e == a ? 1.0 : 0.0;
+                } else {
+                    w = exact_double(P[(pl.Ps[a] - k) * k + pl.S[j - 2 * e]]);
+                }
+                pl.W[0][j][a] = w;
+            }
+        }
+        // pivot of column 0 (half-warp 0): the fp64 entries are the fp32 values
+        const int a = tid & 15;
+        const int b0 = half_argmax(tid < 16 && a < e ? (long long)__float_as_int(fabsf(q0)) : -1ll, a);
+        if (tid == 0) {
+            pl.bi[0] = b0;
+            pl.piv[0] = exact_double(P[(pl.Ps[b0] - k) * k + pl.M[0]]);
+        }
+        cta_max(qm, &pl.qmax);
+    }
+    __syncthreads();
+    for (int col = 0; col < e; ++col) {
+        const int cur = col & 1, nxt = cur ^ 1;
+        const int bi = pl.bi[col];
+        const double piv = pl.piv[col];
+        const long long pk = mag_key(piv);
+        if (pk == 0 || pk >= kInfKey) {   // zero, infinite or not a number
+            __syncthreads();
+            if (tid == 0) pl.singular = 1;
+            __syncthreads();
+            return;
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int t = tid + u * kPlanThreads;
+            const int j = t >> 4, a = t & 15;
+            double nv = 0.0;
+            if (j < ncol && a < e) {
+                if (a == col) {
+                    nv = pl.W[cur][j][bi];
+                } else if (j != col) {
+                    const int r = a == bi ? col : a;
+                    nv = __dsub_rn(__dmul_rn(piv, pl.W[cur][j][r]),
+                                   __dmul_rn(pl.W[cur][col][r], pl.W[cur][j][bi]));
+                }
+                pl.W[nxt][j][a] = nv;
+            }
+            if (u == 0 && col + 1 < e) {   // the half-warp of column col + 1 picks its pivot
+                const bool cand = j == col + 1 && a > col && a < e;
+                const int nb = half_argmax(cand ? mag_key(nv) : -1ll, a);
+                if (j == col + 1 && a == nb) {
+                    pl.bi[col + 1] = nb;
+                    pl.piv[col + 1] = nv;
+                }
+            }
+        }
+        __syncthreads();
+    }
+    const int fin = e & 1;
+    if (tid < e) pl.rcp[tid] = 1.0 / pl.W[fin][tid][tid];
+    __syncthreads();
+    // D rows (one entry per thread): scaled entries of the last two blocks
+    long long qk = 0;
+    if (tid < e * k) {
+        const int c = tid / k, p = tid - c * k;
+        double v;
+        if (p >= ks) {
+            v = __dmul_rn(pl.W[fin][e + (p - ks)][c], pl.rcp[c]);
+            qk = mag_key(v);
+        } else {
+            v = -__dmul_rn(pl.W[fin][2 * e + p][c], pl.rcp[c]);
+        }
+        float h, l;
+        split_double(v, h, l);
+        pl.Dh[c][p] = h;
+        pl.Dl[c][p] = l;
+    }
+    cta_max_key(qk, &pl.qimax);
+    __syncthreads();
+    const float qi = __double2float_ru(__longlong_as_double((long long)pl.qimax));
+    if (!((float)e * pl.qmax * ((float)e * qi) < (float)(1.0 / (64.0 * DBL_EPSILON)))) {
+        __syncthreads();   // every thread has read the maxima before the flag is set
+        if (tid == 0) pl.singular = 1;
+        __syncthreads();
+    }
+}
+
+// The plan kernel: one CTA inverts Q and writes the decode rows.  It lets
+// the apply kernel launch at once; that kernel's griddepcontrol.wait still
+// waits for this grid to complete and its writes to be visible.
+__global__ void __launch_bounds__(kPlanThreads, 1)
+plan_kernel(const CodeParams cp, uint32_t survivors, DecodeRows *out)
+{
+    griddep_launch_dependents();
+    __shared__ DecodePlan pl;
+    decode_plan(cp, survivors, pl);
+    const int e = pl.e, k = cp.k;
+    if (threadIdx.x == 0) {
+        out->e = e;
+        out->singular = pl.singular;
+    }
+    if (threadIdx.x < kMaxE) out->M[threadIdx.x] = threadIdx.x < e ? pl.M[threadIdx.x] : 0;
+    if (pl.singular) return;
+    for (int t = threadIdx.x; t < e * k; t += kPlanThreads) {
+        const int c = t / k, p = t - c * k;
+        out->Dh[c][p] = pl.Dh[c][p];
+        out->Dl[c][p] = pl.Dl[c][p];
+    }
+}
+
 struct DecodeArgs {
     int64_t L, m;
     int32_t k;
     int32_t b;
-    DecodePlan plan;
+    uint32_t survivors;       // the first k set bits are the survivors used
+    const DecodeRows *rows;   // the plan kernel's output (when blocks are missing)
     const double *Yt;
     float *Y;
     int32_t *status;
@@ -120,40 +403,70 @@ __device__ __forceinline__ void store_out(const DecodeArgs &a, int64_t out, floa
     }
 }
 
-// The plan stays in the parameter space: every access below is uniform
-// across a warp (one (c, p) at a time; S and M indexed by a block number that
-// is fixed per CTA), which the constant cache serves by broadcast; copying it
-// to shared memory would read it divergently.
-//
-// Every CTA has one role, fixed by its index with one division per CTA: the
-// first dec_ctas CTAs form the missing blocks (group g = CTA / dec_per_group
-// of CG blocks, one row position per thread and pass), the others pass one
-// surviving systematic block through (kPassItems positions per thread, loads
-// issued together).  Decode CTAs come first so that their longer chains
-// (k loads, then k CG double-float FMAs) start first.
+// Index of the t-th set bit of x (t from 0; x has more than t set bits).
+__device__ __forceinline__ int nth_set_bit(uint32_t x, int t)
+{
+    for (int i = 0; i < t; ++i) x &= x - 1u;
+    return __ffs((int)x) - 1;
+}
+
+// Loads of the k surviving values at position rv (the survivors are the
+// first k set bits of the mask).
+__device__ __forceinline__ void load_survivors(const DecodeArgs &a, int64_t per_block, int64_t rv,
+                                               double (&yv)[CM_MAX_N])
+{
+    uint32_t rest = a.survivors;
+#pragma unroll
+    for (int p = 0; p < CM_MAX_N; ++p) {
+        if (p < a.k) {
+            const int s = __ffs((int)rest) - 1;
+            rest &= rest - 1u;
+            yv[p] = a.Yt[(int64_t)s * per_block + rv];
+        }
+    }
+}
+
+// K3, the apply kernel.  Every CTA has one role, fixed by its index with one
+// division per CTA: the first dec_ctas CTAs form the missing blocks (group
+// g = CTA / dec_per_group of CG blocks, one row position per thread and
+// pass), the others pass one surviving systematic block through (kPassItems
+// positions per thread, loads issued together).  Decode CTAs come first;
+// they issue their first loads, then wait for the plan and copy their CG
+// rows of it to shared memory (read there with warp-uniform addresses).
 constexpr int kPassItems = 4;
 
 __global__ void __launch_bounds__(kThreads) decode_kernel(const __grid_constant__ DecodeArgs a)
 {
-    const DecodePlan &sh = a.plan;
-    const int k = a.k, e = sh.e;
+    const int k = a.k;
     const int64_t per_block = a.L * a.b;
     const int64_t mb = a.m * a.b;
     int bx = (int)blockIdx.x;
     if (bx < a.dec_ctas) {
-        if (sh.singular) {
-            if (bx == 0 && threadIdx.x == 0 && a.status) *a.status = CM_ESINGULAR;
-            return;
-        }
+        __shared__ float Dh[CG][CM_MAX_N], Dl[CG][CM_MAX_N];
+        __shared__ int32_t Mo[CG], ctl[2];
         const int g = bx / a.dec_per_group;
         const int c0 = g * CG;
         const int64_t step = (int64_t)a.dec_per_group * kThreads;
-        for (int64_t rv = (int64_t)(bx - g * a.dec_per_group) * kThreads + threadIdx.x;
-             rv < per_block; rv += step) {
-            double yv[CM_MAX_N];
-#pragma unroll
-            for (int p = 0; p < CM_MAX_N; ++p)
-                if (p < k) yv[p] = a.Yt[(int64_t)sh.S[p] * per_block + rv];
+        int64_t rv = (int64_t)(bx - g * a.dec_per_group) * kThreads + threadIdx.x;
+        double yv[CM_MAX_N];
+        if (rv < per_block) load_survivors(a, per_block, rv, yv);
+        griddep_wait();   // the plan kernel has completed
+        const DecodeRows *rows = a.rows;
+        if (threadIdx.x < 2) ctl[threadIdx.x] = threadIdx.x == 0 ? rows->e : rows->singular;
+        if (threadIdx.x < CG) Mo[threadIdx.x] = rows->M[(c0 + threadIdx.x) & (kMaxE - 1)];
+        for (int t = threadIdx.x; t < CG * CM_MAX_N; t += kThreads) {
+            const int c = t / CM_MAX_N, p = t - c * CM_MAX_N;
+            const int cc = (c0 + c) & (kMaxE - 1);
+            Dh[c][p] = rows->Dh[cc][p];
+            Dl[c][p] = rows->Dl[cc][p];
+        }
+        __syncthreads();
+        if (ctl[1]) {
+            if (bx == 0 && threadIdx.x == 0 && a.status) *a.status = CM_ESINGULAR;
+            return;
+        }
+        const int e = ctl[0];
+        while (rv < per_block) {
             float sh_[CG], sl_[CG];
 #pragma unroll
             for (int c = 0; c < CG; ++c) sh_[c] = sl_[c] = 0.f;
@@ -164,24 +477,28 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const __grid_constant_
                     split_double(yv[p], yh, yl);
 #pragma unroll
                     for (int c = 0; c < CG; ++c)
-                        if (c0 + c < e)
-                            df_fma(sh.Dh[c0 + c][p], sh.Dl[c0 + c][p], yh, yl, sh_[c], sl_[c]);
+                        if (c0 + c < e) df_fma(Dh[c][p], Dl[c][p], yh, yl, sh_[c], sl_[c]);
                 }
             }
 #pragma unroll
             for (int c = 0; c < CG; ++c) {
                 if (c0 + c < e) {
-                    const int64_t out = (int64_t)sh.M[c0 + c] * per_block + rv;
+                    const int64_t out = (int64_t)Mo[c] * per_block + rv;
                     if (out < mb) store_out(a, out, sh_[c], sl_[c]);
                 }
             }
+            rv += step;
+            if (rv >= per_block) break;
+            load_survivors(a, per_block, rv, yv);
         }
         return;
     }
-    // a surviving systematic block passes through (exactly rounded to fp32)
+    // a surviving systematic block passes through (exactly rounded to fp32);
+    // block t is the t-th set bit of the mask below k
     bx -= a.dec_ctas;
     const int t = bx / a.pass_per_block;
-    const int64_t base = (int64_t)sh.S[t] * per_block;
+    const int64_t base =
+        (int64_t)nth_set_bit(a.survivors & (k < 32 ? (1u << k) - 1u : 0xffffffffu), t) * per_block;
     const int64_t lim = (mb - base < per_block ? mb - base : per_block);
     const int64_t step = (int64_t)a.pass_per_block * kThreads * kPassItems;
     for (int64_t i0 = (int64_t)(bx - t * a.pass_per_block) * kThreads * kPassItems + threadIdx.x;
@@ -206,19 +523,33 @@ __global__ void __launch_bounds__(kThreads) decode_kernel(const __grid_constant_
 }
 
 // K6: fp32 results, all e missing blocks of one row position per thread, so
-// every surviving element is read once.
+// every surviving element is read once.  Launched behind the plan kernel
+// like K3; every CTA waits for the plan and copies its fp32 coefficients
+// (the high parts) to shared memory.
 template <int EMAX>
 __global__ void __launch_bounds__(kThreads)
-decode_mat_kernel(const CodeParams cp, const __grid_constant__ DecodePlan plan, const float *Ct,
-                  int64_t ldc, int N, float *C, int64_t ldcc, int32_t *status)
+decode_mat_kernel(int32_t k, int64_t L, int64_t m, uint32_t survivors, const DecodeRows *rows,
+                  const float *Ct, int64_t ldc, int N, float *C, int64_t ldcc, int32_t *status)
 {
-    const DecodePlan &sh = plan;   // read in place (uniform accesses)
-    if (sh.singular) {
+    __shared__ float Dh[EMAX][CM_MAX_N];
+    __shared__ int32_t S[CM_MAX_N], Mo[EMAX], ctl[2];
+    if (threadIdx.x < CM_MAX_N) {
+        // survivors: the first k set bits of the mask
+        const uint32_t below = (1u << threadIdx.x) - 1u;
+        if (((survivors >> threadIdx.x) & 1u) && __popc(survivors & below) < k)
+            S[__popc(survivors & below)] = threadIdx.x;
+    }
+    griddep_wait();   // the plan kernel has completed
+    if (threadIdx.x < 2) ctl[threadIdx.x] = threadIdx.x == 0 ? rows->e : rows->singular;
+    if (threadIdx.x < EMAX) Mo[threadIdx.x] = rows->M[threadIdx.x];
+    for (int t = threadIdx.x; t < EMAX * CM_MAX_N; t += kThreads)
+        Dh[t / CM_MAX_N][t % CM_MAX_N] = rows->Dh[t / CM_MAX_N][t % CM_MAX_N];
+    __syncthreads();
+    if (ctl[1]) {
         if (blockIdx.x == 0 && threadIdx.x == 0 && status) *status = CM_ESINGULAR;
         return;
     }
-    const int k = cp.k, e = sh.e;
-    const int64_t L = cp.L, m = cp.m;
+    const int e = ctl[0];
     const bool inplace = C == Ct;
     const bool vec = (N % 4 == 0) && (ldc % 4 == 0) && (ldcc % 4 == 0) &&
                      (((uintptr_t)Ct | (uintptr_t)C) & 15u) == 0;
@@ -227,7 +558,7 @@ decode_mat_kernel(const CodeParams cp, const __grid_constant__ DecodePlan plan, 
     const int64_t total = L * nw;
     int M[EMAX];
 #pragma unroll
-    for (int c = 0; c < EMAX; ++c) M[c] = c < e ? sh.M[c] : 0;
+    for (int c = 0; c < EMAX; ++c) M[c] = c < e ? Mo[c] : 0;
     for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < total;
          it += (int64_t)gridDim.x * blockDim.x) {
         const int64_t r = it / nw;
@@ -236,7 +567,7 @@ decode_mat_kernel(const CodeParams cp, const __grid_constant__ DecodePlan plan, 
 #pragma unroll
         for (int c = 0; c < EMAX; ++c) acc[c] = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int p = 0; p < k; ++p) {
-            const int s = sh.S[p];
+            const int s = S[p];
             const float *src = Ct + ((int64_t)s * L + r) * ldc + col;
             float4 v;
             if (vec) {
@@ -255,7 +586,7 @@ decode_mat_kernel(const CodeParams cp, const __grid_constant__ DecodePlan plan, 
 #pragma unroll
             for (int c = 0; c < EMAX; ++c) {
                 if (c < e) {
-                    const float w = sh.Dh[c][p];
+                    const float w = Dh[c][p];
                     acc[c].x = fmaf(w, v.x, acc[c].x);
                     acc[c].y = fmaf(w, v.y, acc[c].y);
                     acc[c].z = fmaf(w, v.z, acc[c].z);
@@ -287,97 +618,42 @@ int grid_for(int64_t items, int per_sm)
     return (int)g;
 }
 
-// The decode of `survivors` (host, fp64): the survivor lists, then
-// Gauss-Jordan on [Q | I], Q = P[Ps][M] (e x e), fraction-free (a non-pivot
-// row becomes piv W[a] - W[a][col] W[col], two separately rounded products),
-// with partial pivoting on the fp32 image of |W[a][col]| (lowest index on
-// ties) and one division per row at the end: Q^-1[c][a] = W[c][e+a] / W[c][c].
-// G_S counts as singular when a pivot is zero or not finite, or when
-// ||Q||_inf ||Q^-1||_inf, bounded by ||Q||_inf e max|Q^-1|, exceeds
-// 1 / (64 eps).  Host code is compiled without floating-point contraction, so
-// the plan is the same on every host.
-void plan_decode(const CodeParams &cp, uint32_t survivors, DecodePlan &pl)
+// Missing systematic blocks of a survivor mask (its first k set bits).
+int missing_blocks(int k, uint32_t survivors)
 {
-    const int n = cp.n, k = cp.k;
-    int Ps[kMaxE];
-    int ns = 0, e = 0, np = 0;
-    for (int j = 0; j < n && ns < k; ++j)
-        if ((survivors >> j) & 1u) {
-            pl.S[ns++] = j;
-            if (j >= k) Ps[np++] = j;
-        }
-    for (int i = 0; i < k; ++i) {
-        bool in = false;
-        for (int p = 0; p < ns; ++p) in = in || pl.S[p] == i;
-        if (!in) pl.M[e++] = i;
-    }
-    pl.e = e;
-    pl.singular = 0;
-    if (e == 0) return;
-    double W[kMaxE][2 * kMaxE];
-    double qnorm = 0.0;
-    for (int a = 0; a < e; ++a) {
-        double row = 0.0;
-        for (int c = 0; c < e; ++c) {
-            W[a][c] = (double)cp.P[(Ps[a] - k) * k + pl.M[c]];
-            row += std::fabs(W[a][c]);
-        }
-        for (int c = 0; c < e; ++c) W[a][e + c] = a == c ? 1.0 : 0.0;
-        qnorm = std::max(qnorm, row);
-    }
-    for (int col = 0; col < e; ++col) {
-        int bi = col;
-        float best = -1.f;
-        for (int a = col; a < e; ++a) {
-            const float f = (float)std::fabs(W[a][col]);
-            if (f > best) {
-                best = f;
-                bi = a;
-            }
-        }
-        const double piv = W[bi][col];
-        if (!(std::fabs(piv) > 0.0) || !std::isfinite(piv)) {
-            pl.singular = 1;
-            return;
-        }
-        if (bi != col)
-            for (int j = 0; j < 2 * e; ++j) std::swap(W[col][j], W[bi][j]);
-        for (int a = 0; a < e; ++a) {
-            if (a == col) continue;
-            const double fa = W[a][col];
-            for (int j = 0; j < 2 * e; ++j) {
-                const double p1 = piv * W[a][j], p2 = fa * W[col][j];
-                W[a][j] = j == col ? 0.0 : p1 - p2;
-            }
-        }
-    }
-    double Qi[kMaxE][kMaxE], qimax = 0.0;
-    for (int c = 0; c < e; ++c) {
-        const double dinv = 1.0 / W[c][c];
-        for (int a = 0; a < e; ++a) {
-            Qi[c][a] = W[c][e + a] * dinv;
-            qimax = std::max(qimax, std::fabs(Qi[c][a]));
-        }
-    }
-    if (!(qnorm * qimax * e < 1.0 / (64.0 * DBL_EPSILON))) {
-        pl.singular = 1;
-        return;
-    }
-    for (int c = 0; c < e; ++c)
-        for (int p = 0; p < k; ++p) {
-            const int sp = pl.S[p];
-            double v = 0.0;
-            if (sp >= k) {
-                for (int a = 0; a < e; ++a)
-                    if (Ps[a] == sp) v = Qi[c][a];
-            } else {
-                for (int a = 0; a < e; ++a)
-                    v = std::fma(-Qi[c][a], (double)cp.P[(Ps[a] - k) * k + sp], v);
-            }
-            const float h = (float)v;
-            pl.Dh[c][p] = h;
-            pl.Dl[c][p] = (float)(v - (double)h);
-        }
+    const uint32_t sys = k < 32 ? survivors & ((1u << k) - 1u) : survivors;
+    return k - __builtin_popcount(sys);
+}
+
+// Launches the plan kernel into the next slot of the ring.
+cudaError_t launch_plan(const CodeParams &cp, uint32_t survivors, cudaStream_t s,
+                        DecodeRows **rows)
+{
+    void *base = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&base, g_decode_rows);
+    if (e != cudaSuccess) return e;
+    *rows = static_cast<DecodeRows *>(base) +
+            g_next_rows.fetch_add(1, std::memory_order_relaxed) % kPlanSlots;
+    plan_kernel<<<1, kPlanThreads, 0, s>>>(cp, survivors, *rows);
+    return cudaGetLastError();
+}
+
+// Launch behind the plan kernel as a programmatic dependent launch.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_behind_plan(void (*kern)(KArgs...), unsigned grid, cudaStream_t s,
+                               Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
 }  // namespace
@@ -387,12 +663,12 @@ cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survi
                           cudaStream_t s)
 {
     DecodeArgs a;
-    std::memset(&a.plan, 0, sizeof(a.plan));
-    plan_decode(cp, survivors, a.plan);
     a.L = cp.L;
     a.m = cp.m;
     a.k = cp.k;
     a.b = b;
+    a.survivors = survivors;
+    a.rows = nullptr;
     a.Yt = Yt;
     a.Y = Y;
     a.status = status;
@@ -401,33 +677,44 @@ cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survi
     a.eta = eta;
     // CTAs per role, capped (threads then loop) so the grid stays well inside
     // the launch limit for any block size
+    const int e = missing_blocks(cp.k, survivors), ngroups = (e + CG - 1) / CG;
     const int64_t per_block = cp.L * (int64_t)b;
     const int64_t cap = 1 << 20;
-    const int e = a.plan.e, ngroups = (e + CG - 1) / CG;
     a.dec_per_group = (int32_t)std::min(cap, (per_block + kThreads - 1) / kThreads);
-    a.dec_ctas = a.plan.singular ? 1 : ngroups * a.dec_per_group;
+    a.dec_ctas = ngroups * a.dec_per_group;
     a.pass_per_block = (int32_t)std::min(
         cap, (per_block + kThreads * kPassItems - 1) / (kThreads * kPassItems));
     const int64_t grid = a.dec_ctas + (int64_t)(cp.k - e) * a.pass_per_block;
     if (grid < 1) return cudaSuccess;
-    decode_kernel<<<(unsigned)grid, kThreads, 0, s>>>(a);
-    return cudaGetLastError();
+    if (e == 0) {   // nothing to invert: the pass-through alone
+        decode_kernel<<<(unsigned)grid, kThreads, 0, s>>>(a);
+        return cudaGetLastError();
+    }
+    DecodeRows *rows = nullptr;
+    cudaError_t err = launch_plan(cp, survivors, s, &rows);
+    if (err != cudaSuccess) return err;
+    a.rows = rows;
+    return launch_behind_plan(decode_kernel, (unsigned)grid, s, a);
 }
 
 cudaError_t launch_decode_mat(const CodeParams &cp, const float *Ct, int64_t ldc,
                               uint32_t survivors, int N, float *C, int64_t ldcc, int32_t *status,
                               cudaStream_t s)
 {
-    DecodePlan plan;
-    std::memset(&plan, 0, sizeof(plan));
-    plan_decode(cp, survivors, plan);
+    const int e = missing_blocks(cp.k, survivors);
+    DecodeRows *rows = nullptr;
+    cudaError_t err = launch_plan(cp, survivors, s, &rows);
+    if (err != cudaSuccess) return err;
     const int64_t items = cp.L * (int64_t)N / 4 + 1;
-    const int g = grid_for(items, 8);
-    if (plan.e <= 4)
-        decode_mat_kernel<4><<<g, kThreads, 0, s>>>(cp, plan, Ct, ldc, N, C, ldcc, status);
-    else if (plan.e <= 8)
-        decode_mat_kernel<8><<<g, kThreads, 0, s>>>(cp, plan, Ct, ldc, N, C, ldcc, status);
-    else
-        decode_mat_kernel<16><<<g, kThreads, 0, s>>>(cp, plan, Ct, ldc, N, C, ldcc, status);
-    return cudaGetLastError();
+    const unsigned g = (unsigned)grid_for(items, 8);
+    const int32_t k = cp.k;
+    const int64_t L = cp.L, m = cp.m;
+    if (e <= 4)
+        return launch_behind_plan(decode_mat_kernel<4>, g, s, k, L, m, survivors,
+                                  (const DecodeRows *)rows, Ct, ldc, N, C, ldcc, status);
+    if (e <= 8)
+        return launch_behind_plan(decode_mat_kernel<8>, g, s, k, L, m, survivors,
+                                  (const DecodeRows *)rows, Ct, ldc, N, C, ldcc, status);
+    return launch_behind_plan(decode_mat_kernel<16>, g, s, k, L, m, survivors,
+                              (const DecodeRows *)rows, Ct, ldc, N, C, ldcc, status);
 }

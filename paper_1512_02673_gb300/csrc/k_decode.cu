@@ -58,12 +58,12 @@ struct DecodePlan {
     double piv[kMaxE];       // that pivot's value
     float qmax;              // max |Q| (bounds ||Q||_inf by e max|Q|)
     unsigned long long qimax;   // max |Q^-1| as a magnitude key
-    // [Q | I | P_K] column-major, W[buf][column][row], ping-pong; P_K holds
-    // P[Ps][s] for the surviving systematic workers s
-    double W[2][kMaxE + CM_MAX_N][kMaxE];
-    double rcp[kMaxE];       // 1 / final pivot of each row
-    float Dh[kMaxE][CM_MAX_N];   // D[c][p] (p = position in S), high part
-    float Dl[kMaxE][CM_MAX_N];   // D - Dh
+    float P[CM_MAX_P];               // the parity coefficients ((n - k) x k)
+    double W[2][2 * kMaxE][kMaxE];   // [Q | I] column-major, W[buf][column][row], ping-pong
+    double Pd[kMaxE][CM_MAX_N];      // P[Ps[a]][S[p]] for the surviving systematic S[p]
+    double rcp[kMaxE];               // 1 / final pivot of each row
+    float Dh[kMaxE][CM_MAX_N];       // D[c][p] (p = position in S), high part
+    float Dl[kMaxE][CM_MAX_N];       // D - Dh
 };
 
 // What the apply kernels need of a plan: written by the plan kernel into a
@@ -143,17 +143,20 @@ __device__ __forceinline__ long long mag_key(double v)
 
 constexpr long long kInfKey = 0x7ff0000000000000ll;
 
-// Largest key over the 16 lanes of this half-warp, lowest row on ties; every
-// lane of the half ends with the winner's row.
-__device__ __forceinline__ int half_argmax(long long key, int row)
+// Largest key over an aligned segment of `seg` lanes (a power of two up to
+// 16), lowest row on ties; every lane of the segment ends with the winner's
+// row.  All 32 lanes of the warp take part.
+__device__ __forceinline__ int seg_argmax(long long key, int row, int seg)
 {
 #pragma unroll
     for (int off = 8; off; off >>= 1) {
-        const long long ok = __shfl_xor_sync(0xffffffffu, key, off);
-        const int orow = __shfl_xor_sync(0xffffffffu, row, off);
-        if (ok > key || (ok == key && orow < row)) {
-            key = ok;
-            row = orow;
+        if (off < seg) {
+            const long long ok = __shfl_xor_sync(0xffffffffu, key, off);
+            const int orow = __shfl_xor_sync(0xffffffffu, row, off);
+            if (ok > key || (ok == key && orow < row)) {
+                key = ok;
+                row = orow;
+            }
         }
     }
     return row;
@@ -205,30 +208,45 @@ __device__ __forceinline__ double exact_double(float f)
 //  * Survivor lists by ballots in warp 0: S (the first k set bits), Ps (the
 //    surviving parity workers among them), M (the missing systematic blocks);
 //    the ks = k - e surviving systematic workers are S[0, ks).
-//  * Gauss-Jordan in fp64 on W = [Q | I | P_K], Q = P[Ps][M] (e x e),
-//    P_K = P[Ps][S[0, ks)]; thread t holds entry (row t % 16, column t / 16)
-//    and the one 512 further on.  fp64 latency is long on this part, so the
-//    elimination is fraction-free: at column col with pivot row bi, the pivot
-//    row moves to position col unchanged and every other row r becomes
-//    piv W[r] - W[r][col] W[bi] (two separately rounded products, so
-//    duplicated rows cancel to exactly zero); each row is scaled by its
-//    pivot once at the end, which leaves Q^-1 in the second block and
-//    Q^-1 P_K in the third.  The row swap is part of the update, which reads
-//    one buffer and writes the other: one CTA barrier per column.  The 16
-//    rows of a column sit in one half-warp, which picks the next column's
-//    pivot right after computing it: the largest |W[a][col]|, a >= col
-//    (exact magnitudes compared as integers), lowest row on ties.
+//  * Gauss-Jordan in fp64 on W = [Q | I], Q = P[Ps][M] (e x e).  Thread t
+//    holds entry (row t % E, column t / E), E the power of two at or above
+//    e: the rows of a column are an aligned lane segment and the warps are
+//    dense (the fp64 pipe of this part takes about 19 cycles per warp
+//    instruction, whatever the number of active lanes, and 65 cycles of
+//    latency).  The elimination is fraction-free: at column col with pivot
+//    row bi, the pivot row moves to position col unchanged and every other
+//    row r becomes piv W[r] - W[r][col] W[bi] (two separately rounded
+//    products, so duplicated rows cancel to exactly zero); each row is
+//    scaled by its pivot once at the end: Q^-1[c][a] = W[c][e + a] / W[c][c].
+//    The row swap is part of the update, which reads one buffer and writes
+//    the other: one CTA barrier per column.  The segment of column col + 1
+//    picks that column's pivot right after computing it: the largest
+//    |W[a][col + 1]|, a > col (exact magnitudes compared as integers), lowest
+//    row on ties.
 //  * G_S counts as singular when a pivot is zero or not finite, or when
 //    ||Q||_inf ||Q^-1||_inf, bounded by (e max|Q|) (e max|Q^-1|), exceeds
 //    1 / (64 eps) (evaluated in fp32: it is a threshold).
 //  * D[c][p], the coefficient of the p-th survivor in missing block M[c]:
 //    Q^-1[c][a] for the surviving parity worker Ps[a] = S[ks + a], and
-//    -(Q^-1 P_K)[c][p] for the surviving systematic worker S[p], p < ks;
-//    kept as a (high, low) fp32 pair.
+//    -sum_a Q^-1[c][a] P[Ps[a]][S[p]] for the surviving systematic worker
+//    S[p], p < ks; kept as a (high, low) fp32 pair.
 __device__ void decode_plan(const CodeParams &cp, uint32_t survivors, DecodePlan &pl)
 {
     const int tid = threadIdx.x, lane = tid & 31;
     const int n = cp.n, k = cp.k;
+    {
+        // P into shared memory by warp-uniform reads of the parameter space
+        // (lanes reading different addresses there are served one address at
+        // a time): warp w takes entries [16 w, 16 w + 16)
+        const int w = tid >> 5;
+        float v = 0.f;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const float x = cp.P[(w * 16 + i) & (CM_MAX_P - 1)];
+            if (lane == i) v = x;
+        }
+        if (lane < 16 && w * 16 + lane < CM_MAX_P) pl.P[w * 16 + lane] = v;
+    }
     if (tid < 32) {
         const uint32_t below = (1u << lane) - 1u;
         const bool set = lane < n && ((survivors >> lane) & 1u);
@@ -251,37 +269,30 @@ __device__ void decode_plan(const CodeParams &cp, uint32_t survivors, DecodePlan
     __syncthreads();
     const int e = pl.e, ks = k - e;
     if (e == 0) return;
-    const float *P = cp.P;
-    const int ncol = 2 * e + ks;   // e + k columns
+    const float *P = pl.P;
+    const int lg = 32 - __clz(e - 1);   // E = 1 << lg rows per column
+    const int E = 1 << lg;
+    const int j = tid >> lg, a = tid & (E - 1);
+    const bool live = j < 2 * e && a < e;
     {
-        float q0 = 0.f, qm = 0.f;
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int t = tid + u * kPlanThreads;
-            const int j = t >> 4, a = t & 15;
-            if (j < ncol && a < e) {
-                double w;
-                if (j < e) {
-                    const float q = P[(pl.Ps[a] - k) * k + pl.M[j]];
-                    w = exact_double(q);
-                    qm = fmaxf(qm, fabsf(q));
-                    if (j == 0) q0 = q;
-                } else if (j < 2 * e) {
-                    w = j - e == a ? 1.0 : 0.0;
-                } else {
-                    w = exact_double(P[(pl.Ps[a] - k) * k + pl.S[j - 2 * e]]);
-                }
-                pl.W[0][j][a] = w;
-            }
+        // [Q | I] into buffer 0, max |Q|, the pivot of column 0 (exact: the
+        // fp64 entries are the fp32 values of P), P at the surviving
+        // systematic columns
+        float q = 0.f;
+        if (live) {
+            if (j < e) q = P[(pl.Ps[a] - k) * k + pl.M[j]];
+            pl.W[0][j][a] = j < e ? exact_double(q) : (j - e == a ? 1.0 : 0.0);
         }
-        // pivot of column 0 (half-warp 0): the fp64 entries are the fp32 values
-        const int a = tid & 15;
-        const int b0 = half_argmax(tid < 16 && a < e ? (long long)__float_as_int(fabsf(q0)) : -1ll, a);
-        if (tid == 0) {
+        const int b0 = seg_argmax(j == 0 && a < e ? (long long)__float_as_int(fabsf(q)) : -1ll, a, E);
+        if (tid == b0 && j == 0) {
             pl.bi[0] = b0;
-            pl.piv[0] = exact_double(P[(pl.Ps[b0] - k) * k + pl.M[0]]);
+            pl.piv[0] = exact_double(q);
         }
-        cta_max(qm, &pl.qmax);
+        if (tid < e * ks) {
+            const int pa = tid / ks, pp = tid - pa * ks;
+            pl.Pd[pa][pp] = exact_double(P[(pl.Ps[pa] - k) * k + pl.S[pp]]);
+        }
+        cta_max(live && j < e ? fabsf(q) : 0.f, &pl.qmax);
     }
     __syncthreads();
     for (int col = 0; col < e; ++col) {
@@ -295,28 +306,23 @@ __device__ void decode_plan(const CodeParams &cp, uint32_t survivors, DecodePlan
             __syncthreads();
             return;
         }
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int t = tid + u * kPlanThreads;
-            const int j = t >> 4, a = t & 15;
-            double nv = 0.0;
-            if (j < ncol && a < e) {
-                if (a == col) {
-                    nv = pl.W[cur][j][bi];
-                } else if (j != col) {
-                    const int r = a == bi ? col : a;
-                    nv = __dsub_rn(__dmul_rn(piv, pl.W[cur][j][r]),
-                                   __dmul_rn(pl.W[cur][col][r], pl.W[cur][j][bi]));
-                }
-                pl.W[nxt][j][a] = nv;
+        double nv = 0.0;
+        if (live) {
+            if (a == col) {
+                nv = pl.W[cur][j][bi];
+            } else if (j != col) {
+                const int r = a == bi ? col : a;
+                nv = __dsub_rn(__dmul_rn(piv, pl.W[cur][j][r]),
+                               __dmul_rn(pl.W[cur][col][r], pl.W[cur][j][bi]));
             }
-            if (u == 0 && col + 1 < e) {   // the half-warp of column col + 1 picks its pivot
-                const bool cand = j == col + 1 && a > col && a < e;
-                const int nb = half_argmax(cand ? mag_key(nv) : -1ll, a);
-                if (j == col + 1 && a == nb) {
-                    pl.bi[col + 1] = nb;
-                    pl.piv[col + 1] = nv;
-                }
+            pl.W[nxt][j][a] = nv;
+        }
+        if (col + 1 < e) {   // the segment of column col + 1 picks its pivot
+            const bool cand = j == col + 1 && a > col && a < e;
+            const int nb = seg_argmax(cand ? mag_key(nv) : -1ll, a, E);
+            if (j == col + 1 && a == nb) {
+                pl.bi[col + 1] = nb;
+                pl.piv[col + 1] = nv;
             }
         }
         __syncthreads();
@@ -324,7 +330,7 @@ __device__ void decode_plan(const CodeParams &cp, uint32_t survivors, DecodePlan
     const int fin = e & 1;
     if (tid < e) pl.rcp[tid] = 1.0 / pl.W[fin][tid][tid];
     __syncthreads();
-    // D rows (one entry per thread): scaled entries of the last two blocks
+    // D rows, one entry per thread; the dot products run as two chains
     long long qk = 0;
     if (tid < e * k) {
         const int c = tid / k, p = tid - c * k;
@@ -333,7 +339,13 @@ __device__ void decode_plan(const CodeParams &cp, uint32_t survivors, DecodePlan
             v = __dmul_rn(pl.W[fin][e + (p - ks)][c], pl.rcp[c]);
             qk = mag_key(v);
         } else {
-            v = -__dmul_rn(pl.W[fin][2 * e + p][c], pl.rcp[c]);
+            double s0 = 0.0, s1 = 0.0;
+            for (int aa = 0; aa + 1 < e; aa += 2) {
+                s0 = fma(pl.W[fin][e + aa][c], pl.Pd[aa][p], s0);
+                s1 = fma(pl.W[fin][e + aa + 1][c], pl.Pd[aa + 1][p], s1);
+            }
+            if (e & 1) s0 = fma(pl.W[fin][2 * e - 1][c], pl.Pd[e - 1][p], s0);
+            v = -__dmul_rn(__dadd_rn(s0, s1), pl.rcp[c]);
         }
         float h, l;
         split_double(v, h, l);

@@ -182,6 +182,19 @@ __device__ __forceinline__ void cta_max_key(long long v, unsigned long long *dst
     if ((threadIdx.x & 31) == 0 && v > 0) atomicMax(dst, (unsigned long long)v);
 }
 
+// x 2^-s for a power-of-two scale, exact, by bit manipulation of the
+// exponent (no fp64 instruction); zero, subnormal and underflowing values
+// give a zero of the same sign (they are below 2^-1022 and only ever meet
+// entries of order one).
+__device__ __forceinline__ double scale_pow2(double x, int s)
+{
+    const long long b = __double_as_longlong(x);
+    const int ex = (int)((b >> 52) & 0x7FF);
+    const long long sign = b & (long long)0x8000000000000000ull;
+    if (ex == 0 || ex - s <= 0) return __longlong_as_double(sign);
+    return __longlong_as_double((b & ~(0x7FFll << 52)) | ((long long)(ex - s) << 52));
+}
+
 // fp64 value of an fp32 value by bit manipulation (exact; no fp64
 // instruction: single fp64 operations have a long latency on this part).
 __device__ __forceinline__ double exact_double(float f)
@@ -215,17 +228,20 @@ __device__ __forceinline__ double exact_double(float f)
 //    instruction, whatever the number of active lanes, and 65 cycles of
 //    latency).  The elimination is fraction-free: at column col with pivot
 //    row bi, the pivot row moves to position col unchanged and every other
-//    row r becomes piv W[r] - W[r][col] W[bi] (two separately rounded
-//    products, so duplicated rows cancel to exactly zero); each row is
-//    scaled by its pivot once at the end: Q^-1[c][a] = W[c][e + a] / W[c][c].
+//    row r becomes 2^-s (piv W[r] - W[r][col] W[bi]), 2^s the binade of piv
+//    (two separately rounded products, so duplicated rows cancel to exactly
+//    zero; the exact power-of-two scale keeps the rows from growing by a
+//    product of pivots, which overflows fp64 past about ten columns); each
+//    row is scaled by its pivot once at the end:
+//    Q^-1[c][a] = W[c][e + a] / W[c][c].
 //    The row swap is part of the update, which reads one buffer and writes
 //    the other: one CTA barrier per column.  The segment of column col + 1
 //    picks that column's pivot right after computing it: the largest
 //    |W[a][col + 1]|, a > col (exact magnitudes compared as integers), lowest
 //    row on ties.
-//  * G_S counts as singular when a pivot is zero or not finite, or when
-//    ||Q||_inf ||Q^-1||_inf, bounded by (e max|Q|) (e max|Q^-1|), exceeds
-//    1 / (64 eps) (evaluated in fp32: it is a threshold).
+//  * G_S counts as singular when a pivot is zero, subnormal or not finite,
+//    or when ||Q||_inf ||Q^-1||_inf, bounded by (e max|Q|) (e max|Q^-1|),
+//    exceeds 1 / (64 eps) (evaluated in fp32: it is a threshold).
 //  * D[c][p], the coefficient of the p-th survivor in missing block M[c]:
 //    Q^-1[c][a] for the surviving parity worker Ps[a] = S[ks + a], and
 //    -sum_a Q^-1[c][a] P[Ps[a]][S[p]] for the surviving systematic worker
@@ -298,14 +314,19 @@ __device__ void decode_plan(const CodeParams &cp, uint32_t survivors, DecodePlan
     for (int col = 0; col < e; ++col) {
         const int cur = col & 1, nxt = cur ^ 1;
         const int bi = pl.bi[col];
-        const double piv = pl.piv[col];
-        const long long pk = mag_key(piv);
-        if (pk == 0 || pk >= kInfKey) {   // zero, infinite or not a number
+        const long long pk = mag_key(pl.piv[col]);
+        if (pk < (1ll << 52) || pk >= kInfKey) {   // zero, subnormal, infinite or not a number
             __syncthreads();
             if (tid == 0) pl.singular = 1;
             __syncthreads();
             return;
         }
+        // the update is scaled by 2^-s, 2^s the pivot's binade: the pivot
+        // factor becomes piv 2^-s in [1, 2) and W[r][col] is scaled alike
+        // (exact), so rows grow as in Gauss-Jordan with division rather
+        // than by a product of pivots per column
+        const int sc = (int)(pk >> 52) - 1023;
+        const double piv = scale_pow2(pl.piv[col], sc);
         double nv = 0.0;
         if (live) {
             if (a == col) {
@@ -313,7 +334,7 @@ __device__ void decode_plan(const CodeParams &cp, uint32_t survivors, DecodePlan
             } else if (j != col) {
                 const int r = a == bi ? col : a;
                 nv = __dsub_rn(__dmul_rn(piv, pl.W[cur][j][r]),
-                               __dmul_rn(pl.W[cur][col][r], pl.W[cur][j][bi]));
+                               __dmul_rn(scale_pow2(pl.W[cur][col][r], sc), pl.W[cur][j][bi]));
             }
             pl.W[nxt][j][a] = nv;
         }

@@ -188,3 +188,24 @@ def test_coded_gemm_writes_every_row_and_nothing_else(cm, orc, n, k, m, d, N):
     for j in range(n):
         err = rel_cols(got[j * L:(j + 1) * L], want[j * L:(j + 1) * L])
         assert err.max() <= worker_tol(d), (j, err.max())
+
+
+@pytest.mark.parametrize("n,k,e", [(32, 16, 16), (20, 10, 9)])
+def test_decode_mat_many_missing_blocks(cm, orc, n, k, e):
+    """Matrix decode with up to 16 missing blocks against the oracle's fp64
+    decode of the same fp32 results.  The coefficients are applied in fp32:
+    the tolerance grows with the condition number of the e x e block."""
+    m, N = 23 * k + 3, 40
+    P = synth.parity_coefficients(n, k)
+    code = cm.Code(n, k, m, 64, P, dtype="bf16")
+    L = code.L
+    Ct = synth.gaussian((n * L, N), 31).to(DEV)
+    mask = ((1 << (k - e)) - 1) | (((1 << e) - 1) << k)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    C = cm.decode_mat(code, Ct, mask, status=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    want = orc.decode(n, k, m, P.astype(np.float64), mask, Ct.double().cpu().numpy())
+    Q = P.astype(np.float64)[:e, k - e:]      # parity rows 0..e-1, missing columns k-e..k-1
+    tol = max(1e-5, 100 * np.linalg.cond(Q) * U32)
+    assert rel_cols(C.double().cpu().numpy(), want).max() <= tol

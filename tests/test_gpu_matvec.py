@@ -194,6 +194,42 @@ def test_decode_from_every_k_subset(cm, orc):
             assert err.max() <= 1e-4, (S, err)
 
 
+def _masks_with_e_missing(n, k, e, seed):
+    """Two survivor masks with exactly e missing systematic blocks: the last
+    e systematic and the first e parity workers, and a seeded scatter."""
+    masks = [((1 << (k - e)) - 1) | (((1 << e) - 1) << k)]
+    rng = np.random.default_rng(seed)
+    miss = rng.choice(k, e, replace=False)
+    keep = rng.choice(np.arange(k, n), e, replace=False)
+    masks.append(sum(1 << j for j in range(k) if j not in miss) + sum(1 << int(j) for j in keep))
+    return masks
+
+
+@pytest.mark.parametrize("n,k,e", [(32, 24, 8), (32, 16, 9), (20, 10, 10), (26, 13, 12),
+                                   (32, 16, 16)])
+def test_decode_many_missing_blocks(cm, orc, n, k, e):
+    """Large erasure counts (up to 16 rows of the inverse per column
+    segment): the GPU decode of the GPU's worker results against the
+    oracle's fp64 decode of the same results.  Both solve G_S exactly up to
+    rounding, so they agree to the fp32 output rounding."""
+    m, d, b = 37 * k + 5, 96, 3
+    P = synth.parity_coefficients(n, k)
+    code = cm.Code(n, k, m, d, P)
+    A = synth.gaussian((m, d), 21).to(DEV)
+    X = synth.gaussian((d, b), 22).to(DEV)
+    par = cm.encode(code, A)
+    Yt = cm.matvec(code, A, par, X)
+    for mask in _masks_with_e_missing(n, k, e, seed=n * 100 + e):
+        assert bin(mask).count("1") == k
+        status = torch.zeros(1, dtype=torch.int32, device=DEV)
+        Y = cm.decode(code, Yt, mask, status=status)
+        torch.cuda.synchronize()
+        assert status.item() == 0
+        want = orc.decode(n, k, m, P.astype(np.float64), mask, Yt.cpu().numpy())
+        err = rel_l2_cols(Y.cpu().numpy(), want)
+        assert err.max() <= 1e-6, (hex(mask), err)
+
+
 def test_extra_survivors_use_the_lowest_k(cm, orc):
     n, k, m, d = 10, 5, 400, 128
     r = run_path(cm, orc, n, k, m, d, 1)

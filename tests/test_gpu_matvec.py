@@ -230,6 +230,31 @@ def test_decode_many_missing_blocks(cm, orc, n, k, e):
         assert err.max() <= 1e-6, (hex(mask), err)
 
 
+def test_pass_through_is_rounded_to_nearest(cm):
+    """Surviving systematic blocks are the fp64 results rounded to fp32 (to
+    nearest, ties to even; the kernels convert by integer arithmetic): bit
+    for bit equal to the device's own conversion, on values that include
+    ties, fp32 subnormals, underflow to zero, overflow and signed zeros."""
+    n, k, m = 6, 3, 3000
+    code = cm.Code(n, k, m, 16, synth.parity_coefficients(n, k))
+    L = code.L
+    rng = np.random.default_rng(4)
+    y = rng.standard_normal(n * L) * np.exp2(rng.integers(-160, 140, n * L))
+    # exact ties: the 29 bits below the fp32 mantissa are 1000...0
+    bits = y[:400].view(np.uint64)
+    bits &= ~np.uint64((1 << 29) - 1)
+    bits |= np.uint64(1 << 28)
+    special = np.array([0.0, -0.0, 1e-40, -1e-40, 1e-46, 3e-45, 7e-46, 1.4e-45, 1e39, -1e39,
+                        3.4028235677973366e38, 3.4028234663852886e38, np.inf, -np.inf,
+                        1.1754942e-38, 5.877471754111438e-39, 1.0 + 2.0 ** -24, 1.0 + 3 * 2.0 ** -24])
+    y[400:400 + len(special)] = special
+    Yt = torch.from_numpy(y.reshape(n * L, 1)).to(DEV)
+    Y = cm.decode(code, Yt, (1 << k) - 1)          # every systematic block survives
+    torch.cuda.synchronize()
+    want = Yt[:m].float()
+    assert torch.equal(Y.view(torch.int32), want.view(torch.int32))
+
+
 def test_extra_survivors_use_the_lowest_k(cm, orc):
     n, k, m, d = 10, 5, 400, 128
     r = run_path(cm, orc, n, k, m, d, 1)

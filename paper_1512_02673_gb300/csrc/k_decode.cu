@@ -589,6 +589,8 @@ decode_mat_kernel(int32_t k, int64_t L, int64_t m, uint32_t survivors, const Dec
     const int W = vec ? 4 : 1;
     const int64_t nw = N / W;
     const int64_t total = L * nw;
+    // survivors whose loads are issued together (fewer with more accumulators)
+    constexpr int kBatch = EMAX <= 8 ? 4 : 2;
     int M[EMAX];
 #pragma unroll
     for (int c = 0; c < EMAX; ++c) M[c] = c < e ? Mo[c] : 0;
@@ -599,31 +601,39 @@ decode_mat_kernel(int32_t k, int64_t L, int64_t m, uint32_t survivors, const Dec
         float4 acc[EMAX];
 #pragma unroll
         for (int c = 0; c < EMAX; ++c) acc[c] = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int p = 0; p < k; ++p) {
-            const int s = S[p];
-            const float *src = Ct + ((int64_t)s * L + r) * ldc + col;
-            float4 v;
-            if (vec) {
-                v = __ldg(reinterpret_cast<const float4 *>(src));
-            } else {
-                v = make_float4(__ldg(src), 0.f, 0.f, 0.f);
-            }
-            if (!inplace && s < k) {   // surviving systematic block passes through
-                const int64_t g = (int64_t)s * L + r;
-                if (g < m) {
-                    float *dst = C + g * ldcc + col;
-                    if (vec) *reinterpret_cast<float4 *>(dst) = v;
-                    else *dst = v.x;
+        // survivors in batches of kBatch: their loads are issued together
+        for (int p0 = 0; p0 < k; p0 += kBatch) {
+            float4 v[kBatch];
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u) {
+                if (p0 + u < k) {
+                    const float *src = Ct + ((int64_t)S[p0 + u] * L + r) * ldc + col;
+                    v[u] = vec ? __ldg(reinterpret_cast<const float4 *>(src))
+                               : make_float4(__ldg(src), 0.f, 0.f, 0.f);
                 }
             }
 #pragma unroll
-            for (int c = 0; c < EMAX; ++c) {
-                if (c < e) {
-                    const float w = Dh[c][p];
-                    acc[c].x = fmaf(w, v.x, acc[c].x);
-                    acc[c].y = fmaf(w, v.y, acc[c].y);
-                    acc[c].z = fmaf(w, v.z, acc[c].z);
-                    acc[c].w = fmaf(w, v.w, acc[c].w);
+            for (int u = 0; u < kBatch; ++u) {
+                const int p = p0 + u;
+                if (p >= k) break;
+                const int s = S[p];
+                if (!inplace && s < k) {   // surviving systematic block passes through
+                    const int64_t g = (int64_t)s * L + r;
+                    if (g < m) {
+                        float *dst = C + g * ldcc + col;
+                        if (vec) *reinterpret_cast<float4 *>(dst) = v[u];
+                        else *dst = v[u].x;
+                    }
+                }
+#pragma unroll
+                for (int c = 0; c < EMAX; ++c) {
+                    if (c < e) {
+                        const float w = Dh[c][p];
+                        acc[c].x = fmaf(w, v[u].x, acc[c].x);
+                        acc[c].y = fmaf(w, v[u].y, acc[c].y);
+                        acc[c].z = fmaf(w, v[u].z, acc[c].z);
+                        acc[c].w = fmaf(w, v[u].w, acc[c].w);
+                    }
                 }
             }
         }

@@ -32,9 +32,12 @@
 //
 // One persistent CTA per SM, warp-specialised, in both CTAs of a pair:
 //   warp 0 lane 0  TMA producer of the CTA's halves (128B-swizzled 128 x 64
-//                  boxes) into a 6-stage ring; every load completes on the
-//                  leader CTA's stage barrier, which the leader's producer
-//                  arms with the bytes of both CTAs;
+//                  boxes) into a 6-stage ring whose stages are guarded in
+//                  pairs (one full and one empty barrier per 2 K blocks: half
+//                  the barrier round trips, +1 %; three per barrier left two
+//                  groups and ran 10 % slower); every load completes on the
+//                  leader CTA's barrier, which the leader's producer arms
+//                  with the bytes of both CTAs;
 //   warp 1         allocates 512 TMEM columns together with the peer
 //                  (cta_group::2: two 128 x 256 fp32 accumulators per CTA);
 //                  in the leader (rank 0), lane 0 issues the MMAs and
@@ -57,6 +60,8 @@ namespace {
 
 constexpr int BM = 128;              // rows per CTA (256 per pair)
 constexpr int BN = 256, BK = 64, STAGES = 6, ACCS = 2;
+constexpr int KG = 2;                 // K blocks per barrier
+constexpr int GROUPS = STAGES / KG;   // barrier groups in the ring
 constexpr int BNH = BN / 2;          // Bt rows staged per CTA
 constexpr int TMEM_COLS = ACCS * BN;   // 512
 constexpr int kThreads = 192;
@@ -252,7 +257,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
     const int rank = (int)cluster_ctarank();
     const bool leader = rank == 0;
     if (threadIdx.x == 0) {
-        for (int s = 0; s < STAGES; ++s) {
+        for (int s = 0; s < GROUPS; ++s) {
             cm_mbar_init(&full[s], 1);    // leader: its producer's arrive (+ both CTAs' bytes)
             cm_mbar_init(&empty[s], 1);   // the leader's MMA commit
         }
@@ -291,18 +296,21 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
         for (int64_t p = first; p < g.pairs && !*abort_flag; p += stride) {
             const Tile x = tile_of(g, p, rank);
             const CUtensorMap *ma = x.parity ? &tmP : &tmA;
-            for (int kb = 0; kb < g.kblocks; ++kb) {
+            for (int kb = 0; kb < g.kblocks; kb += KG) {
                 if (*abort_flag || !cm_mbar_wait(&empty[s], ph ^ 1u)) {
                     fail();
                     break;
                 }
-                unsigned char *sa = base + s * STAGE_BYTES;
+                const int nb = g.kblocks - kb < KG ? g.kblocks - kb : KG;
                 const uint32_t bar = map_to_rank(&full[s], 0);   // the leader's stage barrier
-                if (leader) cm_mbar_arrive_expect_tx(&full[s], 2 * STAGE_BYTES);
-                tma_load_2d_pair(sa, ma, kb * BK, x.y, bar);
-                tma_load_2d_pair(sa + A_BYTES, &tmB, kb * BK, x.n0 + rank * BNH, bar);
+                if (leader) cm_mbar_arrive_expect_tx(&full[s], 2 * STAGE_BYTES * nb);
+                for (int u = 0; u < nb; ++u) {
+                    unsigned char *sa = base + (s * KG + u) * STAGE_BYTES;
+                    tma_load_2d_pair(sa, ma, (kb + u) * BK, x.y, bar);
+                    tma_load_2d_pair(sa + A_BYTES, &tmB, (kb + u) * BK, x.n0 + rank * BNH, bar);
+                }
                 ++issued;
-                if (++s == STAGES) {
+                if (++s == GROUPS) {
                     s = 0;
                     ph ^= 1u;
                 }
@@ -310,9 +318,9 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
         }
         if (*abort_flag && leader) {
             // drain: wait (bounded) for the last phase of every stage in flight
-            for (int i = 0; i < STAGES && i < issued; ++i) {
+            for (int i = 0; i < GROUPS && i < issued; ++i) {
                 if (--s < 0) {
-                    s = STAGES - 1;
+                    s = GROUPS - 1;
                     ph ^= 1u;
                 }
                 cm_mbar_wait(&full[s], ph, 100000000ull);
@@ -330,21 +338,24 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
             tc_fence_after();
             const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
             bool ok = true;
-            for (int kb = 0; kb < g.kblocks; ++kb) {
+            for (int kb = 0; kb < g.kblocks; kb += KG) {
                 if (*abort_flag || !cm_mbar_wait(&full[s], ph)) {
                     fail();
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                const uint32_t sa = cm_smem_u32(base + s * STAGE_BYTES);
-                const uint32_t sb = sa + A_BYTES;
+                const int nb = g.kblocks - kb < KG ? g.kblocks - kb : KG;
+                for (int u = 0; u < nb; ++u) {
+                    const uint32_t sa = cm_smem_u32(base + (s * KG + u) * STAGE_BYTES);
+                    const uint32_t sb = sa + A_BYTES;
 #pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk)
-                    mma_bf16_pair(d_tmem, smem_desc_sw128(sa + kk * 32),
-                                  smem_desc_sw128(sb + kk * 32), (kb | kk) != 0);
-                mma_commit_pair(&empty[s]);   // the stage is free in both CTAs
-                if (++s == STAGES) {
+                    for (int kk = 0; kk < BK / 16; ++kk)
+                        mma_bf16_pair(d_tmem, smem_desc_sw128(sa + kk * 32),
+                                      smem_desc_sw128(sb + kk * 32), ((kb + u) | kk) != 0);
+                }
+                mma_commit_pair(&empty[s]);   // the group is free in both CTAs
+                if (++s == GROUPS) {
                     s = 0;
                     ph ^= 1u;
                 }

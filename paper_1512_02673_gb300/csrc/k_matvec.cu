@@ -13,8 +13,10 @@
 //
 // Data movement.  The unit's rows stream through a per-warp ring of ST
 // shared-memory slots, one 2-D TMA box (R rows x 128 columns) per step issued
-// by the warp's lane 0 and counted on the slot's mbarrier, so ST steps are in
-// flight per warp without any per-lane copy work.  Lane 0 refills a slot after
+// by the warp's lane 0.  Slots are guarded in pairs: the two boxes of steps
+// (2i, 2i + 1) complete on one mbarrier, so ST steps are in flight per warp
+// without any per-lane copy work and the wait, the refill and the ring
+// bookkeeping come once per two steps.  Lane 0 refills a slot after
 // a __syncwarp that follows every lane's reads of it: the warp barrier orders
 // those reads before the copy is issued, and the slot is only ever written by
 // TMA, so there is no generic-proxy write for a proxy fence to publish (one
@@ -204,11 +206,13 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     float *xs = reinterpret_cast<float *>(base + S::RING_BYTES);
     uint64_t *bars = reinterpret_cast<uint64_t *>(base + S::RING_BYTES + S::X_BYTES);
 
+    static_assert(ST % 2 == 0, "ring slots are guarded in pairs");
+    constexpr int NG = ST / 2;   // slot pairs (barrier groups) per warp
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     float *ring = rings + warp * (ST * S::SLOT_FLOATS);
-    uint64_t *bar = bars + warp * ST;
-    if (threadIdx.x < kWarps * ST) cm_mbar_init(&bars[threadIdx.x], 1);
+    uint64_t *bar = bars + warp * NG;
+    if (threadIdx.x < kWarps * NG) cm_mbar_init(&bars[threadIdx.x], 1);
     cm_fence_mbar_init();
     __syncthreads();
 
@@ -219,37 +223,79 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     const int nchunks = (int)((a.d + C::CX - 1) / C::CX);
     // rounds in which this warp has a unit (a prefix: unit index grows with round)
     const int64_t my_rounds = gw < a.groups ? (a.groups - 1 - gw) / total_warps + 1 : 0;
-    const int64_t my_steps = my_rounds * steps;
+    // A unit's steps go in pairs (0, 1), (2, 3), ... (its last one alone when
+    // the count is odd); a pair fills two ring slots and completes on one
+    // mbarrier, so a wait, a refill and the ring bookkeeping come once per two
+    // 4 KB boxes.  Pairs start at even steps and chunks hold an even number
+    // of steps, so no pair spans two X chunks.
+    const int pairs_per_unit = (steps + 1) / 2;
+    const int64_t my_pairs = my_rounds * pairs_per_unit;
 
-    // ---- producer state (lane 0): next step to load ----
-    int64_t p_idx = 0;
-    int p_slot = 0, p_s = 0, p_round = 0;
+    // ---- producer state (lane 0): next pair to load ----
+    int64_t p_idx = 0;   // pairs issued
+    int p_g = 0, p_s = 0, p_round = 0;
     Unit pu = unit_of(a, gw, R);
-    auto produce = [&]() {   // lane 0 only; loads step p_idx into slot p_slot
-        cm_mbar_arrive_expect_tx(&bar[p_slot], STEP_BYTES);
-        cm_tma_load_2d(ring + p_slot * S::SLOT_FLOATS, pu.parity ? &tmP : &tmA, 128 * p_s, pu.y,
-                       &bar[p_slot]);
+    auto produce = [&]() {   // lane 0 only; loads the next pair into group p_g
+        const int nb = steps - p_s < 2 ? steps - p_s : 2;
+        cm_mbar_arrive_expect_tx(&bar[p_g], nb * STEP_BYTES);
+        for (int u = 0; u < nb; ++u)
+            cm_tma_load_2d(ring + (2 * p_g + u) * S::SLOT_FLOATS, pu.parity ? &tmP : &tmA,
+                           128 * (p_s + u), pu.y, &bar[p_g]);
         ++p_idx;
-        p_slot = p_slot + 1 == ST ? 0 : p_slot + 1;
-        if (++p_s == steps) {
+        p_g = p_g + 1 == NG ? 0 : p_g + 1;
+        p_s += nb;
+        if (p_s == steps) {
             p_s = 0;
             ++p_round;
             pu = unit_of(a, (int64_t)p_round * total_warps + gw, R);
         }
     };
     if (lane == 0)
-        while (p_idx < my_steps && p_idx < ST) produce();
+        while (p_idx < my_pairs && p_idx < NG) produce();
 
     stage_x<BP, XF, kThreads>(a, xs, 0);
 
     // ---- consumer ----
     int xbuf = 0;             // X buffer of the current chunk
-    int64_t c_idx = 0;        // steps of this warp consumed so far
-    int slot = 0;             // ring slot of step c_idx
-    uint32_t phase = 0;       // mbarrier phase parity of that slot's current use
+    int64_t c_idx = 0;        // pairs of this warp consumed so far
+    int grp = 0;              // ring group of pair c_idx
+    uint32_t phase = 0;       // mbarrier phase parity of that group's current use
     bool failed = false;
     float2 acc[V];            // (even-column, odd-column) partial pairs
     double acc64[NH];
+    // one 128-column step: the 4 columns of this lane, R rows, BP vectors
+    auto step = [&](const float *ab, const float *xb) {
+        float2 x01[BP], x23[BP];
+#pragma unroll
+        for (int v = 0; v < BP; ++v) {
+            const float4 xv = *reinterpret_cast<const float4 *>(xb + v * C::GS);
+            x01[v] = make_float2(xv.x, xv.y);
+            x23[v] = make_float2(xv.z, xv.w);
+        }
+        // rows in groups of RH: all even-pair FMAs of the group, then all
+        // odd-pair ones, so two updates of an accumulator sit RH * BP
+        // instructions apart
+        constexpr int RH = R >= 4 ? 4 : R;
+#pragma unroll
+        for (int r0 = 0; r0 < R; r0 += RH) {
+            float4 av[RH];
+#pragma unroll
+            for (int r = 0; r < RH; ++r)
+                av[r] = *reinterpret_cast<const float4 *>(ab + (r0 + r) * 128);
+#pragma unroll
+            for (int r = 0; r < RH; ++r)
+#pragma unroll
+                for (int v = 0; v < BP; ++v)
+                    acc[(r0 + r) * BP + v] = __ffma2_rn(make_float2(av[r].x, av[r].y), x01[v],
+                                                        acc[(r0 + r) * BP + v]);
+#pragma unroll
+            for (int r = 0; r < RH; ++r)
+#pragma unroll
+                for (int v = 0; v < BP; ++v)
+                    acc[(r0 + r) * BP + v] = __ffma2_rn(make_float2(av[r].z, av[r].w), x23[v],
+                                                        acc[(r0 + r) * BP + v]);
+        }
+    };
 #pragma unroll 1
     for (int round = 0; round < rounds; ++round) {
         const bool has = round < my_rounds;
@@ -270,53 +316,25 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
             if (has && !failed) {
                 const float *xchunk = xs + xbuf * C::FLOATS + 4 * lane;
 #pragma unroll
-                for (int cs = 0; cs < IPC; ++cs) {
+                for (int cs = 0; cs < IPC; cs += 2) {
                     if (cs >= ns || failed) break;
-                    if (!cm_mbar_wait(&bar[slot], phase)) {
+                    if (!cm_mbar_wait(&bar[grp], phase)) {
                         failed = true;
                         if (lane == 0 && a.status) *a.status = CM_ETIMEOUT;
                         break;
                     }
-                    const float *xb = xchunk + cs * 128;
-                    const float *ab = ring + slot * S::SLOT_FLOATS + 4 * lane;
-                    float2 x01[BP], x23[BP];
-#pragma unroll
-                    for (int v = 0; v < BP; ++v) {
-                        const float4 xv = *reinterpret_cast<const float4 *>(xb + v * C::GS);
-                        x01[v] = make_float2(xv.x, xv.y);
-                        x23[v] = make_float2(xv.z, xv.w);
-                    }
-                    // rows in groups of RH: all even-pair FMAs of the group, then all
-                    // odd-pair ones, so two updates of an accumulator sit RH * BP
-                    // instructions apart
-                    constexpr int RH = R >= 4 ? 4 : R;
-#pragma unroll
-                    for (int r0 = 0; r0 < R; r0 += RH) {
-                        float4 av[RH];
-#pragma unroll
-                        for (int r = 0; r < RH; ++r)
-                            av[r] = *reinterpret_cast<const float4 *>(ab + (r0 + r) * 128);
-#pragma unroll
-                        for (int r = 0; r < RH; ++r)
-#pragma unroll
-                            for (int v = 0; v < BP; ++v)
-                                acc[(r0 + r) * BP + v] = __ffma2_rn(
-                                    make_float2(av[r].x, av[r].y), x01[v], acc[(r0 + r) * BP + v]);
-#pragma unroll
-                        for (int r = 0; r < RH; ++r)
-#pragma unroll
-                            for (int v = 0; v < BP; ++v)
-                                acc[(r0 + r) * BP + v] = __ffma2_rn(
-                                    make_float2(av[r].z, av[r].w), x23[v], acc[(r0 + r) * BP + v]);
-                    }
+                    const float *ab = ring + 2 * grp * S::SLOT_FLOATS + 4 * lane;
+                    step(ab, xchunk + cs * 128);
+                    if (cs + 1 < ns) step(ab + S::SLOT_FLOATS, xchunk + (cs + 1) * 128);
                     ++c_idx;
-                    if (++slot == ST) {
-                        slot = 0;
+                    if (++grp == NG) {
+                        grp = 0;
                         phase ^= 1u;
                     }
-                    __syncwarp();   // every lane is done reading the slot
-                    if (lane == 0 && p_idx < my_steps) produce();   // refill it
-                    if (++fl == F) {
+                    __syncwarp();   // every lane is done reading the pair
+                    if (lane == 0 && p_idx < my_pairs) produce();   // refill it
+                    fl += cs + 1 < ns ? 2 : 1;
+                    if (fl >= F) {
                         flush_pairs<V>(acc, acc64, lane);
                         fl = 0;
                     }
@@ -349,9 +367,9 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     // the CTA's shared memory is released.
     if (failed && lane == 0) {
         for (int64_t i = c_idx; i < p_idx; ++i) {
-            cm_mbar_wait(&bar[slot], phase, 100000000ull);
-            if (++slot == ST) {
-                slot = 0;
+            cm_mbar_wait(&bar[grp], phase, 100000000ull);
+            if (++grp == NG) {
+                grp = 0;
                 phase ^= 1u;
             }
         }

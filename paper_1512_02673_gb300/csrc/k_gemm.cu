@@ -460,9 +460,6 @@ cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t l
     g.ntiles = (N + BN - 1) / BN;
     g.kblocks = (int)((cp.d + BK - 1) / BK);
     g.pairs = (int64_t)(g.psys + g.ppar) * g.ntiles;
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         SMEM_BYTES);
-    if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -474,15 +471,24 @@ cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t l
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cfg.gridDim = dim3(2 * (unsigned)((cm_sm_count() + 1) / 2));
-    // persistent: as many pairs as can be resident at once
-    int clusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&clusters, gemm_kernel, &cfg);
-    if (e != cudaSuccess) return e;
+    // persistent: as many pairs as can be resident at once (the attribute and
+    // the occupancy query are the same for every call: done once, thread-safe)
+    static const int resident = [&cfg]() -> int {
+        if (cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 SMEM_BYTES) != cudaSuccess)
+            return -1;
+        cudaLaunchConfig_t q = cfg;
+        q.gridDim = dim3(2 * (unsigned)((cm_sm_count() + 1) / 2));
+        int c = 0;
+        if (cudaOccupancyMaxActiveClusters(&c, gemm_kernel, &q) != cudaSuccess) return -1;
+        return c;
+    }();
+    if (resident < 0) return cudaErrorInvalidConfiguration;
+    int clusters = resident;
     if (clusters < 1) return cudaErrorInvalidConfiguration;
     if (clusters > g.pairs) clusters = (int)g.pairs;
     cfg.gridDim = dim3(2 * (unsigned)clusters);
-    e = cudaLaunchKernelEx(&cfg, gemm_kernel, tmA, tmP, tmB, g);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_kernel, tmA, tmP, tmB, g);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

@@ -13,10 +13,11 @@
 //
 // Data movement.  The unit's rows stream through a per-warp ring of ST
 // shared-memory slots, one 2-D TMA box (R rows x 128 columns) per step issued
-// by the warp's lane 0.  Slots are guarded in pairs: the two boxes of steps
-// (2i, 2i + 1) complete on one mbarrier, so ST steps are in flight per warp
+// by the warp's lane 0.  Slots are guarded in groups of GS (2; 4 for the
+// 12-slot ring of 4-row units): the GS boxes of steps (GS i, ..., GS i +
+// GS - 1) complete on one mbarrier, so ST steps are in flight per warp
 // without any per-lane copy work and the wait, the refill and the ring
-// bookkeeping come once per two steps.  Lane 0 refills a slot after
+// bookkeeping come once per GS steps.  Lane 0 refills a slot after
 // a __syncwarp that follows every lane's reads of it: the warp barrier orders
 // those reads before the copy is issued, and the slot is only ever written by
 // TMA, so there is no generic-proxy write for a proxy fence to publish (one
@@ -206,8 +207,11 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     float *xs = reinterpret_cast<float *>(base + S::RING_BYTES);
     uint64_t *bars = reinterpret_cast<uint64_t *>(base + S::RING_BYTES + S::X_BYTES);
 
-    static_assert(ST % 2 == 0, "ring slots are guarded in pairs");
-    constexpr int NG = ST / 2;   // slot pairs (barrier groups) per warp
+    // slots per barrier group: 4 with the 12-slot ring, else 2 (3 groups of 2
+    // for 6 slots; groups of 3 would leave two)
+    constexpr int GS = ST % 4 == 0 && ST >= 12 ? 4 : 2;
+    static_assert(ST % GS == 0 && IPC % GS == 0, "ring slots are guarded in groups");
+    constexpr int NG = ST / GS;   // barrier groups per warp
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     float *ring = rings + warp * (ST * S::SLOT_FLOATS);
@@ -223,23 +227,22 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     const int nchunks = (int)((a.d + C::CX - 1) / C::CX);
     // rounds in which this warp has a unit (a prefix: unit index grows with round)
     const int64_t my_rounds = gw < a.groups ? (a.groups - 1 - gw) / total_warps + 1 : 0;
-    // A unit's steps go in pairs (0, 1), (2, 3), ... (its last one alone when
-    // the count is odd); a pair fills two ring slots and completes on one
-    // mbarrier, so a wait, a refill and the ring bookkeeping come once per two
-    // 4 KB boxes.  Pairs start at even steps and chunks hold an even number
-    // of steps, so no pair spans two X chunks.
-    const int pairs_per_unit = (steps + 1) / 2;
+    // A unit's steps go in groups of GS (the last one shorter when GS does
+    // not divide the count); a group fills GS ring slots and completes on one
+    // mbarrier.  Groups start at multiples of GS and chunks hold a multiple of
+    // GS steps, so no group spans two X chunks.
+    const int pairs_per_unit = (steps + GS - 1) / GS;
     const int64_t my_pairs = my_rounds * pairs_per_unit;
 
-    // ---- producer state (lane 0): next pair to load ----
-    int64_t p_idx = 0;   // pairs issued
+    // ---- producer state (lane 0): next group to load ----
+    int64_t p_idx = 0;   // groups issued
     int p_g = 0, p_s = 0, p_round = 0;
     Unit pu = unit_of(a, gw, R);
-    auto produce = [&]() {   // lane 0 only; loads the next pair into group p_g
-        const int nb = steps - p_s < 2 ? steps - p_s : 2;
+    auto produce = [&]() {   // lane 0 only; loads the next group into ring group p_g
+        const int nb = steps - p_s < GS ? steps - p_s : GS;
         cm_mbar_arrive_expect_tx(&bar[p_g], nb * STEP_BYTES);
         for (int u = 0; u < nb; ++u)
-            cm_tma_load_2d(ring + (2 * p_g + u) * S::SLOT_FLOATS, pu.parity ? &tmP : &tmA,
+            cm_tma_load_2d(ring + (GS * p_g + u) * S::SLOT_FLOATS, pu.parity ? &tmP : &tmA,
                            128 * (p_s + u), pu.y, &bar[p_g]);
         ++p_idx;
         p_g = p_g + 1 == NG ? 0 : p_g + 1;
@@ -257,8 +260,8 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
 
     // ---- consumer ----
     int xbuf = 0;             // X buffer of the current chunk
-    int64_t c_idx = 0;        // pairs of this warp consumed so far
-    int grp = 0;              // ring group of pair c_idx
+    int64_t c_idx = 0;        // groups of this warp consumed so far
+    int grp = 0;              // ring group of group c_idx
     uint32_t phase = 0;       // mbarrier phase parity of that group's current use
     bool failed = false;
     float2 acc[V];            // (even-column, odd-column) partial pairs
@@ -316,24 +319,25 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
             if (has && !failed) {
                 const float *xchunk = xs + xbuf * C::FLOATS + 4 * lane;
 #pragma unroll
-                for (int cs = 0; cs < IPC; cs += 2) {
+                for (int cs = 0; cs < IPC; cs += GS) {
                     if (cs >= ns || failed) break;
                     if (!cm_mbar_wait(&bar[grp], phase)) {
                         failed = true;
                         if (lane == 0 && a.status) *a.status = CM_ETIMEOUT;
                         break;
                     }
-                    const float *ab = ring + 2 * grp * S::SLOT_FLOATS + 4 * lane;
-                    step(ab, xchunk + cs * 128);
-                    if (cs + 1 < ns) step(ab + S::SLOT_FLOATS, xchunk + (cs + 1) * 128);
+                    const float *ab = ring + GS * grp * S::SLOT_FLOATS + 4 * lane;
+#pragma unroll
+                    for (int u = 0; u < GS; ++u)
+                        if (cs + u < ns) step(ab + u * S::SLOT_FLOATS, xchunk + (cs + u) * 128);
                     ++c_idx;
                     if (++grp == NG) {
                         grp = 0;
                         phase ^= 1u;
                     }
-                    __syncwarp();   // every lane is done reading the pair
+                    __syncwarp();   // every lane is done reading the group
                     if (lane == 0 && p_idx < my_pairs) produce();   // refill it
-                    fl += cs + 1 < ns ? 2 : 1;
+                    fl += ns - cs < GS ? ns - cs : GS;
                     if (fl >= F) {
                         flush_pairs<V>(acc, acc64, lane);
                         fl = 0;

@@ -1,4 +1,4 @@
-// K6: coded shuffling data plane (Sec. IV) -- row programs on HBM-resident
+// K7: coded shuffling data plane (Sec. IV) -- row programs on HBM-resident
 // rows.
 //
 // One kernel runs every step of a transition: output row o is

@@ -128,6 +128,35 @@ __global__ void __launch_bounds__(kScanBlock) scan_add_kernel(int32_t *out, int6
         if (base + k < count) out[base + k] += add;
 }
 
+// The second pass when the block sums are few: every block sums the block
+// sums before its own (at most kScanDirect of them, one or a few per thread)
+// instead of waiting for a scan of them in a launch of its own, then adds
+// that offset; the last block also writes the total.
+constexpr int64_t kScanDirect = 4 * kScanBlock;
+
+__global__ void __launch_bounds__(kScanBlock) scan_add_direct_kernel(int32_t *out, int64_t count,
+                                                                     const int32_t *block_sums,
+                                                                     int32_t *total)
+{
+    __shared__ int32_t warp_part[32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int32_t part = 0;
+    for (int64_t i = threadIdx.x; i < (int64_t)blockIdx.x; i += kScanBlock) part += block_sums[i];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+    if (lane == 0) warp_part[warp] = part;
+    __syncthreads();
+    int32_t add = 0;
+#pragma unroll 1
+    for (int w = 0; w < kScanBlock / 32; ++w) add += warp_part[w];
+    const int64_t base = (int64_t)blockIdx.x * kScanItems + 4 * (int64_t)threadIdx.x;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        if (base + k < count) out[base + k] += add;
+    if (total && threadIdx.x == 0 && blockIdx.x == gridDim.x - 1)
+        *total = add + block_sums[blockIdx.x];
+}
+
 int64_t up256(int64_t x) { return (x + 255) & ~(int64_t)255; }
 
 // out[i] = in[0] + ... + in[i-1] for i < count (in may be out); the sum of
@@ -146,6 +175,10 @@ cudaError_t scan_exclusive(const int32_t *in, int32_t *out, int64_t count, int32
         return cudaGetLastError();
     }
     scan_block_kernel<<<(unsigned)nb, kScanBlock, 0, s>>>(in, out, count, scratch);
+    if (nb <= kScanDirect) {
+        scan_add_direct_kernel<<<(unsigned)nb, kScanBlock, 0, s>>>(out, count, scratch, total);
+        return cudaGetLastError();
+    }
     cudaError_t e = scan_exclusive(scratch, scratch, nb, scratch + up256(nb), total, s);
     if (e != cudaSuccess) return e;
     scan_add_kernel<<<(unsigned)nb, kScanBlock, 0, s>>>(out, count, scratch);

@@ -218,6 +218,18 @@ cm_status cm_coded_gemm(const cm_code *code, const void *A, int64_t lda,
                         int32_t N, float *Ct, int64_t ldc, int32_t *dev_status,
                         cm_stream_t stream);
 
+/* The coded matrix-matrix products of the k workers that cm_decode_mat will
+ * read (the first k set bits of `survivors`; for a repetition code the
+ * first survivor of each block), when the stragglers are known before the
+ * products run (Sec. III-A: the master needs only k results).  Arguments
+ * and layout as cm_coded_gemm; the blocks of the other workers in Ct are not
+ * written.  The computed blocks equal cm_coded_gemm's bit for bit.  Returns
+ * CM_ENOTDECODABLE when the survivors cannot be decoded. */
+cm_status cm_coded_gemm_survivors(const cm_code *code, const void *A, int64_t lda,
+                                  const void *parity, int64_t ldp, const void *Bt, int64_t ldb,
+                                  int32_t N, uint32_t survivors, float *Ct, int64_t ldc,
+                                  int32_t *dev_status, cm_stream_t stream);
+
 /* Decoding of matrix results: as cm_decode with b = N columns of fp32
  * stacked results Ct (leading dimension ldc) into C (m x N fp32, leading
  * dimension ldcc).  The decode coefficients are formed in fp64 by the same

@@ -65,6 +65,8 @@ def lib() -> ctypes.CDLL:
             "cm_gd_step_noalloc": (st, [vp, vp, i64, vp, i64, vp, vp, i64, vp, i64, vp, vp,
                                         f32, u32, u32, vp, vp]),
             "cm_coded_gemm": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, vp, vp]),
+            "cm_coded_gemm_survivors": (st, [vp, vp, i64, vp, i64, vp, i64, i32, u32, vp,
+                                             i64, vp, vp]),
             "cm_decode_mat": (st, [vp, vp, i64, u32, i32, vp, i64, vp, vp]),
             "cm_matmat": (st, [vp, vp, i64, vp, i64, vp, i64, i32, vp, i64, u32, vp, i64,
                                vp, vp]),
@@ -375,6 +377,28 @@ def coded_gemm(code: Code, A, parity, Bt, Ct=None, status=None) -> torch.Tensor:
     _check(lib().cm_coded_gemm(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
                                _ld(parity, "parity"), Bt.data_ptr(), _ld(Bt, "Bt"), N,
                                Ct.data_ptr(), _ld(Ct, "Ct"), sp, _stream()), "cm_coded_gemm")
+    return Ct
+
+
+def coded_gemm_survivors(code: Code, A, parity, Bt, survivors: int, Ct=None,
+                         status=None) -> torch.Tensor:
+    """Worker products of the k workers decode_mat reads (the other blocks of Ct
+    untouched)."""
+    for t, name in ((A, "A"), (parity, "parity"), (Bt, "Bt")):
+        _dev(t, torch.bfloat16, name, 2)
+    N = Bt.shape[0]
+    if Ct is None:
+        Ct = torch.empty((code.n * code.L, N), dtype=torch.float32, device=A.device)
+    _dev(Ct, torch.float32, "Ct", 2)
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
+    _check(lib().cm_coded_gemm_survivors(code.handle, A.data_ptr(), _ld(A, "A"),
+                                         parity.data_ptr(), _ld(parity, "parity"),
+                                         Bt.data_ptr(), _ld(Bt, "Bt"), N, survivors,
+                                         Ct.data_ptr(), _ld(Ct, "Ct"), sp, _stream()),
+           "cm_coded_gemm_survivors")
     return Ct
 
 

@@ -251,7 +251,26 @@ cm_status cm_coded_gemm(const cm_code *c, const void *A, int64_t lda, const void
     if (!Ct || ((uintptr_t)Ct & 15u) || ldc < N) return CM_EINVAL;
     return from_cuda(launch_coded_gemm(code_params(c), (const uint16_t *)A, lda,
                                        (const uint16_t *)par, ldp, (const uint16_t *)Bt, ldb,
-                                       N, Ct, ldc, dev_status, (cudaStream_t)stream));
+                                       N, Ct, ldc, dev_status, 0u, (cudaStream_t)stream));
+}
+
+cm_status cm_coded_gemm_survivors(const cm_code *c, const void *A, int64_t lda, const void *par,
+                                  int64_t ldp, const void *Bt, int64_t ldb, int32_t N,
+                                  uint32_t survivors, float *Ct, int64_t ldc,
+                                  int32_t *dev_status, cm_stream_t stream)
+{
+    if (!c || c->dt != CM_BF16) return CM_EINVAL;
+    uint32_t eff;
+    cm_status st = resolve_survivors(c, survivors, &eff);
+    if (st != CM_OK) return st;
+    if (N < 1) return CM_EINVAL;
+    if (!layout_ok(A, lda, c->d, 2) || !layout_ok(par, ldp, c->d, 2) ||
+        !layout_ok(Bt, ldb, c->d, 2))
+        return CM_EINVAL;
+    if (!Ct || ((uintptr_t)Ct & 15u) || ldc < N) return CM_EINVAL;
+    return from_cuda(launch_coded_gemm(code_params(c), (const uint16_t *)A, lda,
+                                       (const uint16_t *)par, ldp, (const uint16_t *)Bt, ldb,
+                                       N, Ct, ldc, dev_status, eff, (cudaStream_t)stream));
 }
 
 cm_status cm_decode_mat(const cm_code *c, const float *Ct, int64_t ldc, uint32_t survivors,

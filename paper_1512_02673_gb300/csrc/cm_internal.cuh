@@ -64,6 +64,6 @@ cudaError_t launch_decode_mat(const CodeParams &cp, const float *Ct, int64_t ldc
                               uint32_t survivors, int N, float *C, int64_t ldcc,
                               int32_t *status, cudaStream_t s);
 cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t lda,
-                              const uint16_t *par, int64_t ldp, const uint16_t *Bt,
-                              int64_t ldb, int N, float *Ct, int64_t ldc, int32_t *status,
+                              const uint16_t *par, int64_t ldp, const uint16_t *Bt, int64_t ldb,
+                              int N, float *Ct, int64_t ldc, int32_t *status, uint32_t only,
                               cudaStream_t s);

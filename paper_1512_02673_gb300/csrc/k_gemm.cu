@@ -16,7 +16,7 @@
 // was held near 0.8 of peak by shared-memory traffic (TMA fills plus tensor-
 // core operand reads).
 //
-// Row tiling.  The coded rows are two contiguous ranges: Ct rows [0, kL) are
+// Row tiling (all workers).  The coded rows are two contiguous ranges: Ct rows [0, kL) are
 // rows of A in place (worker j < k owns [jL, jL + L)), Ct rows [kL, nL) are
 // rows of the parity buffer.  Each range is cut into 256-row pairs of its
 // own, A's over its m real rows only, so no tile computes the virtual zero
@@ -29,6 +29,11 @@
 // cover them and by its rank-1 CTA's epilogue past its end.  Pair order:
 // column tile fastest, so the 16 column tiles of one row pair run together
 // and the A~ row slab comes from HBM once; Bt (64 MB) stays L2-resident.
+//
+// Survivors only (cm_coded_gemm_survivors): the listed workers fall into
+// runs of consecutive workers (none across the A | parity boundary), each a
+// contiguous row range of A or of the parity and of Ct, tiled like the two
+// ranges above; the other blocks of Ct are not written.
 //
 // One persistent CTA per SM, warp-specialised, in both CTAs of a pair:
 //   warp 0 lane 0  TMA producer of the CTA's halves (128B-swizzled 128 x 64
@@ -82,6 +87,14 @@ struct GemmArgs {
     int32_t ntiles;    // column tiles
     int32_t kblocks;   // 64-wide K blocks
     int64_t pairs;     // (row pair, column tile) work items
+    // survivors only: runs of consecutive computed workers (0 runs: all of
+    // them, two contiguous ranges)
+    int64_t L;
+    int32_t k;
+    int32_t nruns;
+    int32_t run_p0[CM_MAX_N + 1];   // first row pair of each run; run_p0[nruns] = all
+    int8_t run_w[CM_MAX_N];         // first worker of each run
+    int8_t run_cnt[CM_MAX_N];       // workers in each run
 };
 
 // ---- tcgen05 / cluster helpers (inline PTX) ------------------------------------------
@@ -228,6 +241,22 @@ __device__ __forceinline__ Tile tile_of(const GemmArgs &g, int64_t p, int rank)
     const int nt = (int)(p % g.ntiles);
     const int rp = (int)(p / g.ntiles);
     x.n0 = nt * BN;
+    if (g.nruns > 0) {
+        // survivors only: a pair of one run of consecutive workers; a tile may
+        // read past its run (the next block's rows, or zeros past m) but
+        // stores only the run's rows, its pad rows (zeros past m) included
+        int r = 0;
+        while (r + 1 < g.nruns && rp >= g.run_p0[r + 1]) ++r;
+        const int j = g.run_w[r];
+        const int64_t R = (int64_t)g.run_cnt[r] * g.L;
+        const int64_t r0 = (int64_t)(rp - g.run_p0[r]) * (2 * BM) + rank * BM;
+        x.parity = j >= g.k;
+        x.y = (int32_t)((x.parity ? (int64_t)(j - g.k) : (int64_t)j) * g.L + r0);
+        x.crow = (int64_t)j * g.L + r0;
+        x.rows = (int32_t)(R - r0 < BM ? R - r0 : BM);
+        x.pad = 0;
+        return x;
+    }
     x.parity = rp >= g.psys;
     const int64_t y = (int64_t)(x.parity ? rp - g.psys : rp) * (2 * BM) + rank * BM;
     x.y = (int32_t)y;
@@ -436,7 +465,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUt
 
 cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t lda,
                               const uint16_t *par, int64_t ldp, const uint16_t *Bt, int64_t ldb,
-                              int N, float *Ct, int64_t ldc, int32_t *status, cudaStream_t s)
+                              int N, float *Ct, int64_t ldc, int32_t *status, uint32_t only,
+                              cudaStream_t s)
 {
     CUtensorMap tmA, tmP, tmB;
     const uint64_t d = (uint64_t)cp.d;
@@ -460,6 +490,30 @@ cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t l
     g.ntiles = (N + BN - 1) / BN;
     g.kblocks = (int)((cp.d + BK - 1) / BK);
     g.pairs = (int64_t)(g.psys + g.ppar) * g.ntiles;
+    g.L = cp.L;
+    g.k = cp.k;
+    g.nruns = 0;
+    for (int j = 0; j <= CM_MAX_N; ++j) g.run_p0[j] = 0;
+    for (int j = 0; j < CM_MAX_N; ++j) g.run_w[j] = g.run_cnt[j] = 0;
+    if (only) {   // runs of consecutive workers of `only`, none across A | parity
+        int32_t p0 = 0;
+        for (int j = 0; j < cp.n;) {
+            if (!((only >> j) & 1u)) {
+                ++j;
+                continue;
+            }
+            const int end = j < cp.k ? cp.k : cp.n;
+            int c = 0;
+            while (j + c < end && ((only >> (j + c)) & 1u)) ++c;
+            g.run_w[g.nruns] = (int8_t)j;
+            g.run_cnt[g.nruns] = (int8_t)c;
+            g.run_p0[g.nruns++] = p0;
+            p0 += (int32_t)((c * cp.L + 2 * BM - 1) / (2 * BM));
+            j += c;
+        }
+        g.run_p0[g.nruns] = p0;
+        g.pairs = (int64_t)p0 * g.ntiles;
+    }
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;

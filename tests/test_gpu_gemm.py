@@ -190,6 +190,53 @@ def test_coded_gemm_writes_every_row_and_nothing_else(cm, orc, n, k, m, d, N):
         assert err.max() <= worker_tol(d), (j, err.max())
 
 
+@pytest.mark.parametrize("n,k,m,d,N,kind", [
+    (16, 12, 3000, 192, 200, "mds"),     # L = 250: one row pair per block, rank 1 short
+    (10, 5, 1300, 64, 96, "mds"),        # L = 260: the second pair holds 4 rows
+    (24, 20, 762, 64, 300, "mds"),       # pad rows in the last systematic block
+    (6, 3, 900, 128, 64, "repetition"),
+])
+def test_coded_gemm_survivors_only(cm, orc, n, k, m, d, N, kind):
+    """Survivors-only GEMM: the k blocks that the decode reads equal the full
+    GEMM's bit for bit, no other row of Ct is written, and the decode of them
+    equals the decode after the full GEMM."""
+    P = synth.parity_coefficients(n, k) if kind == "mds" else "repetition"
+    code = cm.Code(n, k, m, d, P, dtype="bf16")
+    L = code.L
+    A = synth.gaussian((m, d), 21, dtype=torch.bfloat16).to(DEV)
+    Bt = synth.gaussian((N, d), 22, dtype=torch.bfloat16).to(DEV)
+    par = cm.encode(code, A)
+    full = cm.coded_gemm(code, A, par, Bt)
+    if kind == "mds":
+        masks = [cm.draw_erasures(synth.ERASURE_SEED, c, n, k)[0] for c in range(3)]
+        # one run of all systematic blocks (pad rows at its end); the last k
+        # workers (a systematic run ending at block k - 1, then the parity)
+        masks += [(1 << k) - 1, ((1 << n) - 1) ^ ((1 << (n - k)) - 1)]
+    else:   # block j of worker j mod k: every block among the survivors
+        masks = [0b111000, 0b100011, 0b111111]
+    for mask in masks:
+        sel = code.select_decodable(mask)
+        buf = torch.full((n * L + 5, N), float("nan"), dtype=torch.float32, device=DEV)
+        status = torch.zeros(1, dtype=torch.int32, device=DEV)
+        Ct = cm.coded_gemm_survivors(code, A, par, Bt, mask, Ct=buf[:n * L], status=status)
+        C = cm.decode_mat(code, Ct, mask, status=status)
+        C_full = cm.decode_mat(code, full, mask)
+        torch.cuda.synchronize()
+        assert status.item() == 0
+        got = buf.cpu()
+        for j in range(n):
+            blk = got[j * L:(j + 1) * L]
+            if (sel >> j) & 1:
+                assert torch.equal(blk, full[j * L:(j + 1) * L].cpu()), j
+            else:
+                assert torch.isnan(blk).all(), j
+        assert torch.isnan(got[n * L:]).all()
+        assert torch.equal(C, C_full)
+    # not decodable: rejected before any launch
+    with pytest.raises(cm.CodedError):
+        cm.coded_gemm_survivors(code, A, par, Bt, (1 << (k - 1)) - 1)
+
+
 @pytest.mark.parametrize("n,k,e", [(32, 16, 16), (20, 10, 9)])
 def test_decode_mat_many_missing_blocks(cm, orc, n, k, e):
     """Matrix decode with up to 16 missing blocks against the oracle's fp64

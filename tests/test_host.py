@@ -116,6 +116,15 @@ def test_synchronous_checks_precede_any_launch(cm):
     assert L.cm_coded_gemm(cb.handle, fake, 68, fake, 64, fake, 64, 32, fake, 32,
                            None, None) == cm.CM_EINVAL    # lda not 16-byte pitched
     assert L.cm_matvec(cb.handle, fake, 64, fake, 64, fake, 1, fake, None, None) == cm.CM_EINVAL
+    # survivors-only GEMM: the survivor checks come before any launch
+    assert L.cm_coded_gemm_survivors(cb.handle, fake, 64, fake, 64, fake, 64, 32, 0b000011,
+                                     fake, 32, None, None) == cm.CM_ENOTDECODABLE
+    assert L.cm_coded_gemm_survivors(cb.handle, fake, 64, fake, 64, fake, 64, 32, 0b1000111,
+                                     fake, 32, None, None) == cm.CM_EINVAL
+    assert L.cm_coded_gemm_survivors(c.handle, fake, 512, fake, 512, fake, 512, 32, 0b111,
+                                     fake, 32, None, None) == cm.CM_EINVAL   # f32 code
+    assert L.cm_coded_gemm_survivors(cb.handle, fake, 64, fake, 64, fake, 64, 32, 0b111,
+                                     fake, 24, None, None) == cm.CM_EINVAL   # ldc < N
 
 
 def test_gd_workspace_and_checks(cm):

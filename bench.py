@@ -418,6 +418,9 @@ def run_ours(args, world, rank, local):
     torch.cuda.empty_cache()
     shuffle = bench_shuffle(cm, dev, synth.SHUFFLE)
     torch.cuda.empty_cache()
+    paper = {w.name: bench_repeats(cm, dev, w) for w in synth.PAPER_MATVEC}
+    paper.update({w.name: bench_gd(cm, dev, args.steps, w) for w in synth.PAPER_GD})
+    torch.cuda.empty_cache()
 
     peaks = measured_peaks()
     achieved = nbytes["matvec"] / (avg["matvec"] * 1e-3) / 1e9
@@ -451,7 +454,7 @@ def run_ours(args, world, rank, local):
         "clocks": clk.summary(),
         "secondary": {"survivors_only": so, "gemm": gemm, "gd": gd,
                       "matvec_100_repeats": mv100, "tiny": tiny,
-                      "coded_shuffling": shuffle,
+                      "coded_shuffling": shuffle, "paper_shaped": paper,
                       "runtime_model": runtime_model_report(cm)},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -600,7 +603,7 @@ def runtime_model_report(cm) -> dict:
     schemes, the simulated MDS mean over the bench's draws, and the optimal k."""
     out = {}
     for name, n, k in [("(32,24)", 32, 24), ("(10,5)", 10, 5), ("(20,10)", 20, 10),
-                       ("(16,12)", 16, 12)]:
+                       ("(16,12)", 16, 12), ("(25,23)", 25, 23), ("(10,8)", 10, 8)]:
         r = {"uncoded": cm.runtime_mean("uncoded", n, n),
              "mds": cm.runtime_mean("mds", n, k)}
         if n % k == 0:
@@ -615,11 +618,10 @@ def runtime_model_report(cm) -> dict:
     return out
 
 
-def bench_gd(cm, dev, steps: int) -> dict:
-    """Coded GD on the 40000 x 8000 regression: seconds per iteration (6
-    launches: two coded products, two plan kernels, two fused decodes),
+def bench_gd(cm, dev, steps: int, w: synth.GDWorkload = synth.GD) -> dict:
+    """Coded GD (default: the 40000 x 8000 regression): seconds per iteration
+    (6 launches: two coded products, two plan kernels, two fused decodes),
     effective GB/s."""
-    w = synth.GD
     A, _, y = synth.regression_inputs(w, device=dev)
     AT = A.t().contiguous()
     cA = cm.Code(w.n, w.k_a, w.m, w.d, synth.parity_coefficients(w.n, w.k_a))
@@ -732,6 +734,10 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
     P = synth.parity_coefficients(w.n, w.k)
     code = cm.Code(w.n, w.k, w.m, w.d, P)
     A, X = synth.matvec_inputs(w, device=dev)
+    if w.d % 4:   # rows on a 16-byte pitch (the library's layout contract)
+        Ap = torch.empty((w.m, (w.d + 3) // 4 * 4), device=dev)[:, :w.d]
+        Ap.copy_(A)
+        A = Ap
     status = torch.zeros(1, dtype=torch.int32, device=dev)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     parity = cm.encode(code, A)

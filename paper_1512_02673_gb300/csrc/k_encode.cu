@@ -3,19 +3,21 @@
 // blocks of A (rows past m are the appended zero rows).
 //
 // A short contraction (k <= 31 terms per output) that streams A once.  Work
-// unit = one block row r and a 4096-column segment, owned by one warp; a
-// persistent grid sweeps the units.  Each 128-column step of a unit gathers
-// row r of every data block into shared memory with TMA in sub-steps of KC
-// blocks: 3-D boxes of KC full blocks (block stride L rows; boxes past the
-// last full block read as zero) plus, if m is not a multiple of L, one 2-D
-// box of the partial block whose rows past m read as zero; blocks wholly past
-// m are skipped.  Sub-steps stream through a per-warp ring of ST slots with
-// one mbarrier each (lane 0 issues, the warp consumes), so several KB per
-// warp are in flight with no per-lane copy work, and small slots leave room
-// for 16 warps per SM.  Lane l owns
-// columns [4l, 4l+4) of the step and keeps the accumulators of all parity
-// blocks of the pass in registers (packed fp32x2 FMAs with the coefficient
-// pair (P[p][i], P[p][i]) read as a shared-memory broadcast), then stores them
+// unit = one block row r and a segment of at most 4096 columns, owned by one
+// warp; a persistent grid sweeps the units.  The launcher takes the longest
+// segment whose units fill the rounds of the grid's warps to 90 % (at L of a
+// few hundred rows, 4096-column segments leave most warps idle).  Each
+// 128-column step of a unit gathers row r of every data block into shared
+// memory with TMA in sub-steps of KC blocks: 3-D boxes of KC full blocks
+// (block stride L rows; boxes past the last full block read as zero) plus, if
+// m is not a multiple of L, one 2-D box of the partial block whose rows past
+// m read as zero; blocks wholly past m are skipped.  Sub-steps stream through
+// a per-warp ring of ST slots with one mbarrier each (lane 0 issues, the warp
+// consumes), so several KB per warp are in flight with no per-lane copy work,
+// and small slots leave room for 16 warps per SM.  Lane l owns columns
+// [4l, 4l+4) of the step and keeps the accumulators of all parity blocks of
+// the pass in registers (packed fp32x2 FMAs with the coefficient pair
+// (P[p][i], P[p][i]) read as a shared-memory broadcast), then stores them
 // with coalesced streaming stores.  Every element of A is read once per pass
 // and every parity element written once; n - k <= 16 is one pass.  fp32
 // accumulation in the order i = 0..k-1; bf16 outputs are rounded to nearest
@@ -29,7 +31,7 @@
 namespace {
 
 constexpr int STEP = 128;       // columns per step
-constexpr int SEG = 32;         // steps per work unit
+constexpr int SEG = 32;         // steps per work unit, at most
 constexpr int KC = 8;           // data blocks per sub-step (one TMA box)
 constexpr int ST = 3;           // ring slots per warp
 constexpr int kWarps = 8;
@@ -87,15 +89,15 @@ struct EncodeArgs {
     int32_t kv;          // data blocks with at least one row below m
     int32_t p0, np;      // parity blocks of this pass
     int32_t steps;       // 128-column steps per row
+    int32_t seg;         // steps per segment
     int32_t nseg;        // segments per row
     int32_t nsub;        // sub-steps per step: ceil(kf / KC) + (kv > kf)
     int64_t units;       // L * nseg
 };
 
 template <typename T, int NPG>
-__global__ void __launch_bounds__(kWarps * 32)
-encode_kernel(const __grid_constant__ CUtensorMap tmF, const __grid_constant__ CUtensorMap tmP,
-              const CodeParams cp, const EncodeArgs a)
+__device__ __forceinline__ void encode_body(const CUtensorMap &tmF, const CUtensorMap &tmP,
+                                            const CodeParams &cp, const EncodeArgs &a)
 {
     constexpr uint32_t SLOT = KC * STEP * sizeof(T);
     // dynamic shared memory: [rings, 1024-aligned][coefficient pairs][mbarriers]
@@ -123,8 +125,8 @@ encode_kernel(const __grid_constant__ CUtensorMap tmF, const __grid_constant__ C
     const int nfull = (a.kf + KC - 1) / KC;      // sub-steps of full blocks
 
     auto unit_steps = [&](int64_t u) {           // the last segment of a row may be short
-        const int s0 = (int)(u % a.nseg) * SEG;
-        return (a.steps - s0) < SEG ? a.steps - s0 : SEG;
+        const int s0 = (int)(u % a.nseg) * a.seg;
+        return (a.steps - s0) < a.seg ? a.steps - s0 : a.seg;
     };
 
     // ---- producer (lane 0): sub-step c of step p_s of unit p_unit ----
@@ -132,7 +134,7 @@ encode_kernel(const __grid_constant__ CUtensorMap tmF, const __grid_constant__ C
     int p_s = 0, p_c = 0, p_slot = 0, in_flight = 0;
     auto produce = [&]() {
         const int64_t r = p_unit / a.nseg;
-        const int32_t x = ((int)(p_unit % a.nseg) * SEG + p_s) * STEP;
+        const int32_t x = ((int)(p_unit % a.nseg) * a.seg + p_s) * STEP;
         unsigned char *dst = ring + p_slot * SLOT;
         // no proxy fence: the slot is only written by TMA, and the __syncwarp
         // before every refill orders the lanes' reads of it before the copy
@@ -211,7 +213,7 @@ encode_kernel(const __grid_constant__ CUtensorMap tmF, const __grid_constant__ C
                     if (p_unit < a.units) produce();   // refill it
                 }
             }
-            const int64_t col = (int64_t)(seg * SEG + s) * STEP + 4 * lane;
+            const int64_t col = (int64_t)(seg * a.seg + s) * STEP + 4 * lane;
             if (col < a.d) {
 #pragma unroll
                 for (int j = 0; j < NPG; ++j) {
@@ -229,6 +231,24 @@ encode_kernel(const __grid_constant__ CUtensorMap tmF, const __grid_constant__ C
             }
         }
     }
+}
+
+// up to 8 parity blocks per pass: the compiler's own register choice (two or
+// three CTAs per SM); 16: capped at 128 registers, two CTAs per SM
+template <typename T, int NPG>
+__global__ void __launch_bounds__(kWarps * 32)
+encode_kernel(const __grid_constant__ CUtensorMap tmF, const __grid_constant__ CUtensorMap tmP,
+              const CodeParams cp, const EncodeArgs a)
+{
+    encode_body<T, NPG>(tmF, tmP, cp, a);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kWarps * 32, 2)
+encode_kernel16(const __grid_constant__ CUtensorMap tmF, const __grid_constant__ CUtensorMap tmP,
+                const CodeParams cp, const EncodeArgs a)
+{
+    encode_body<T, 16>(tmF, tmP, cp, a);
 }
 
 template <typename T, int NPG>
@@ -260,10 +280,12 @@ cudaError_t launch_passes(const CodeParams &cp, const T *A, int64_t lda, T *par,
     a.kf = kf;
     a.kv = kv;
     a.steps = (int)((cp.d + STEP - 1) / STEP);
-    a.nseg = (a.steps + SEG - 1) / SEG;
-    a.units = cp.L * a.nseg;
     a.nsub = (kf + KC - 1) / KC + (kv > kf ? 1 : 0);
-    auto kern = encode_kernel<T, NPG>;
+    void (*kern)(const CUtensorMap, const CUtensorMap, const CodeParams, const EncodeArgs);
+    if constexpr (NPG > 8)
+        kern = encode_kernel16<T>;
+    else
+        kern = encode_kernel<T, NPG>;
     const int smem = 1024 + kWarps * ST * KC * STEP * (int)es + 32 * NPG * 8 + kWarps * ST * 8;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
@@ -272,6 +294,24 @@ cudaError_t launch_passes(const CodeParams &cp, const T *A, int64_t lda, T *par,
     if (e != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
     int64_t grid = (int64_t)cm_sm_count() * per_sm;
+    {   // segment length (see the header)
+        const int64_t warps = grid * kWarps;
+        double best = -1.0;
+        for (int ns = (a.steps + SEG - 1) / SEG; ns <= a.steps; ++ns) {
+            const int sg = (a.steps + ns - 1) / ns;
+            const int nsg = (a.steps + sg - 1) / sg;
+            const int64_t units = cp.L * nsg;
+            const int64_t rounds = (units + warps - 1) / warps;
+            const double fill = (double)cp.L * a.steps / ((double)rounds * sg * warps);
+            if (fill > best + 1e-9) {
+                best = fill;
+                a.seg = sg;
+                a.nseg = nsg;
+            }
+            if (fill >= 0.9) break;
+        }
+    }
+    a.units = cp.L * a.nseg;
     const int64_t need = (a.units + kWarps - 1) / kWarps;
     if (grid > need) grid = need;
     if (grid < 1) grid = 1;

@@ -74,6 +74,13 @@ BANDWIDTH = Workload("coded mat-multi-vec (32,24) 65536x65536 b=8", m=65536,
                      d=65536, b=8, n=32, k=24, data_device="cuda")
 GEMM = Workload("coded GEMM bf16 (16,12) 32768x8192x4096", m=32768, d=8192,
                 b=0, n=16, k=12, dtype="bf16", gemm_n=4096)
+# the matrix shapes of the paper's cluster experiments (Sec. III-F): a (25,23)
+# code on square, fat and tall matrices times one vector, and (10,8) coded
+# gradient descent (iteration count not given there: 50, as above)
+PAPER_MATVEC = [Workload("paper (25,23) %dx%d" % (m, d), m=m, d=d, b=1, n=25, k=23,
+                         repeats=20) for m, d in [(5750, 5750), (5750, 11500), (11500, 5750)]]
+PAPER_GD = [GDWorkload("paper GD (10,8) %dx%d" % (m, d), m=m, d=d, n=10, k_a=8, k_at=8,
+                       iters=50) for m, d in [(2000, 2000), (400, 10000), (10000, 400)]]
 
 
 @dataclasses.dataclass(frozen=True)

@@ -80,3 +80,14 @@ def test_gd_config_50_iterations(cm, orc):
     want = orc.gd(A.numpy(), y.numpy(), w.eta, w.iters)
     err = np.linalg.norm(x - want) / np.linalg.norm(want)
     assert err <= 1e-3, err
+
+
+@pytest.mark.parametrize("w", synth.PAPER_GD, ids=lambda w: "%dx%d" % (w.m, w.d))
+def test_gd_paper_shapes(cm, orc, w):
+    """(10,8) coded gradient descent on the square, fat and tall matrices of
+    Sec. III-F, 50 iterations against the oracle's fp64 iteration."""
+    A, _, y = synth.regression_inputs(w, device="cpu")
+    x, _ = run_coded_gd(cm, A, y, w.n, w.k_a, w.k_at, w.iters, w.eta)
+    want = orc.gd(A.numpy(), y.numpy(), w.eta, w.iters)
+    err = np.linalg.norm(x - want) / np.linalg.norm(want)
+    assert err <= 1e-3, err

@@ -128,6 +128,11 @@ SHAPES = [
     (16, 12, 3001, 4096, 4, None),
     (7, 3, 300, 9000, 6, 9004),    # several X chunks (b = 6 pads to 8)
     (12, 5, 700, 17000, 1, None),  # several X chunks at b = 1
+    # the (25,23) code on the square, fat and tall matrices of Sec. III-F
+    # (rows of 5750 floats padded to a 16-byte pitch)
+    (25, 23, 5750, 5750, 1, 5752),
+    (25, 23, 5750, 11500, 1, None),
+    (25, 23, 11500, 5750, 1, 5752),
 ]
 
 

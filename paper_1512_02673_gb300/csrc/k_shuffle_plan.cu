@@ -6,25 +6,31 @@
 // (partition, cache masks, slot tables) resident in the caller's workspace,
 // so that a transition needs no host work beyond reading back four counts.
 // The definitions are the host planner's (see its header comment); the
-// device version reaches the same order through stable sorts:
-//   partition     rows sorted by (key, row): a stable LSD radix sort of the
-//                 rows (ascending) on the top 24 bits of their 64-bit keys,
-//                 then each run of equal top bits sorted by (key, row);
+// device version reaches the same result through selections and stable sorts:
+//   partition     owner = rank of the row in (key, row) order / (q/n): a
+//                 histogram of the top bits of the keys and its scan give
+//                 every bucket its first rank; a bucket inside one owner's
+//                 positions gives its rows that owner, and the few rows of
+//                 the buckets across a boundary are ranked among themselves;
 //   received      missing rows in (worker, row) order: a stable sort by
 //                 worker of the rows in ascending order;
 //   messages      received rows stably sorted by the set I (bit mask), i.e.
 //                 (I, worker, row); row j of a worker's run in I goes to
 //                 message row base(I) + j, entries ordered by worker;
-//   cache update  candidates (worker, row) stably sorted on the top key bits,
-//                 then by worker, runs of equal (worker, top bits) by
-//                 (key, row): the first s - q/n of each worker are kept;
+//   cache update  the s - q/n candidates (worker, row) of smallest (key, row)
+//                 of every worker: per worker a histogram of the top 16 key
+//                 bits locates the bucket of its (s - q/n)-th candidate;
+//                 candidates below it are kept, those in it ranked exactly;
 //   commit        dropped slots of each worker, ascending, take its received
 //                 rows in order.
-// Radix passes: one warp per tile of 1024 items, 8-bit digits; a tile's
-// histogram by shared-memory atomics, global offsets by an exclusive scan of
-// the (digit, tile) matrix, and a stable scatter that ranks equal digits
-// within each 32-item step by __match_any_sync, reorders the tile by digit in
-// shared memory and writes each digit's run to consecutive addresses.
+// Radix sorts: 8-bit digits, one histogram launch for all passes of a sort
+// and one launch per pass.  A pass takes tiles of 4096 items in the order of
+// an atomic counter; a tile ranks its items stably (equal digits of a 32-item
+// step by __match_any_sync, warps in order), publishes its digit counts, and
+// finds its global digit offsets by looking back over the flags of the tiles
+// before it (decoupled look-back: a tile's flag holds its count, then its
+// inclusive prefix; a bounded wait, an error flag on time-out), then writes
+// each digit's run to consecutive addresses through shared memory.
 // Device scans: 4096 items per 1024-thread block, block sums scanned
 // recursively.
 #include <cuda_runtime.h>
@@ -38,11 +44,25 @@
 
 namespace {
 
-constexpr int kTile = 1024;        // items per warp in a radix pass
-constexpr int kRadixWarps = 4;     // warps (tiles) per radix block
-// shared memory of one warp's scatter: its tile's keys and values in digit
-// order, and three 256-entry tables (local starts, running counts, global bases)
-constexpr int kScatterWarpBytes = kTile * 12 + 3 * 256 * 4;
+constexpr int kSortThreads = 256;  // one radix tile per block: 8 warps
+constexpr int kSortWarps = kSortThreads / 32;
+constexpr int kSortIpt = 16;       // items per thread
+constexpr int kTile = kSortThreads * kSortIpt;   // items per tile
+constexpr int kMaxPasses = 2;      // 16-bit keys at most
+constexpr int kSortSlots = 2;      // sorts per transition (own global histograms)
+constexpr int kCBits = 16;         // bucket bits of the cache-update selection
+// shared memory of a pass: the tile's keys and values in digit order, the
+// per-warp digit counts, the tile's digit starts and global bases
+constexpr int kSortSmem = kTile * 12 + (kSortWarps + 2) * 256 * 4 + 64;
+// the totals array: T_COUNT counters read back by the host; the lengths of
+// the two selections' boundary lists (kListP, kListC); per worker the
+// cache-update bucket (kThr) and how many of its candidates to keep
+// (kNeed); the tile and done counters of the running radix pass at kCtr;
+// the global histograms of the radix sorts from word 64
+constexpr int kListP = 8, kListC = 9, kThr = 16, kNeed = 32;
+constexpr int kCtr = 56;
+constexpr int kGhist = 64;
+constexpr int kTotalsWords = kGhist + kSortSlots * kMaxPasses * 256;
 constexpr int kScanBlock = 1024;
 constexpr int kScanItems = 4 * kScanBlock;
 constexpr int kMaxDeviceN = 16;    // dense tables over all 2^n worker sets
@@ -187,140 +207,231 @@ cudaError_t scan_exclusive(const int32_t *in, int32_t *out, int64_t count, int32
 
 // ---- stable LSD radix sort (64-bit keys, int32 values) ---------------------------------
 
-__global__ void radix_hist_kernel(const uint64_t *keys, const int32_t *countp, int64_t cap,
-                                  int shift, int32_t *hist, int64_t tiles)
+// Counts of every digit of every pass of a sort, summed into ghist[pass][256]
+// (zero on entry).
+__global__ void __launch_bounds__(256) radix_hist_kernel(const uint64_t *keys,
+                                                         const int32_t *countp, int64_t cap,
+                                                         int lo, int passes, int32_t *ghist)
 {
-    __shared__ int32_t cnt[kRadixWarps][256];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int64_t tile = (int64_t)blockIdx.x * kRadixWarps + warp;
-    for (int d = lane; d < 256; d += 32) cnt[warp][d] = 0;
-    __syncwarp();
-    if (tile >= tiles) return;
+    __shared__ int32_t h[kMaxPasses][256];
+    for (int t = threadIdx.x; t < kMaxPasses * 256; t += blockDim.x) h[t / 256][t % 256] = 0;
+    __syncthreads();
     const int64_t count = countp ? (int64_t)*countp : cap;
-    const int64_t beg = tile * kTile, end = std::min(count, beg + kTile);
-#pragma unroll 8
-    for (int64_t i = beg + lane; i < end; i += 32) atomicAdd(&cnt[warp][(keys[i] >> shift) & 255], 1);
-    __syncwarp();
-    for (int d = lane; d < 256; d += 32) hist[(int64_t)d * tiles + tile] = cnt[warp][d];
+    GS_LOOP(i, count)
+    {
+        const uint64_t k = keys[i];
+        for (int p = 0; p < passes; ++p) atomicAdd(&h[p][(k >> (lo + 8 * p)) & 255], 1);
+    }
+    __syncthreads();
+    for (int t = threadIdx.x; t < passes * 256; t += blockDim.x)
+        if (h[t / 256][t % 256]) atomicAdd(&ghist[t], h[t / 256][t % 256]);
 }
 
-// One warp per tile of 32 x 32 items: (1) the tile loaded into registers
-// (lane l holds items l, 32 + l, ...; all loads in flight together), its digit
-// counts and their exclusive scan (local starts); (2) every item placed,
-// stably, at its digit's local start plus its rank in shared memory (equal
-// digits of a 32-item step ranked by lane with __match_any_sync); (3) the
-// tile written out in that digit order: a run of equal digits goes to
-// consecutive global positions, so the writes coalesce.
-__global__ void __launch_bounds__(32 * kRadixWarps)
-radix_scatter_kernel(const uint64_t *kin, const int32_t *vin, uint64_t *kout, int32_t *vout,
-                     const int32_t *countp, int64_t cap, int shift, const int32_t *offsets,
-                     int64_t tiles)
+// Tile flags of the decoupled look-back: epoch << 32 | status << 30 | value.
+constexpr uint64_t kFlagAgg = 1, kFlagInc = 2;
+constexpr int kLook = 16;   // tiles read together by one step of the look-back
+
+__device__ __forceinline__ uint64_t flag_word(uint32_t epoch, uint64_t status, int32_t v)
 {
-    static_assert(kTile == 32 * 32, "a tile is 32 steps of 32 items");
-    extern __shared__ __align__(16) unsigned char smem[];
+    return ((uint64_t)epoch << 32) | (status << 30) | (uint64_t)(uint32_t)v;
+}
+
+// Exclusive scan over the block's 256 threads (one value each); returns the
+// thread's exclusive prefix and leaves the total in *total.
+__device__ __forceinline__ int32_t block_scan256(int32_t x, int32_t *wsum, int32_t *total)
+{
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    unsigned char *mine = smem + warp * kScatterWarpBytes;
-    uint64_t *sk = reinterpret_cast<uint64_t *>(mine);
-    int32_t *sv = reinterpret_cast<int32_t *>(mine + kTile * 8);
-    int32_t *start = reinterpret_cast<int32_t *>(mine + kTile * 12);
-    int32_t *run = start + 256;
-    int32_t *base = run + 256;
-    const int64_t tile = (int64_t)blockIdx.x * kRadixWarps + warp;
-    if (tile >= tiles) return;
+    int32_t inc = x;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+    }
+    if (lane == 31) wsum[warp] = inc;
+    __syncthreads();
+    int32_t before = 0, all = 0;
+#pragma unroll
+    for (int w = 0; w < kSortWarps; ++w) {
+        const int32_t v = wsum[w];
+        before += w < warp ? v : 0;
+        all += v;
+    }
+    __syncthreads();
+    *total = all;
+    return before + inc - x;
+}
+
+// One pass: bits [shift, shift + 8) of the keys.  ctr[0] hands out tiles,
+// ctr[1] counts finished blocks; the last block resets both.
+__global__ void __launch_bounds__(kSortThreads)
+radix_pass_kernel(const uint64_t *kin, const int32_t *vin, uint64_t *kout, int32_t *vout,
+                  const int32_t *countp, int64_t cap, int shift, const int32_t *ghist,
+                  uint64_t *flags, uint32_t epoch, int32_t *ctr, int32_t *err)
+{
+    extern __shared__ __align__(16) unsigned char smem[];
+    uint64_t *sk = reinterpret_cast<uint64_t *>(smem);
+    int32_t *sv = reinterpret_cast<int32_t *>(smem + kTile * 8);
+    int32_t *wcnt = sv + kTile;                      // [warp][digit]
+    int32_t *dstart = wcnt + kSortWarps * 256;       // tile-local start of each digit
+    int32_t *gbase = dstart + 256;                   // global position of that start
+    int32_t *misc = gbase + 256;                     // [0]: tile, [1..8]: warp sums
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, d = threadIdx.x;
+    if (threadIdx.x == 0) misc[0] = atomicAdd(&ctr[0], 1);
+    __syncthreads();
+    const int64_t tile = misc[0];
     const int64_t count = countp ? (int64_t)*countp : cap;
-    const int64_t beg = tile * kTile, end = std::min(count, beg + kTile);
-    const int nt = end > beg ? (int)(end - beg) : 0;
-    for (int d = lane; d < 256; d += 32) {
-        run[d] = 0;
-        base[d] = offsets[(int64_t)d * tiles + tile];
-    }
-    uint64_t k[32];
-    int32_t v[32];
+    const int64_t beg = tile * kTile;
+    if (beg < count) {
+        const int nt = (int)(count - beg < kTile ? count - beg : kTile);
+        // items w * 512 + 32 j + lane of the tile, in registers
+        uint64_t k[kSortIpt];
+        int32_t v[kSortIpt], r[kSortIpt];
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
-        const int p = 32 * j + lane;
-        k[j] = p < nt ? kin[beg + p] : 0;
-        v[j] = p < nt ? vin[beg + p] : 0;
-    }
-    __syncwarp();
-#pragma unroll
-    for (int j = 0; j < 32; ++j)
-        if (32 * j + lane < nt) atomicAdd(&run[(k[j] >> shift) & 255], 1);
-    __syncwarp();
-    {   // exclusive scan of the 256 counts: 8 per lane
-        int32_t c[8], sum = 0;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            c[q] = run[8 * lane + q];
-            sum += c[q];
+        for (int j = 0; j < kSortIpt; ++j) {
+            const int p = warp * 32 * kSortIpt + 32 * j + lane;
+            k[j] = p < nt ? kin[beg + p] : 0;
+            v[j] = p < nt ? vin[beg + p] : 0;
         }
-        int32_t x = sum;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int32_t y = __shfl_up_sync(0xffffffffu, x, o);
-            if (lane >= o) x += y;
-        }
-        int32_t at = x - sum;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            start[8 * lane + q] = at;
-            at += c[q];
-        }
-    }
-    __syncwarp();
-    for (int d = lane; d < 256; d += 32) run[d] = 0;
-    __syncwarp();
-    const unsigned below = (1u << lane) - 1u;
-#pragma unroll
-    for (int j = 0; j < 32; ++j) {
-        if (32 * j >= nt) break;   // warp-uniform
-        const bool valid = 32 * j + lane < nt;
-        const int d = valid ? (int)((k[j] >> shift) & 255) : 256;   // 256: not an item
-        const unsigned peers = __match_any_sync(0xffffffffu, d);
-        if (valid) {
-            const int pos = start[d] + run[d] + __popc(peers & below);
-            sk[pos] = k[j];
-            sv[pos] = v[j];
-        }
+        int32_t *mine = wcnt + warp * 256;
+        for (int t = lane; t < 256; t += 32) mine[t] = 0;
         __syncwarp();
-        if (valid && (peers & below) == 0) run[d] += __popc(peers);
-        __syncwarp();
+        const unsigned below = (1u << lane) - 1u;
+#pragma unroll
+        for (int j = 0; j < kSortIpt; ++j) {
+            const bool valid = warp * 32 * kSortIpt + 32 * j + lane < nt;
+            const int dg = valid ? (int)((k[j] >> shift) & 255) : 256;   // 256: not an item
+            const unsigned peers = __match_any_sync(0xffffffffu, dg);
+            r[j] = valid ? mine[dg] + __popc(peers & below) : 0;
+            __syncwarp();
+            if (valid && (peers & below) == 0) mine[dg] += __popc(peers);
+            __syncwarp();
+        }
+        __syncthreads();
+        // digit d: prefixes over the warps, its total, its tile-local start
+        int32_t tot = 0;
+#pragma unroll
+        for (int w = 0; w < kSortWarps; ++w) {
+            const int32_t c = wcnt[w * 256 + d];
+            wcnt[w * 256 + d] = tot;
+            tot += c;
+        }
+        // publish the tile's count of digit d (tile 0: its inclusive prefix,
+        // from the digit's start over all keys) for the tiles after it
+        int32_t gd = 0;
+        uint64_t *f = flags + tile * 256 + d;
+        if (tile == 0) {
+            int32_t ga;
+            gd = block_scan256(ghist[d], misc + 1, &ga);
+            atomicExch(reinterpret_cast<unsigned long long *>(f),
+                       (unsigned long long)flag_word(epoch, kFlagInc, gd + tot));
+        } else {
+            atomicExch(reinterpret_cast<unsigned long long *>(f),
+                       (unsigned long long)flag_word(epoch, kFlagAgg, tot));
+        }
+        int32_t all;
+        const int32_t ds = block_scan256(tot, misc + 1, &all);
+        dstart[d] = ds;
+        __syncthreads();
+        // the tile in digit order in shared memory (the registers are free
+        // before the look-back)
+#pragma unroll
+        for (int j = 0; j < kSortIpt; ++j) {
+            if (warp * 32 * kSortIpt + 32 * j + lane < nt) {
+                const int dg = (int)((k[j] >> shift) & 255);
+                const int pos = dstart[dg] + wcnt[warp * 256 + dg] + r[j];
+                sk[pos] = k[j];
+                sv[pos] = v[j];
+            }
+        }
+        if (tile > 0) {   // the counts of digit d in the tiles before this one
+            // look back kLook tiles at a time: their flags are read together,
+            // then summed newest first up to the first inclusive one; an
+            // unpublished flag is read again (a bounded wait)
+            int32_t excl = 0;
+            int64_t t = tile - 1;
+            uint32_t it = 0;
+            while (t >= 0) {
+                uint64_t w[kLook];
+#pragma unroll
+                for (int i = 0; i < kLook; ++i)
+                    w[i] = t - i >= 0 ? *(const volatile uint64_t *)(flags + (t - i) * 256 + d)
+                                      : flag_word(epoch, kFlagInc, 0);
+                int used = kLook;
+                bool done = false;
+#pragma unroll
+                for (int i = 0; i < kLook; ++i) {
+                    if (done || used < kLook) continue;
+                    if ((uint32_t)(w[i] >> 32) != epoch) {
+                        used = i;   // not yet published: read again from tile t - i
+                    } else {
+                        excl += (int32_t)(w[i] & 0x3fffffffu);
+                        if (((w[i] >> 30) & 3u) == kFlagInc) done = true;
+                    }
+                }
+                if (done) break;
+                t -= used;
+                if (used < kLook) {
+                    // give up after about 0.1-1 s, or at once if another thread has
+                    if (++it > (1u << 21) || *(volatile int32_t *)err) {
+                        atomicExch(err, 1);
+                        break;
+                    }
+                    __nanosleep(64);
+                }
+            }
+            atomicExch(reinterpret_cast<unsigned long long *>(f),
+                       (unsigned long long)flag_word(epoch, kFlagInc, excl + tot));
+            gd = excl;
+        }
+        gbase[d] = gd;
+        __syncthreads();
+        // each digit's run out
+        for (int p = threadIdx.x; p < nt; p += kSortThreads) {
+            const uint64_t kk = sk[p];
+            const int dg = (int)((kk >> shift) & 255);
+            const int64_t g = (int64_t)gbase[dg] + (p - dstart[dg]);
+            kout[g] = kk;
+            vout[g] = sv[p];
+        }
     }
-    for (int p = lane; p < nt; p += 32) {
-        const uint64_t kk = sk[p];
-        const int d = (int)((kk >> shift) & 255);
-        const int g = base[d] + (p - start[d]);
-        kout[g] = kk;
-        vout[g] = sv[p];
+    __syncthreads();
+    if (threadIdx.x == 0 && atomicAdd(&ctr[1], 1) == (int32_t)gridDim.x - 1) {
+        ctr[0] = 0;   // every block has taken its tile: ready for the next pass
+        ctr[1] = 0;
     }
 }
 
 struct SortBufs {
     uint64_t *kA, *kB;
     int32_t *vA, *vB;
-    int32_t *hist, *scan;
+    uint64_t *flags;
+    int32_t *ghist;   // kSortSlots x kMaxPasses x 256, zero at the start of a transition
+    int32_t *ctr, *err;
+    uint32_t *epoch;
 };
 
 // Stable sort of items [0, count) (count = *countp, or cap if countp is null)
-// by bits [lo, hi) of their keys; on return the sorted keys and values are in
+// by bits [lo, hi) of their keys (at most kMaxPasses digits), using global
+// histogram slot `slot`; on return the sorted keys and values are in
 // (*k_out, *v_out), one of the two buffer pairs.
 cudaError_t radix_sort(const SortBufs &b, const int32_t *countp, int64_t cap, int lo, int hi,
-                       cudaStream_t s, uint64_t **k_out, int32_t **v_out)
+                       int slot, cudaStream_t s, uint64_t **k_out, int32_t **v_out)
 {
+    const int passes = (hi - lo + 7) / 8;
+    if (passes < 1 || passes > kMaxPasses || slot < 0 || slot >= kSortSlots)
+        return cudaErrorInvalidValue;
     const int64_t tiles = std::max<int64_t>(1, (cap + kTile - 1) / kTile);
-    const unsigned blocks = (unsigned)((tiles + kRadixWarps - 1) / kRadixWarps);
+    int32_t *gh = b.ghist + slot * kMaxPasses * 256;
     uint64_t *ki = b.kA, *ko = b.kB;
     int32_t *vi = b.vA, *vo = b.vB;
-    cudaError_t ea = cudaFuncSetAttribute(radix_scatter_kernel,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          kRadixWarps * kScatterWarpBytes);
+    cudaError_t ea = cudaFuncSetAttribute(radix_pass_kernel,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, kSortSmem);
     if (ea != cudaSuccess) return ea;
-    for (int shift = lo; shift < hi; shift += 8) {
-        radix_hist_kernel<<<blocks, 32 * kRadixWarps, 0, s>>>(ki, countp, cap, shift, b.hist, tiles);
-        cudaError_t e = scan_exclusive(b.hist, b.hist, 256 * tiles, b.scan, nullptr, s);
-        if (e != cudaSuccess) return e;
-        radix_scatter_kernel<<<blocks, 32 * kRadixWarps, kRadixWarps * kScatterWarpBytes, s>>>(
-            ki, vi, ko, vo, countp, cap, shift, b.hist, tiles);
+    radix_hist_kernel<<<grid_for(cap), 256, 0, s>>>(ki, countp, cap, lo, passes, gh);
+    for (int p = 0; p < passes; ++p) {
+        const uint32_t epoch = ++*b.epoch;
+        radix_pass_kernel<<<(unsigned)tiles, kSortThreads, kSortSmem, s>>>(
+            ki, vi, ko, vo, countp, cap, lo + 8 * p, gh + p * 256, b.flags, epoch, b.ctr, b.err);
         std::swap(ki, ko);
         std::swap(vi, vo);
     }
@@ -331,39 +442,187 @@ cudaError_t radix_sort(const SortBufs &b, const int32_t *countp, int64_t cap, in
 
 // ---- planner kernels --------------------------------------------------------------------
 
-__global__ void partition_keys_kernel(uint64_t *keys, int32_t *vals, int64_t q, uint64_t seed,
-                                      int64_t t1)
+// ---- partition by selection ------------------------------------------------------------
+
+__device__ __forceinline__ uint64_t part_key(uint64_t seed, int64_t t1, int64_t q, int64_t r)
+{
+    return mix64(seed, (uint64_t)t1 * (uint64_t)q + (uint64_t)r);
+}
+
+// rows per bucket of the top `bits` key bits (hist zero on entry)
+__global__ void part_hist_kernel(int64_t q, uint64_t seed, int64_t t1, int bits, int32_t *hist)
+{
+    GS_LOOP(r, q) atomicAdd(&hist[part_key(seed, t1, q, r) >> (64 - bits)], 1);
+}
+
+// The owner of every row whose bucket's ranks [bstart, bstart + count) lie
+// inside one owner's positions; the rows of the other buckets are listed.
+__global__ void part_owner_kernel(int64_t q, uint64_t seed, int64_t t1, int bits, int64_t per,
+                                  const int32_t *hist, const int32_t *bstart, int32_t *owner1,
+                                  int32_t *list, int32_t *nlist)
 {
     GS_LOOP(r, q)
     {
-        keys[r] = mix64(seed, (uint64_t)t1 * (uint64_t)q + (uint64_t)r);
-        vals[r] = (int32_t)r;
+        const int64_t b = (int64_t)(part_key(seed, t1, q, r) >> (64 - bits));
+        const int64_t lo = bstart[b], hi = lo + hist[b] - 1;
+        if (lo / per == hi / per) owner1[r] = (int32_t)(lo / per);
+        else list[atomicAdd(nlist, 1)] = (int32_t)r;
     }
 }
 
-__global__ void owner_kernel(const int32_t *order, int64_t q, int64_t per, int32_t *owner1)
+// A listed row's rank: its bucket's first rank plus the listed rows of the
+// same bucket before it in (key, row) order.
+__global__ void part_rank_kernel(int64_t q, uint64_t seed, int64_t t1, int bits, int64_t per,
+                                 const int32_t *bstart, const int32_t *list,
+                                 const int32_t *nlist, int32_t *owner1)
 {
-    GS_LOOP(pos, q) owner1[order[pos]] = (int32_t)(pos / per);
+    const int64_t m = *nlist;
+    GS_LOOP(x, m)
+    {
+        const int32_t r = list[x];
+        const uint64_t k = part_key(seed, t1, q, r), b = k >> (64 - bits);
+        int64_t rank = bstart[b];
+        for (int64_t y = 0; y < m; ++y) {
+            const int32_t r2 = list[y];
+            const uint64_t k2 = part_key(seed, t1, q, r2);
+            if ((k2 >> (64 - bits)) == b && (k2 < k || (k2 == k && r2 < r))) ++rank;
+        }
+        owner1[r] = (int32_t)(rank / per);
+    }
 }
 
-// Per row: missing from its new owner's cache?  Its set I, its candidate
-// bits for the cache refill; counts per (I, worker), per worker and per
-// candidate worker.  Counters of n bins are aggregated in shared memory.
-// Per row: missing from its new owner's cache?  Its set I, its candidate
-// bits for the cache refill; counts per (I, worker), per worker and per
-// candidate worker.  The per-worker counters are aggregated in shared memory
-// per block, and so are the (I, worker) counters when their table fits
-// (`local` = 2^n n entries, else 0: global atomics).
+// ---- cache update by selection ---------------------------------------------------------
+
+__device__ __forceinline__ uint64_t cache_key(uint64_t seed, int64_t t1, int n, int i, int64_t q,
+                                              int64_t r)
+{
+    return mix64(seed, ((uint64_t)t1 * (uint64_t)n + (uint64_t)i) * (uint64_t)q + (uint64_t)r);
+}
+
+// Candidates of worker i: rows it caches outside its new set.  Counts per
+// (worker, top kCBits key bits) (hist zero on entry).
+__global__ void cand_hist_kernel(int64_t q, int n, int64_t t1, uint64_t seed,
+                                 const int32_t *owner1, const uint64_t *cached0, int32_t *hist)
+{
+    GS_LOOP(r, q)
+    {
+        for (uint64_t b = cached0[r] & ~(1ull << owner1[r]); b; b &= b - 1) {
+            const int i = __ffsll((long long)b) - 1;
+            const uint64_t k = cache_key(seed, t1, n, i, q, r);
+            atomicAdd(&hist[((int64_t)i << kCBits) + (int64_t)(k >> (64 - kCBits))], 1);
+        }
+    }
+}
+
+// One block per worker: the bucket that holds its keep-th candidate (thr)
+// and how many of that bucket's candidates it keeps (need); thr = 2^kCBits
+// when it keeps all, -1 when it keeps none.
+__global__ void __launch_bounds__(1024) cand_threshold_kernel(const int32_t *hist, int64_t keep,
+                                                              int32_t *thr, int32_t *need)
+{
+    constexpr int kPer = (1 << kCBits) / 1024;
+    __shared__ int32_t wsum[32];
+    const int i = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int32_t *h = hist + ((int64_t)i << kCBits) + (int64_t)threadIdx.x * kPer;
+    int32_t sum = 0;
+    for (int j = 0; j < kPer; ++j) sum += h[j];
+    int32_t inc = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
+    }
+    if (lane == 31) wsum[warp] = inc;
+    __syncthreads();
+    int32_t before = 0, total = 0;
+    for (int w = 0; w < 32; ++w) {
+        before += w < warp ? wsum[w] : 0;
+        total += wsum[w];
+    }
+    const int64_t excl = before + inc - sum;
+    if (threadIdx.x == 0) {
+        if (keep <= 0) {
+            thr[i] = -1;
+            need[i] = 0;
+        } else if (total <= keep) {
+            thr[i] = 1 << kCBits;
+            need[i] = 0;
+        }
+    }
+    if (keep > 0 && total > keep && excl < keep && keep <= excl + sum) {
+        int64_t c = excl;   // the thread whose buckets hold the keep-th candidate
+        for (int j = 0; j < kPer; ++j) {
+            if (c + h[j] >= keep) {
+                thr[i] = (int32_t)(threadIdx.x * kPer + j);
+                need[i] = (int32_t)(keep - c);
+                break;
+            }
+            c += h[j];
+        }
+    }
+}
+
+// Candidates below their worker's bucket are kept (bits added to the new
+// cache mask); those in it are listed.
+__global__ void cand_classify_kernel(int64_t q, int n, int64_t t1, uint64_t seed,
+                                     const int32_t *owner1, const uint64_t *cached0,
+                                     const int32_t *thr, uint64_t *next, int32_t *lw,
+                                     int32_t *lr, uint64_t *lk, int32_t *nlist)
+{
+    __shared__ int32_t sthr[kMaxDeviceN];
+    if (threadIdx.x < n) sthr[threadIdx.x] = thr[threadIdx.x];
+    __syncthreads();
+    GS_LOOP(r, q)
+    {
+        uint64_t add = 0;
+        for (uint64_t b = cached0[r] & ~(1ull << owner1[r]); b; b &= b - 1) {
+            const int i = __ffsll((long long)b) - 1;
+            const uint64_t k = cache_key(seed, t1, n, i, q, r);
+            const int64_t bk = (int64_t)(k >> (64 - kCBits));
+            if (bk < sthr[i]) {
+                add |= 1ull << i;
+            } else if (bk == sthr[i]) {
+                const int32_t x = atomicAdd(nlist, 1);
+                lw[x] = i;
+                lr[x] = (int32_t)r;
+                lk[x] = k;
+            }
+        }
+        if (add) next[r] |= add;
+    }
+}
+
+// A listed candidate is kept if fewer than need[i] listed candidates of its
+// worker come before it in (key, row) order.
+__global__ void cand_rank_kernel(const int32_t *nlist, const int32_t *lw, const int32_t *lr,
+                                 const uint64_t *lk, const int32_t *need,
+                                 unsigned long long *next)
+{
+    const int64_t m = *nlist;
+    GS_LOOP(x, m)
+    {
+        const int i = lw[x];
+        const int32_t r = lr[x];
+        const uint64_t k = lk[x];
+        int64_t rank = 0;
+        for (int64_t y = 0; y < m; ++y)
+            if (lw[y] == i && (lk[y] < k || (lk[y] == k && lr[y] < r))) ++rank;
+        if (rank < need[i]) atomicOr(&next[r], 1ull << i);
+    }
+}
+
+// Per row: missing from its new owner's cache?  Its set I; counts per
+// (I, worker) and per worker.  The per-worker counters are aggregated in
+// shared memory per block, and so are the (I, worker) counters when their
+// table fits (`local` = 2^n n entries, else 0: global atomics).  The new
+// cache masks start as the owner's bit.
 __global__ void need_kernel(int64_t q, int n, const int32_t *owner1, const uint64_t *cached0,
-                            uint64_t *rmask, int32_t *needflag, int32_t *ccnt_row, uint64_t *next,
-                            int32_t *counts, int32_t *wcount, int32_t *ccount, int local)
+                            uint64_t *rmask, int32_t *needflag, uint64_t *next, int32_t *counts,
+                            int32_t *wcount, int local)
 {
     extern __shared__ int32_t sl[];
-    __shared__ int32_t sw[kMaxDeviceN], sc[kMaxDeviceN];
-    if (threadIdx.x < kMaxDeviceN) {
-        sw[threadIdx.x] = 0;
-        sc[threadIdx.x] = 0;
-    }
+    __shared__ int32_t sw[kMaxDeviceN];
+    if (threadIdx.x < kMaxDeviceN) sw[threadIdx.x] = 0;
     for (int i = threadIdx.x; i < local; i += blockDim.x) sl[i] = 0;
     __syncthreads();
     GS_LOOP(r, q)
@@ -371,24 +630,18 @@ __global__ void need_kernel(int64_t q, int n, const int32_t *owner1, const uint6
         const int i = owner1[r];
         const uint64_t bit = 1ull << i, have = cached0[r];
         const int nf = (have & bit) ? 0 : 1;
-        const uint64_t cand = have & ~bit;
         needflag[r] = nf;
         rmask[r] = have | bit;
         next[r] = bit;
-        ccnt_row[r] = __popcll(cand);
         if (nf) {
             const int64_t slot = (int64_t)(have | bit) * n + i;
             if (local) atomicAdd(&sl[slot], 1);
             else atomicAdd(&counts[slot], 1);
             atomicAdd(&sw[i], 1);
         }
-        for (uint64_t b = cand; b; b &= b - 1) atomicAdd(&sc[__ffsll((long long)b) - 1], 1);
     }
     __syncthreads();
-    if (threadIdx.x < n) {
-        atomicAdd(&wcount[threadIdx.x], sw[threadIdx.x]);
-        atomicAdd(&ccount[threadIdx.x], sc[threadIdx.x]);
-    }
+    if (threadIdx.x < n) atomicAdd(&wcount[threadIdx.x], sw[threadIdx.x]);
     for (int i = threadIdx.x; i < local; i += blockDim.x)
         if (sl[i]) atomicAdd(&counts[i], sl[i]);
 }
@@ -515,92 +768,6 @@ __global__ void decslot_kernel(const int32_t *Rp, int64_t q, int64_t s, const in
     }
 }
 
-__global__ void cand_kernel(int64_t q, int n, int64_t t1, uint64_t seed, const int32_t *owner1,
-                            const uint64_t *cached0, const int32_t *cbase, int32_t *cw,
-                            int32_t *cr, uint64_t *ckey, uint64_t *keys, int32_t *vals)
-{
-    GS_LOOP(r, q)
-    {
-        uint64_t b = cached0[r] & ~(1ull << owner1[r]);
-        int32_t c = cbase[r];
-        for (; b; b &= b - 1, ++c) {
-            const int i = __ffsll((long long)b) - 1;
-            cw[c] = i;
-            cr[c] = (int32_t)r;
-            keys[c] = mix64(seed, ((uint64_t)t1 * (uint64_t)n + (uint64_t)i) * (uint64_t)q +
-                                      (uint64_t)r);
-            ckey[c] = keys[c];
-            vals[c] = c;
-        }
-    }
-}
-
-__global__ void cand_worker_keys_kernel(const int32_t *Kp, const int32_t *vals, const int32_t *cw,
-                                        uint64_t *keys)
-{
-    const int64_t K = *Kp;
-    GS_LOOP(p, K) keys[p] = (uint64_t)cw[vals[p]];
-}
-
-// After a stable sort on the top 24 bits of the keys only, items whose top
-// bits tie are adjacent and in their original order; each such run (short:
-// keys are uniform 64-bit values) is put in full (key, row) order by the
-// thread at its start.  `grp` (nullable) adds a group that must also tie
-// (the worker of a candidate); keys and rows are read through the values
-// (`key_of`, `row_of`: item id -> key / row; null: the sorted key array and
-// the value itself).
-__global__ void fixup_runs_kernel(const int32_t *countp, int64_t cap, const uint64_t *skeys,
-                                  int32_t *vals, const uint64_t *key_of, const int32_t *row_of,
-                                  const int32_t *grp)
-{
-    const int64_t count = countp ? (int64_t)*countp : cap;
-    auto key = [&](int32_t v, int64_t p) { return key_of ? key_of[v] : skeys[p]; };
-    auto row = [&](int32_t v) { return row_of ? row_of[v] : v; };
-    auto top = [&](int32_t v, int64_t p) {
-        return ((key(v, p) >> 40) << 8) | (uint64_t)(grp ? grp[v] : 0);
-    };
-    GS_LOOP(p, count)
-    {
-        const int32_t v0 = vals[p];
-        const uint64_t t0 = top(v0, p);
-        if (p > 0 && top(vals[p - 1], p - 1) == t0) continue;   // not a run start
-        int64_t e = p + 1;
-        while (e < count && top(vals[e], e) == t0) ++e;
-        if (e - p < 2) continue;
-        // insertion sort of vals[p, e) by (key, row); with key_of null the
-        // keys move with the values
-        for (int64_t i = p + 1; i < e; ++i) {
-            const int32_t vi = vals[i];
-            const uint64_t ki = key_of ? key_of[vi] : skeys[i];
-            const int32_t ri = row(vi);
-            int64_t j = i - 1;
-            while (j >= p) {
-                const int32_t vj = vals[j];
-                const uint64_t kj = key_of ? key_of[vj] : skeys[j];
-                if (kj < ki || (kj == ki && row(vj) < ri)) break;
-                vals[j + 1] = vj;
-                if (!key_of) const_cast<uint64_t *>(skeys)[j + 1] = kj;
-                --j;
-            }
-            vals[j + 1] = vi;
-            if (!key_of) const_cast<uint64_t *>(skeys)[j + 1] = ki;
-        }
-    }
-}
-
-__global__ void kept_kernel(const int32_t *Kp, int64_t keep, const int32_t *vals,
-                            const int32_t *cw, const int32_t *cr, const int32_t *cstart,
-                            unsigned long long *next)
-{
-    const int64_t K = *Kp;
-    GS_LOOP(p, K)
-    {
-        const int32_t c = vals[p];
-        const int i = cw[c];
-        if (p - cstart[i] < keep) atomicOr(&next[cr[c]], 1ull << i);
-    }
-}
-
 __global__ void evflag_kernel(int64_t ns, int64_t s, const int32_t *slot_row,
                               const uint64_t *next, int32_t *evflag)
 {
@@ -649,12 +816,16 @@ __global__ void check_kernel(int n, int64_t s, const int32_t *evrank, const int3
 struct DevLayout {
     ShuffleLayout prog;       // the row programs, at the start (word offsets)
     int64_t owner[2], cached[2], slot_of;
-    int64_t kA, kB, vA, vB, hist, scan;
+    int64_t kA, kB, vA, vB, flags, scan;
     int64_t rmask, needflag, idx, items, recv_row, wcount, recv_ptr;
     int64_t counts, runstart, ell, msgbase, earr, msg_set, msg_worker, dx;
-    int64_t ccnt_row, cbase, cw, cr, ckey, ccount, cstart, evflag, evrank, totals;
+    int64_t cw, cr, ckey, evflag, evrank, totals;
+    int64_t sel, pstart;      // selection histograms (partition, then cache update); scan
+    int64_t flags_bytes;      // radix tile flags
     int64_t bytes;            // total
     int64_t capK, nm;
+    int pbits;                // bucket bits of the partition selection
+    int64_t sel_words;        // 2^pbits + n 2^kCBits
 };
 
 DevLayout device_layout(int32_t n, int64_t q, int64_t s)
@@ -664,8 +835,13 @@ DevLayout device_layout(int32_t n, int64_t q, int64_t s)
     D.nm = (int64_t)1 << n;
     const int64_t ns = (int64_t)n * s;
     D.capK = std::max(q, ns);
-    const int64_t tiles = std::max<int64_t>(1, (D.capK + kTile - 1) / kTile);
-    const int64_t scan_max = std::max({256 * tiles, D.capK + 1, D.nm * n + 1, q + 1});
+    const int64_t tiles = std::max<int64_t>(1, (q + kTile - 1) / kTile);
+    // about two rows per partition bucket
+    int lg = 0;
+    while (((int64_t)1 << lg) < q) ++lg;
+    D.pbits = std::min(20, std::max(8, lg - 1));
+    D.sel_words = ((int64_t)1 << D.pbits) + ((int64_t)n << kCBits);
+    const int64_t scan_max = std::max({D.nm * n + 1, q + 1, (int64_t)1 << D.pbits, ns + 1});
     int64_t at = up256(D.prog.total * 4);
     auto take = [&](int64_t bytes) {
         const int64_t off = at;
@@ -677,11 +853,12 @@ DevLayout device_layout(int32_t n, int64_t q, int64_t s)
     D.cached[0] = take(8 * q);
     D.cached[1] = take(8 * q);
     D.slot_of = take(4 * (int64_t)n * q);
-    D.kA = take(8 * D.capK);
-    D.kB = take(8 * D.capK);
-    D.vA = take(4 * D.capK);
-    D.vB = take(4 * D.capK);
-    D.hist = take(4 * 256 * tiles);
+    D.kA = take(8 * q);
+    D.kB = take(8 * q);
+    D.vA = take(4 * q);
+    D.vB = take(4 * q);
+    D.flags_bytes = 8 * 256 * tiles;
+    D.flags = take(D.flags_bytes);
     D.scan = take(4 * (scan_max / kScanItems + 8 * 256 + 1024));
     D.rmask = take(8 * q);
     D.needflag = take(4 * (q + 1));
@@ -698,16 +875,14 @@ DevLayout device_layout(int32_t n, int64_t q, int64_t s)
     D.msg_set = take(8 * q);
     D.msg_worker = take(4 * q);
     D.dx = take(4 * (q + 1));
-    D.ccnt_row = take(4 * (q + 1));
-    D.cbase = take(4 * (q + 1));
     D.cw = take(4 * D.capK);
     D.cr = take(4 * D.capK);
     D.ckey = take(8 * D.capK);
-    D.ccount = take(4 * (n + 1));
-    D.cstart = take(4 * (n + 1));
+    D.sel = take(4 * D.sel_words);
+    D.pstart = take(4 * ((int64_t)1 << D.pbits));
     D.evflag = take(4 * (ns + 1));
     D.evrank = take(4 * (ns + 1));
-    D.totals = take(4 * T_COUNT);
+    D.totals = take(4 * kTotalsWords);
     D.bytes = at;
     return D;
 }
@@ -750,10 +925,14 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     int32_t *totals = ptr<int32_t>(ws, D.totals);
     int32_t *scan = ptr<int32_t>(ws, D.scan);
     SortBufs sb{ptr<uint64_t>(ws, D.kA), ptr<uint64_t>(ws, D.kB), ptr<int32_t>(ws, D.vA),
-                ptr<int32_t>(ws, D.vB), ptr<int32_t>(ws, D.hist), scan};
+                ptr<int32_t>(ws, D.vB),           ptr<uint64_t>(ws, D.flags),
+                totals + kGhist,                  totals + kCtr,
+                totals + T_ERR,                   &S->sort_epoch};
     int32_t *counts = ptr<int32_t>(ws, D.counts), *wcount = ptr<int32_t>(ws, D.wcount);
-    int32_t *ccount = ptr<int32_t>(ws, D.ccount), *ell = ptr<int32_t>(ws, D.ell);
+    int32_t *ell = ptr<int32_t>(ws, D.ell);
     int32_t *dx = ptr<int32_t>(ws, D.dx);
+    int32_t *phist = ptr<int32_t>(ws, D.sel), *pstart = ptr<int32_t>(ws, D.pstart);
+    int32_t *chist = phist + ((int64_t)1 << D.pbits);
     cudaError_t e;
 #define CK(x)                                      \
     do {                                           \
@@ -761,33 +940,34 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     } while (0)
 #define LAUNCHED() CK(cudaGetLastError())
 
-    fill_i32<<<1, 32, 0, s>>>(totals, T_COUNT, 0);
+    fill_i32<<<grid_for(kTotalsWords), 256, 0, s>>>(totals, kTotalsWords, 0);
     fill_i32<<<grid_for(nm * n + 1), 256, 0, s>>>(counts, nm * n + 1, 0);
     fill_i32<<<1, 32, 0, s>>>(wcount, n + 1, 0);
-    fill_i32<<<1, 32, 0, s>>>(ccount, n + 1, 0);
     fill_i32<<<grid_for(nm + 1), 256, 0, s>>>(ell, nm + 1, 0);
     fill_i32<<<grid_for(q + 1), 256, 0, s>>>(dx, q + 1, 0);
+    fill_i32<<<grid_for(D.sel_words), 256, 0, s>>>(phist, D.sel_words, 0);
     LAUNCHED();
 
-    // partition: rows sorted by (key, row)
-    partition_keys_kernel<<<grid_for(q), 256, 0, s>>>(sb.kA, sb.vA, q, S->partition_seed, t1);
+    // partition: owner = rank in (key, row) order / (q/n), by selection
+    part_hist_kernel<<<grid_for(q), 256, 0, s>>>(q, S->partition_seed, t1, D.pbits, phist);
+    LAUNCHED();
+    CK(scan_exclusive(phist, pstart, (int64_t)1 << D.pbits, scan, totals + T_DUMMY, s));
+    part_owner_kernel<<<grid_for(q), 256, 0, s>>>(q, S->partition_seed, t1, D.pbits, S->per,
+                                                  phist, pstart, owner1, sb.vA, totals + kListP);
+    LAUNCHED();
+    part_rank_kernel<<<64, 256, 0, s>>>(q, S->partition_seed, t1, D.pbits, S->per,
+                                                 pstart, sb.vA, totals + kListP, owner1);
+    LAUNCHED();
+
+    // missing rows, their sets and the counters
+    uint64_t *rmask = ptr<uint64_t>(ws, D.rmask);
+    int32_t *needflag = ptr<int32_t>(ws, D.needflag), *idx = ptr<int32_t>(ws, D.idx);
+    const int local = nm * n <= 8192 ? (int)(nm * n) : 0;   // 32 KB of shared counters
+    need_kernel<<<grid_for(q), 256, sizeof(int32_t) * local, s>>>(
+        q, n, owner1, cached0, rmask, needflag, next, counts, wcount, local);
     LAUNCHED();
     uint64_t *ko;
     int32_t *vo;
-    CK(radix_sort(sb, nullptr, q, 40, 64, s, &ko, &vo));   // top 24 bits, then the ties
-    fixup_runs_kernel<<<grid_for(q), 256, 0, s>>>(nullptr, q, ko, vo, nullptr, nullptr, nullptr);
-    LAUNCHED();
-    owner_kernel<<<grid_for(q), 256, 0, s>>>(vo, q, S->per, owner1);
-    LAUNCHED();
-
-    // missing rows, their sets, the refill candidates and the counters
-    uint64_t *rmask = ptr<uint64_t>(ws, D.rmask);
-    int32_t *needflag = ptr<int32_t>(ws, D.needflag), *idx = ptr<int32_t>(ws, D.idx);
-    int32_t *ccnt_row = ptr<int32_t>(ws, D.ccnt_row), *cbase = ptr<int32_t>(ws, D.cbase);
-    const int local = nm * n <= 8192 ? (int)(nm * n) : 0;   // 32 KB of shared counters
-    need_kernel<<<grid_for(q), 256, sizeof(int32_t) * local, s>>>(
-        q, n, owner1, cached0, rmask, needflag, ccnt_row, next, counts, wcount, ccount, local);
-    LAUNCHED();
     CK(scan_exclusive(needflag, idx, q, scan, totals + T_R, s));
     int32_t *items = ptr<int32_t>(ws, D.items);
     compact_kernel<<<grid_for(q), 256, 0, s>>>(q, needflag, idx, items);
@@ -797,7 +977,7 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     int32_t *recv_row = ptr<int32_t>(ws, D.recv_row), *recv_ptr = ptr<int32_t>(ws, D.recv_ptr);
     worker_keys_kernel<<<grid_for(q), 256, 0, s>>>(totals + T_R, items, owner1, sb.kA, sb.vA);
     LAUNCHED();
-    CK(radix_sort(sb, totals + T_R, q, 0, 8, s, &ko, &vo));
+    CK(radix_sort(sb, totals + T_R, q, 0, 8, 0, s, &ko, &vo));
     copy_i32_counted<<<grid_for(q), 256, 0, s>>>(totals + T_R, vo, recv_row);
     LAUNCHED();
     CK(scan_exclusive(wcount, recv_ptr, n + 1, scan, totals + T_DUMMY, s));
@@ -805,7 +985,7 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     // message order: (I, worker, row)
     mask_keys_kernel<<<grid_for(q), 256, 0, s>>>(totals + T_R, recv_row, rmask, sb.kA, sb.vA);
     LAUNCHED();
-    CK(radix_sort(sb, totals + T_R, q, 0, (n + 7) / 8 * 8, s, &ko, &vo));
+    CK(radix_sort(sb, totals + T_R, q, 0, (n + 7) / 8 * 8, 1, s, &ko, &vo));
     const int32_t *P = vo;
     int32_t *runstart = ptr<int32_t>(ws, D.runstart), *msgbase = ptr<int32_t>(ws, D.msgbase);
     CK(scan_exclusive(counts, runstart, nm * n + 1, scan, totals + T_DUMMY, s));
@@ -835,32 +1015,19 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
                                                totals + T_ERR);
     LAUNCHED();
 
-    // cache update rule: candidates by (worker, key, row); the first s - q/n kept
-    CK(scan_exclusive(ccnt_row, cbase, q, scan, totals + T_K, s));
+    // cache update rule: the s - q/n candidates of smallest (key, row) of
+    // every worker kept, by selection
     int32_t *cw = ptr<int32_t>(ws, D.cw), *cr = ptr<int32_t>(ws, D.cr);
     uint64_t *ckey = ptr<uint64_t>(ws, D.ckey);
-    cand_kernel<<<grid_for(q), 256, 0, s>>>(q, n, t1, S->cache_seed, owner1, cached0, cbase, cw,
-                                            cr, ckey, sb.kA, sb.vA);
+    cand_hist_kernel<<<grid_for(q), 256, 0, s>>>(q, n, t1, S->cache_seed, owner1, cached0, chist);
     LAUNCHED();
-    // by the top 24 bits of the key, then by worker (both stable), then each
-    // run of equal (worker, top bits) in full (key, row) order
-    CK(radix_sort(sb, totals + T_K, D.capK, 40, 64, s, &ko, &vo));
-    {
-        // the sort leaves its result in A or B: move it to A for the next one
-        if (vo != sb.vA) {
-            copy_i32_counted<<<grid_for(D.capK), 256, 0, s>>>(totals + T_K, vo, sb.vA);
-            LAUNCHED();
-        }
-        cand_worker_keys_kernel<<<grid_for(D.capK), 256, 0, s>>>(totals + T_K, sb.vA, cw, sb.kA);
-        LAUNCHED();
-    }
-    CK(radix_sort(sb, totals + T_K, D.capK, 0, 8, s, &ko, &vo));
-    fixup_runs_kernel<<<grid_for(D.capK), 256, 0, s>>>(totals + T_K, D.capK, ko, vo, ckey, cr,
-                                                        cw);
+    cand_threshold_kernel<<<n, 1024, 0, s>>>(chist, sz - S->per, totals + kThr, totals + kNeed);
     LAUNCHED();
-    int32_t *cstart = ptr<int32_t>(ws, D.cstart);
-    CK(scan_exclusive(ccount, cstart, n + 1, scan, totals + T_DUMMY, s));
-    kept_kernel<<<grid_for(D.capK), 256, 0, s>>>(totals + T_K, sz - S->per, vo, cw, cr, cstart,
+    cand_classify_kernel<<<grid_for(q), 256, 0, s>>>(q, n, t1, S->cache_seed, owner1, cached0,
+                                                     totals + kThr, next, cw, cr, ckey,
+                                                     totals + kListC);
+    LAUNCHED();
+    cand_rank_kernel<<<64, 256, 0, s>>>(totals + kListC, cw, cr, ckey, totals + kNeed,
                                                  reinterpret_cast<unsigned long long *>(next));
     LAUNCHED();
 
@@ -935,6 +1102,10 @@ cm_status cm_shuffle_device_init(cm_shuffle *S, void *ws, size_t bytes, cm_strea
         e = put(ptr<int32_t>(ws, D.slot_of), S->slot_of.data(), 4 * (int64_t)S->n * q, s);
     if (e == cudaSuccess)
         e = put(prog(ws, D.prog.fill_row), S->slot_row.data(), 4 * S->slot_row.size(), s);
+    // radix tile flags (tagged by S->sort_epoch) and the counters
+    if (e == cudaSuccess)
+        e = cudaMemsetAsync(ptr<unsigned char>(ws, D.flags), 0, D.flags_bytes, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(ptr<int32_t>(ws, D.totals), 0, 4 * kTotalsWords, s);
     if (e == cudaSuccess && S->planned) {   // the current transition's programs and tables
         e = put(prog(ws, D.prog.enc_ptr), S->enc_ptr.data(), 4 * S->enc_ptr.size(), s);
         if (e == cudaSuccess) e = put(prog(ws, D.prog.enc_src), S->enc_src.data(), 4 * S->enc_src.size(), s);
@@ -952,6 +1123,7 @@ cm_status cm_shuffle_device_init(cm_shuffle *S, void *ws, size_t bytes, cm_strea
     if (e != cudaSuccess) return CM_ECUDA;
     S->device_ws = ws;
     S->dev_cur = 0;
+    S->sort_epoch = 0;
     S->uploaded_ws = ws;
     S->uploaded_t = S->t;
     return CM_OK;

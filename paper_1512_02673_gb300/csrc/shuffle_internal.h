@@ -46,6 +46,7 @@ struct cm_shuffle {
     // the current copy of the double-buffered partition and cache masks.
     void *device_ws = nullptr;
     int dev_cur = 0;
+    uint32_t sort_epoch = 0;           // tag of the device radix passes' tile flags
 };
 
 ShuffleLayout shuffle_layout(int32_t n, int64_t q, int64_t s);

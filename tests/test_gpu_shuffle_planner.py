@@ -60,7 +60,9 @@ def _same_plan(cm, h, d, n, q, s):
 
 @pytest.mark.parametrize("n,q,s", [(2, 40, 20), (3, 600, 300), (4, 4000, 1700), (5, 1500, 300),
                                    (8, 8000, 2000), (4, 120, 120), (16, 3200, 800),
-                                   (6, 6000, 2500)])
+                                   (6, 6000, 2500),
+                                   (4, 400, 100),    # s = q/n: the cache keeps no candidate
+                                   (16, 32, 3)])     # q/n = 2: most partition buckets straddle
 def test_device_plans_equal_host_plans(cm, n, q, s):
     h = cm.Shuffle(n, q, s, 23, 29)
     d = cm.Shuffle(n, q, s, 23, 29)

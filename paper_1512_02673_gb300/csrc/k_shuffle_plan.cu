@@ -96,15 +96,71 @@ unsigned grid_for(int64_t items)
 
 __global__ void fill_i32(int32_t *p, int64_t count, int32_t v) { GS_LOOP(i, count) p[i] = v; }
 
+// Zero up to 8 int32 regions in one launch.
+struct ZeroList {
+    int32_t *p[8];
+    int64_t n[8];
+    int k;
+};
+
+__global__ void zero_many_kernel(const ZeroList z)
+{
+    for (int r = 0; r < z.k; ++r) GS_LOOP(i, z.n[r]) z.p[r][i] = 0;
+}
+
+// ---- tile flags of the decoupled look-backs --------------------------------------------
+
+// epoch (30 bits) << 34 | status << 32 | 32-bit value.  A flag whose epoch is
+// not the running pass's has not been published yet; flags are never cleared.
+constexpr uint64_t kFlagAgg = 1, kFlagInc = 2;   // the tile's own sum / its inclusive prefix
+constexpr uint32_t kEpochMask = 0x3fffffffu;
+constexpr int kLook = 16;   // tiles read together by one step of a radix look-back
+
+__device__ __forceinline__ uint64_t flag_word(uint32_t epoch, uint64_t status, int32_t v)
+{
+    return ((uint64_t)(epoch & kEpochMask) << 34) | (status << 32) | (uint64_t)(uint32_t)v;
+}
+__device__ __forceinline__ bool flag_ready(uint64_t w, uint32_t epoch)
+{
+    return (uint32_t)(w >> 34) == (epoch & kEpochMask);
+}
+__device__ __forceinline__ uint64_t flag_status(uint64_t w) { return (w >> 32) & 3u; }
+__device__ __forceinline__ int32_t flag_value(uint64_t w) { return (int32_t)(uint32_t)w; }
+
+// Flags, epochs and counters shared by the look-back kernels of a planner
+// workspace; the kernels run one after another on one stream.
+struct LookBack {
+    uint64_t *flags;
+    int64_t nflags;
+    int32_t *ctr;     // [0]: next tile, [1]: finished blocks (reset by the last one)
+    int32_t *err;     // set on a look-back time-out
+    uint32_t *epoch;  // host counter, one value per launch
+};
+
+uint32_t next_epoch(uint32_t *e)
+{
+    if (((++*e) & kEpochMask) == 0) ++*e;   // epoch 0 is the cleared flag
+    return *e;
+}
+
 // ---- exclusive scan (int32) -----------------------------------------------------------
 
-__global__ void __launch_bounds__(kScanBlock) scan_block_kernel(const int32_t *in, int32_t *out,
-                                                                int64_t count,
-                                                                int32_t *block_sums)
+// One pass: tiles of 4096 items in the order of an atomic counter; a tile
+// scans itself, publishes its sum, and warp 0 looks back over the flags of
+// the 32 tiles before it at a time for its prefix (bounded waits).
+__global__ void __launch_bounds__(kScanBlock) scan_kernel(const int32_t *in, int32_t *out,
+                                                          int64_t count, int32_t *total,
+                                                          uint64_t *flags, uint32_t epoch,
+                                                          int32_t *ctr, int32_t *err)
 {
     __shared__ int32_t warp_sums[32];
+    __shared__ int32_t s_tile, s_prefix;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int64_t base = (int64_t)blockIdx.x * kScanItems + 4 * (int64_t)threadIdx.x;
+    const bool multi = gridDim.x > 1;
+    if (threadIdx.x == 0) s_tile = multi ? atomicAdd(&ctr[0], 1) : 0;
+    __syncthreads();
+    const int64_t tile = s_tile;
+    const int64_t base = tile * kScanItems + 4 * (int64_t)threadIdx.x;
     int32_t v[4], sum = 0;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
@@ -126,63 +182,67 @@ __global__ void __launch_bounds__(kScanBlock) scan_block_kernel(const int32_t *i
             const int32_t y = __shfl_up_sync(0xffffffffu, w, o);
             if (lane >= o) w += y;
         }
-        warp_sums[lane] = w;
+        warp_sums[lane] = w;   // inclusive over the warps; [31] = the tile's sum
+        const int32_t agg = __shfl_sync(0xffffffffu, w, 31);
+        int32_t pre = 0;
+        if (multi) {
+            if (lane == 0)
+                atomicExch(reinterpret_cast<unsigned long long *>(flags + tile),
+                           (unsigned long long)flag_word(epoch, tile ? kFlagAgg : kFlagInc, agg));
+            int64_t t = tile - 1;
+            uint32_t it = 0;
+            while (t >= 0) {
+                const int64_t idx = t - lane;
+                const uint64_t f = idx >= 0 ? *(const volatile uint64_t *)(flags + idx)
+                                            : flag_word(epoch, kFlagInc, 0);
+                const bool ready = flag_ready(f, epoch);
+                const unsigned incm = __ballot_sync(0xffffffffu, ready && flag_status(f) == kFlagInc);
+                const unsigned notready = __ballot_sync(0xffffffffu, !ready);
+                const int last = incm ? __ffs(incm) - 1 : 31;   // lanes [0, last] are summed
+                const unsigned upto = last == 31 ? 0xffffffffu : ((2u << last) - 1u);
+                if (notready & upto) {   // wait (bounded) and read the same tiles again
+                    if (++it > (1u << 21) ||
+                        __any_sync(0xffffffffu, *(volatile int32_t *)err != 0)) {
+                        if (lane == 0) atomicExch(err, 1);
+                        break;
+                    }
+                    __nanosleep(64);
+                    continue;
+                }
+                int32_t part = lane <= last ? flag_value(f) : 0;
+#pragma unroll
+                for (int o = 16; o; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+                pre += part;
+                if (incm) break;
+                t -= 32;
+            }
+            if (lane == 0 && tile > 0)
+                atomicExch(reinterpret_cast<unsigned long long *>(flags + tile),
+                           (unsigned long long)flag_word(epoch, kFlagInc, pre + agg));
+        }
+        if (lane == 0) {
+            s_prefix = pre;
+            if (total && tile == (count - 1) / kScanItems) *total = pre + agg;
+        }
     }
     __syncthreads();
-    int32_t excl = x - sum + (warp ? warp_sums[warp - 1] : 0);
+    int32_t excl = x - sum + (warp ? warp_sums[warp - 1] : 0) + s_prefix;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
         if (base + k < count) out[base + k] = excl;
         excl += v[k];
     }
-    if (threadIdx.x == kScanBlock - 1 && block_sums) block_sums[blockIdx.x] = excl;
-}
-
-__global__ void __launch_bounds__(kScanBlock) scan_add_kernel(int32_t *out, int64_t count,
-                                                              const int32_t *offsets)
-{
-    const int32_t add = offsets[blockIdx.x];
-    const int64_t base = (int64_t)blockIdx.x * kScanItems + 4 * (int64_t)threadIdx.x;
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-        if (base + k < count) out[base + k] += add;
-}
-
-// The second pass when the block sums are few: every block sums the block
-// sums before its own (at most kScanDirect of them, one or a few per thread)
-// instead of waiting for a scan of them in a launch of its own, then adds
-// that offset; the last block also writes the total.
-constexpr int64_t kScanDirect = 4 * kScanBlock;
-
-__global__ void __launch_bounds__(kScanBlock) scan_add_direct_kernel(int32_t *out, int64_t count,
-                                                                     const int32_t *block_sums,
-                                                                     int32_t *total)
-{
-    __shared__ int32_t warp_part[32];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    int32_t part = 0;
-    for (int64_t i = threadIdx.x; i < (int64_t)blockIdx.x; i += kScanBlock) part += block_sums[i];
-#pragma unroll
-    for (int o = 16; o; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-    if (lane == 0) warp_part[warp] = part;
-    __syncthreads();
-    int32_t add = 0;
-#pragma unroll 1
-    for (int w = 0; w < kScanBlock / 32; ++w) add += warp_part[w];
-    const int64_t base = (int64_t)blockIdx.x * kScanItems + 4 * (int64_t)threadIdx.x;
-#pragma unroll
-    for (int k = 0; k < 4; ++k)
-        if (base + k < count) out[base + k] += add;
-    if (total && threadIdx.x == 0 && blockIdx.x == gridDim.x - 1)
-        *total = add + block_sums[blockIdx.x];
+    if (multi && threadIdx.x == 0 && atomicAdd(&ctr[1], 1) == (int32_t)gridDim.x - 1) {
+        ctr[0] = 0;
+        ctr[1] = 0;
+    }
 }
 
 int64_t up256(int64_t x) { return (x + 255) & ~(int64_t)255; }
 
 // out[i] = in[0] + ... + in[i-1] for i < count (in may be out); the sum of
-// all of them goes to *total (device, nullable).  `scratch` holds the block
-// sums of every level (count / 4096 + 512 words per level suffice).
-cudaError_t scan_exclusive(const int32_t *in, int32_t *out, int64_t count, int32_t *scratch,
+// all of them goes to *total (device, nullable).  One launch.
+cudaError_t scan_exclusive(const LookBack &lb, const int32_t *in, int32_t *out, int64_t count,
                            int32_t *total, cudaStream_t s)
 {
     if (count <= 0) {
@@ -190,18 +250,10 @@ cudaError_t scan_exclusive(const int32_t *in, int32_t *out, int64_t count, int32
         return cudaGetLastError();
     }
     const int64_t nb = (count + kScanItems - 1) / kScanItems;
-    if (nb == 1) {
-        scan_block_kernel<<<1, kScanBlock, 0, s>>>(in, out, count, total);
-        return cudaGetLastError();
-    }
-    scan_block_kernel<<<(unsigned)nb, kScanBlock, 0, s>>>(in, out, count, scratch);
-    if (nb <= kScanDirect) {
-        scan_add_direct_kernel<<<(unsigned)nb, kScanBlock, 0, s>>>(out, count, scratch, total);
-        return cudaGetLastError();
-    }
-    cudaError_t e = scan_exclusive(scratch, scratch, nb, scratch + up256(nb), total, s);
-    if (e != cudaSuccess) return e;
-    scan_add_kernel<<<(unsigned)nb, kScanBlock, 0, s>>>(out, count, scratch);
+    if (nb > lb.nflags || nb > INT32_MAX) return cudaErrorInvalidValue;
+    const uint32_t epoch = nb > 1 ? next_epoch(lb.epoch) : 0;
+    scan_kernel<<<(unsigned)nb, kScanBlock, 0, s>>>(in, out, count, total, lb.flags, epoch, lb.ctr,
+                                                    lb.err);
     return cudaGetLastError();
 }
 
@@ -225,15 +277,6 @@ __global__ void __launch_bounds__(256) radix_hist_kernel(const uint64_t *keys,
     __syncthreads();
     for (int t = threadIdx.x; t < passes * 256; t += blockDim.x)
         if (h[t / 256][t % 256]) atomicAdd(&ghist[t], h[t / 256][t % 256]);
-}
-
-// Tile flags of the decoupled look-back: epoch << 32 | status << 30 | value.
-constexpr uint64_t kFlagAgg = 1, kFlagInc = 2;
-constexpr int kLook = 16;   // tiles read together by one step of the look-back
-
-__device__ __forceinline__ uint64_t flag_word(uint32_t epoch, uint64_t status, int32_t v)
-{
-    return ((uint64_t)epoch << 32) | (status << 30) | (uint64_t)(uint32_t)v;
 }
 
 // Exclusive scan over the block's 256 threads (one value each); returns the
@@ -361,11 +404,11 @@ radix_pass_kernel(const uint64_t *kin, const int32_t *vin, uint64_t *kout, int32
 #pragma unroll
                 for (int i = 0; i < kLook; ++i) {
                     if (done || used < kLook) continue;
-                    if ((uint32_t)(w[i] >> 32) != epoch) {
+                    if (!flag_ready(w[i], epoch)) {
                         used = i;   // not yet published: read again from tile t - i
                     } else {
-                        excl += (int32_t)(w[i] & 0x3fffffffu);
-                        if (((w[i] >> 30) & 3u) == kFlagInc) done = true;
+                        excl += flag_value(w[i]);
+                        if (flag_status(w[i]) == kFlagInc) done = true;
                     }
                 }
                 if (done) break;
@@ -404,10 +447,8 @@ radix_pass_kernel(const uint64_t *kin, const int32_t *vin, uint64_t *kout, int32
 struct SortBufs {
     uint64_t *kA, *kB;
     int32_t *vA, *vB;
-    uint64_t *flags;
     int32_t *ghist;   // kSortSlots x kMaxPasses x 256, zero at the start of a transition
-    int32_t *ctr, *err;
-    uint32_t *epoch;
+    LookBack lb;
 };
 
 // Stable sort of items [0, count) (count = *countp, or cap if countp is null)
@@ -421,6 +462,7 @@ cudaError_t radix_sort(const SortBufs &b, const int32_t *countp, int64_t cap, in
     if (passes < 1 || passes > kMaxPasses || slot < 0 || slot >= kSortSlots)
         return cudaErrorInvalidValue;
     const int64_t tiles = std::max<int64_t>(1, (cap + kTile - 1) / kTile);
+    if (tiles * 256 > b.lb.nflags) return cudaErrorInvalidValue;
     int32_t *gh = b.ghist + slot * kMaxPasses * 256;
     uint64_t *ki = b.kA, *ko = b.kB;
     int32_t *vi = b.vA, *vo = b.vB;
@@ -429,9 +471,10 @@ cudaError_t radix_sort(const SortBufs &b, const int32_t *countp, int64_t cap, in
     if (ea != cudaSuccess) return ea;
     radix_hist_kernel<<<grid_for(cap), 256, 0, s>>>(ki, countp, cap, lo, passes, gh);
     for (int p = 0; p < passes; ++p) {
-        const uint32_t epoch = ++*b.epoch;
+        const uint32_t epoch = next_epoch(b.lb.epoch);
         radix_pass_kernel<<<(unsigned)tiles, kSortThreads, kSortSmem, s>>>(
-            ki, vi, ko, vo, countp, cap, lo + 8 * p, gh + p * 256, b.flags, epoch, b.ctr, b.err);
+            ki, vi, ko, vo, countp, cap, lo + 8 * p, gh + p * 256, b.lb.flags, epoch, b.lb.ctr,
+            b.lb.err);
         std::swap(ki, ko);
         std::swap(vi, vo);
     }
@@ -516,30 +559,27 @@ __global__ void cand_hist_kernel(int64_t q, int n, int64_t t1, uint64_t seed,
 
 // One block per worker: the bucket that holds its keep-th candidate (thr)
 // and how many of that bucket's candidates it keeps (need); thr = 2^kCBits
-// when it keeps all, -1 when it keeps none.
+// when it keeps all, -1 when it keeps none.  Warp w sums its 2048 buckets
+// (coalesced), the block scans the 32 sums, and the warp whose range holds
+// the keep-th candidate walks its buckets 32 at a time.
 __global__ void __launch_bounds__(1024) cand_threshold_kernel(const int32_t *hist, int64_t keep,
                                                               int32_t *thr, int32_t *need)
 {
-    constexpr int kPer = (1 << kCBits) / 1024;
+    constexpr int kChunk = (1 << kCBits) / 32;
     __shared__ int32_t wsum[32];
     const int i = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int32_t *h = hist + ((int64_t)i << kCBits) + (int64_t)threadIdx.x * kPer;
+    const int32_t *h = hist + ((int64_t)i << kCBits) + (int64_t)warp * kChunk;
     int32_t sum = 0;
-    for (int j = 0; j < kPer; ++j) sum += h[j];
-    int32_t inc = sum;
+    for (int j = lane; j < kChunk; j += 32) sum += h[j];
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int32_t y = __shfl_up_sync(0xffffffffu, inc, o);
-        if (lane >= o) inc += y;
-    }
-    if (lane == 31) wsum[warp] = inc;
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    if (lane == 0) wsum[warp] = sum;
     __syncthreads();
-    int32_t before = 0, total = 0;
+    int64_t before = 0, total = 0;
     for (int w = 0; w < 32; ++w) {
         before += w < warp ? wsum[w] : 0;
         total += wsum[w];
     }
-    const int64_t excl = before + inc - sum;
     if (threadIdx.x == 0) {
         if (keep <= 0) {
             thr[i] = -1;
@@ -549,15 +589,26 @@ __global__ void __launch_bounds__(1024) cand_threshold_kernel(const int32_t *his
             need[i] = 0;
         }
     }
-    if (keep > 0 && total > keep && excl < keep && keep <= excl + sum) {
-        int64_t c = excl;   // the thread whose buckets hold the keep-th candidate
-        for (int j = 0; j < kPer; ++j) {
-            if (c + h[j] >= keep) {
-                thr[i] = (int32_t)(threadIdx.x * kPer + j);
-                need[i] = (int32_t)(keep - c);
+    if (keep > 0 && total > keep && before < keep && keep <= before + sum) {
+        int64_t run = before;   // candidates in the buckets before this step
+        for (int j = 0; j < kChunk; j += 32) {
+            const int32_t v = h[j + lane];
+            int32_t inc = v;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int32_t y = __shfl_up_sync(0xffffffffu, inc, o);
+                if (lane >= o) inc += y;
+            }
+            const unsigned hit = __ballot_sync(0xffffffffu, run + inc >= keep);
+            if (hit) {
+                const int f = __ffs(hit) - 1;
+                if (lane == f) {
+                    thr[i] = warp * kChunk + j + f;
+                    need[i] = (int32_t)(keep - (run + inc - v));
+                }
                 break;
             }
-            c += h[j];
+            run += __shfl_sync(0xffffffffu, inc, 31);
         }
     }
 }
@@ -816,7 +867,7 @@ __global__ void check_kernel(int n, int64_t s, const int32_t *evrank, const int3
 struct DevLayout {
     ShuffleLayout prog;       // the row programs, at the start (word offsets)
     int64_t owner[2], cached[2], slot_of;
-    int64_t kA, kB, vA, vB, flags, scan;
+    int64_t kA, kB, vA, vB, flags;
     int64_t rmask, needflag, idx, items, recv_row, wcount, recv_ptr;
     int64_t counts, runstart, ell, msgbase, earr, msg_set, msg_worker, dx;
     int64_t cw, cr, ckey, evflag, evrank, totals;
@@ -857,9 +908,9 @@ DevLayout device_layout(int32_t n, int64_t q, int64_t s)
     D.kB = take(8 * q);
     D.vA = take(4 * q);
     D.vB = take(4 * q);
-    D.flags_bytes = 8 * 256 * tiles;
+    // tile flags: a radix pass's 256 per tile, or a scan's one per 4096 items
+    D.flags_bytes = 8 * std::max(256 * tiles, scan_max / kScanItems + 1);
     D.flags = take(D.flags_bytes);
-    D.scan = take(4 * (scan_max / kScanItems + 8 * 256 + 1024));
     D.rmask = take(8 * q);
     D.needflag = take(4 * (q + 1));
     D.idx = take(4 * (q + 1));
@@ -923,11 +974,10 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     int32_t *slot_of = ptr<int32_t>(ws, D.slot_of);
     int32_t *slot_row = prog(ws, D.prog.fill_row);
     int32_t *totals = ptr<int32_t>(ws, D.totals);
-    int32_t *scan = ptr<int32_t>(ws, D.scan);
+    const LookBack lb{ptr<uint64_t>(ws, D.flags), D.flags_bytes / 8, totals + kCtr,
+                      totals + T_ERR, &S->sort_epoch};
     SortBufs sb{ptr<uint64_t>(ws, D.kA), ptr<uint64_t>(ws, D.kB), ptr<int32_t>(ws, D.vA),
-                ptr<int32_t>(ws, D.vB),           ptr<uint64_t>(ws, D.flags),
-                totals + kGhist,                  totals + kCtr,
-                totals + T_ERR,                   &S->sort_epoch};
+                ptr<int32_t>(ws, D.vB), totals + kGhist, lb};
     int32_t *counts = ptr<int32_t>(ws, D.counts), *wcount = ptr<int32_t>(ws, D.wcount);
     int32_t *ell = ptr<int32_t>(ws, D.ell);
     int32_t *dx = ptr<int32_t>(ws, D.dx);
@@ -940,18 +990,19 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     } while (0)
 #define LAUNCHED() CK(cudaGetLastError())
 
-    fill_i32<<<grid_for(kTotalsWords), 256, 0, s>>>(totals, kTotalsWords, 0);
-    fill_i32<<<grid_for(nm * n + 1), 256, 0, s>>>(counts, nm * n + 1, 0);
-    fill_i32<<<1, 32, 0, s>>>(wcount, n + 1, 0);
-    fill_i32<<<grid_for(nm + 1), 256, 0, s>>>(ell, nm + 1, 0);
-    fill_i32<<<grid_for(q + 1), 256, 0, s>>>(dx, q + 1, 0);
-    fill_i32<<<grid_for(D.sel_words), 256, 0, s>>>(phist, D.sel_words, 0);
-    LAUNCHED();
+    {
+        int32_t *evflag_end = ptr<int32_t>(ws, D.evflag) + ns;
+        const ZeroList z{{totals, counts, wcount, ell, dx, phist, evflag_end},
+                         {kTotalsWords, nm * n + 1, n + 1, nm + 1, q + 1, D.sel_words, 1},
+                         7};
+        zero_many_kernel<<<grid_for(D.sel_words + q), 256, 0, s>>>(z);
+        LAUNCHED();
+    }
 
     // partition: owner = rank in (key, row) order / (q/n), by selection
     part_hist_kernel<<<grid_for(q), 256, 0, s>>>(q, S->partition_seed, t1, D.pbits, phist);
     LAUNCHED();
-    CK(scan_exclusive(phist, pstart, (int64_t)1 << D.pbits, scan, totals + T_DUMMY, s));
+    CK(scan_exclusive(lb, phist, pstart, (int64_t)1 << D.pbits, totals + T_DUMMY, s));
     part_owner_kernel<<<grid_for(q), 256, 0, s>>>(q, S->partition_seed, t1, D.pbits, S->per,
                                                   phist, pstart, owner1, sb.vA, totals + kListP);
     LAUNCHED();
@@ -968,7 +1019,7 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     LAUNCHED();
     uint64_t *ko;
     int32_t *vo;
-    CK(scan_exclusive(needflag, idx, q, scan, totals + T_R, s));
+    CK(scan_exclusive(lb, needflag, idx, q, totals + T_R, s));
     int32_t *items = ptr<int32_t>(ws, D.items);
     compact_kernel<<<grid_for(q), 256, 0, s>>>(q, needflag, idx, items);
     LAUNCHED();
@@ -980,7 +1031,7 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     CK(radix_sort(sb, totals + T_R, q, 0, 8, 0, s, &ko, &vo));
     copy_i32_counted<<<grid_for(q), 256, 0, s>>>(totals + T_R, vo, recv_row);
     LAUNCHED();
-    CK(scan_exclusive(wcount, recv_ptr, n + 1, scan, totals + T_DUMMY, s));
+    CK(scan_exclusive(lb, wcount, recv_ptr, n + 1, totals + T_DUMMY, s));
 
     // message order: (I, worker, row)
     mask_keys_kernel<<<grid_for(q), 256, 0, s>>>(totals + T_R, recv_row, rmask, sb.kA, sb.vA);
@@ -988,10 +1039,10 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     CK(radix_sort(sb, totals + T_R, q, 0, (n + 7) / 8 * 8, 1, s, &ko, &vo));
     const int32_t *P = vo;
     int32_t *runstart = ptr<int32_t>(ws, D.runstart), *msgbase = ptr<int32_t>(ws, D.msgbase);
-    CK(scan_exclusive(counts, runstart, nm * n + 1, scan, totals + T_DUMMY, s));
+    CK(scan_exclusive(lb, counts, runstart, nm * n + 1, totals + T_DUMMY, s));
     ell_kernel<<<grid_for(nm), 256, 0, s>>>(nm, n, counts, ell, totals + T_SETS);
     LAUNCHED();
-    CK(scan_exclusive(ell, msgbase, nm + 1, scan, totals + T_C, s));
+    CK(scan_exclusive(lb, ell, msgbase, nm + 1, totals + T_C, s));
     int32_t *earr = ptr<int32_t>(ws, D.earr);
     uint64_t *msg_set = ptr<uint64_t>(ws, D.msg_set);
     msgrow_kernel<<<grid_for(q + 1), 256, 0, s>>>(q, nm, n, msgbase, totals + T_C, counts, earr,
@@ -1002,14 +1053,14 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     int32_t *dec_ptr = prog(ws, D.prog.dec_ptr), *dec_slot = prog(ws, D.prog.dec_slot);
     int32_t *com_dst = prog(ws, D.prog.com_dst);
     int32_t *msg_worker = ptr<int32_t>(ws, D.msg_worker);
-    CK(scan_exclusive(earr, enc_ptr, q + 1, scan, totals + T_DUMMY, s));
+    CK(scan_exclusive(lb, earr, enc_ptr, q + 1, totals + T_DUMMY, s));
     entries_kernel<<<grid_for(q), 256, 0, s>>>(totals + T_R, n, P, recv_row, owner1, rmask,
                                                runstart, msgbase, counts, enc_ptr, enc_src,
                                                msg_worker, dec_msg, dec_dst, dx);
     LAUNCHED();
 
     // decoding: the slots each received row subtracts (old slot tables)
-    CK(scan_exclusive(dx, dec_ptr, q + 1, scan, totals + T_X, s));
+    CK(scan_exclusive(lb, dx, dec_ptr, q + 1, totals + T_X, s));
     decslot_kernel<<<grid_for(q), 256, 0, s>>>(totals + T_R, q, sz, msg_worker, dec_msg, enc_ptr,
                                                enc_src, dec_ptr, slot_of, dec_slot,
                                                totals + T_ERR);
@@ -1033,10 +1084,9 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
 
     // commit: dropped slots of each worker take its received rows in order
     int32_t *evflag = ptr<int32_t>(ws, D.evflag), *evrank = ptr<int32_t>(ws, D.evrank);
-    fill_i32<<<1, 32, 0, s>>>(evflag + ns, 1, 0);
     evflag_kernel<<<grid_for(ns), 256, 0, s>>>(ns, sz, slot_row, next, evflag);
     LAUNCHED();
-    CK(scan_exclusive(evflag, evrank, ns + 1, scan, totals + T_DUMMY, s));
+    CK(scan_exclusive(lb, evflag, evrank, ns + 1, totals + T_DUMMY, s));
     commit_kernel<<<grid_for(ns), 256, 0, s>>>(ns, sz, q, evflag, evrank, recv_ptr, recv_row,
                                                com_dst, slot_row, slot_of, totals + T_ERR);
     check_kernel<<<1, 32, 0, s>>>(n, sz, evrank, recv_ptr, totals + T_ERR);

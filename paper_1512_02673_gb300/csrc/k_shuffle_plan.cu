@@ -31,8 +31,9 @@
 // before it (decoupled look-back: a tile's flag holds its count, then its
 // inclusive prefix; a bounded wait, an error flag on time-out), then writes
 // each digit's run to consecutive addresses through shared memory.
-// Device scans: 4096 items per 1024-thread block, block sums scanned
-// recursively.
+// Device scans: one launch, tiles of 4096 items per 1024-thread block taken
+// in atomic-counter order, each tile's prefix by the same kind of look-back
+// (warp 0 reads 32 predecessor flags at a time).
 #include <cuda_runtime.h>
 #include <stdint.h>
 

@@ -146,10 +146,23 @@ uint32_t next_epoch(uint32_t *e)
 
 // ---- exclusive scan (int32) -----------------------------------------------------------
 
+// Scan inputs and epilogues: the default reads an array and writes nothing
+// more; a fused step generates its inputs or consumes (index, value,
+// exclusive prefix) itself.
+struct ArrayIn {
+    const int32_t *p;
+    __device__ int32_t operator()(int64_t i) const { return p[i]; }
+};
+struct NoEpilogue {
+    __device__ void operator()(int64_t, int32_t, int32_t) const {}
+};
+
 // One pass: tiles of 4096 items in the order of an atomic counter; a tile
 // scans itself, publishes its sum, and warp 0 looks back over the flags of
-// the 32 tiles before it at a time for its prefix (bounded waits).
-__global__ void __launch_bounds__(kScanBlock) scan_kernel(const int32_t *in, int32_t *out,
+// the 32 tiles before it at a time for its prefix (bounded waits).  `out`
+// (nullable) receives the exclusive prefixes.
+template <class In, class Epi>
+__global__ void __launch_bounds__(kScanBlock) scan_kernel(In in, Epi epi, int32_t *out,
                                                           int64_t count, int32_t *total,
                                                           uint64_t *flags, uint32_t epoch,
                                                           int32_t *ctr, int32_t *err)
@@ -165,7 +178,7 @@ __global__ void __launch_bounds__(kScanBlock) scan_kernel(const int32_t *in, int
     int32_t v[4], sum = 0;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-        v[k] = base + k < count ? in[base + k] : 0;
+        v[k] = base + k < count ? in(base + k) : 0;
         sum += v[k];
     }
     int32_t x = sum;   // inclusive scan of the thread sums within the warp
@@ -230,7 +243,10 @@ __global__ void __launch_bounds__(kScanBlock) scan_kernel(const int32_t *in, int
     int32_t excl = x - sum + (warp ? warp_sums[warp - 1] : 0) + s_prefix;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-        if (base + k < count) out[base + k] = excl;
+        if (base + k < count) {
+            if (out) out[base + k] = excl;
+            epi(base + k, v[k], excl);
+        }
         excl += v[k];
     }
     if (multi && threadIdx.x == 0 && atomicAdd(&ctr[1], 1) == (int32_t)gridDim.x - 1) {
@@ -241,10 +257,12 @@ __global__ void __launch_bounds__(kScanBlock) scan_kernel(const int32_t *in, int
 
 int64_t up256(int64_t x) { return (x + 255) & ~(int64_t)255; }
 
-// out[i] = in[0] + ... + in[i-1] for i < count (in may be out); the sum of
-// all of them goes to *total (device, nullable).  One launch.
-cudaError_t scan_exclusive(const LookBack &lb, const int32_t *in, int32_t *out, int64_t count,
-                           int32_t *total, cudaStream_t s)
+// out[i] = in(0) + ... + in(i-1) for i < count (out nullable; an input
+// array may be out), epi(i, in(i), out[i]) for every i; the sum of all of
+// them goes to *total (device, nullable).  One launch.
+template <class In, class Epi>
+cudaError_t scan_fused(const LookBack &lb, In in, Epi epi, int32_t *out, int64_t count,
+                       int32_t *total, cudaStream_t s)
 {
     if (count <= 0) {
         if (total) fill_i32<<<1, 32, 0, s>>>(total, 1, 0);
@@ -253,9 +271,15 @@ cudaError_t scan_exclusive(const LookBack &lb, const int32_t *in, int32_t *out, 
     const int64_t nb = (count + kScanItems - 1) / kScanItems;
     if (nb > lb.nflags || nb > INT32_MAX) return cudaErrorInvalidValue;
     const uint32_t epoch = nb > 1 ? next_epoch(lb.epoch) : 0;
-    scan_kernel<<<(unsigned)nb, kScanBlock, 0, s>>>(in, out, count, total, lb.flags, epoch, lb.ctr,
-                                                    lb.err);
+    scan_kernel<In, Epi><<<(unsigned)nb, kScanBlock, 0, s>>>(in, epi, out, count, total, lb.flags,
+                                                             epoch, lb.ctr, lb.err);
     return cudaGetLastError();
+}
+
+cudaError_t scan_exclusive(const LookBack &lb, const int32_t *in, int32_t *out, int64_t count,
+                           int32_t *total, cudaStream_t s)
+{
+    return scan_fused(lb, ArrayIn{in}, NoEpilogue{}, out, count, total, s);
 }
 
 // ---- stable LSD radix sort (64-bit keys, int32 values) ---------------------------------
@@ -669,8 +693,8 @@ __global__ void cand_rank_kernel(const int32_t *nlist, const int32_t *lw, const 
 // table fits (`local` = 2^n n entries, else 0: global atomics).  The new
 // cache masks start as the owner's bit.
 __global__ void need_kernel(int64_t q, int n, const int32_t *owner1, const uint64_t *cached0,
-                            uint64_t *rmask, int32_t *needflag, uint64_t *next, int32_t *counts,
-                            int32_t *wcount, int local)
+                            uint64_t *rmask, uint64_t *next, int32_t *counts, int32_t *wcount,
+                            int local)
 {
     extern __shared__ int32_t sl[];
     __shared__ int32_t sw[kMaxDeviceN];
@@ -682,7 +706,6 @@ __global__ void need_kernel(int64_t q, int n, const int32_t *owner1, const uint6
         const int i = owner1[r];
         const uint64_t bit = 1ull << i, have = cached0[r];
         const int nf = (have & bit) ? 0 : 1;
-        needflag[r] = nf;
         rmask[r] = have | bit;
         next[r] = bit;
         if (nf) {
@@ -698,35 +721,45 @@ __global__ void need_kernel(int64_t q, int n, const int32_t *owner1, const uint6
         if (sl[i]) atomicAdd(&counts[i], sl[i]);
 }
 
-__global__ void compact_kernel(int64_t q, const int32_t *flag, const int32_t *idx, int32_t *items)
-{
-    GS_LOOP(r, q) if (flag[r]) items[idx[r]] = (int32_t)r;
-}
-
-__global__ void worker_keys_kernel(const int32_t *countp, const int32_t *items,
-                                   const int32_t *owner1, uint64_t *keys, int32_t *vals)
-{
-    const int64_t count = *countp;
-    GS_LOOP(u, count)
+// Input of that scan: row r is missing from its new owner's cache.
+struct MissingRow {
+    const int32_t *owner1;
+    const uint64_t *cached0;
+    __device__ int32_t operator()(int64_t r) const
     {
-        keys[u] = (uint64_t)owner1[items[u]];
-        vals[u] = items[u];
+        return (cached0[r] >> owner1[r]) & 1ull ? 0 : 1;
     }
-}
+};
 
-__global__ void copy_i32_counted(const int32_t *countp, const int32_t *src, int32_t *dst)
-{
-    const int64_t count = *countp;
-    GS_LOOP(u, count) dst[u] = src[u];
-}
+// Epilogue of the scan of the missing flags: the missing rows compacted in
+// row order, as (worker, row) keys of the sort by worker.
+struct MissingToKeys {
+    const int32_t *owner1;
+    uint64_t *keys;
+    int32_t *vals;
+    __device__ void operator()(int64_t r, int32_t flag, int32_t pos) const
+    {
+        if (flag) {
+            keys[pos] = (uint64_t)owner1[r];
+            vals[pos] = (int32_t)r;
+        }
+    }
+};
 
-__global__ void mask_keys_kernel(const int32_t *countp, const int32_t *recv_row,
-                                 const uint64_t *rmask, uint64_t *keys, int32_t *vals)
+
+
+// The received rows (sorted by worker) stored, and keyed by their sets I for
+// the sort into messages.
+__global__ void mask_keys_kernel(const int32_t *countp, const int32_t *sorted,
+                                 int32_t *recv_row, const uint64_t *rmask, uint64_t *keys,
+                                 int32_t *vals)
 {
     const int64_t count = *countp;
     GS_LOOP(v, count)
     {
-        keys[v] = rmask[recv_row[v]];
+        const int32_t r = sorted[v];
+        recv_row[v] = r;
+        keys[v] = rmask[r];
         vals[v] = (int32_t)v;
     }
 }
@@ -820,24 +853,27 @@ __global__ void decslot_kernel(const int32_t *Rp, int64_t q, int64_t s, const in
     }
 }
 
-__global__ void evflag_kernel(int64_t ns, int64_t s, const int32_t *slot_row,
-                              const uint64_t *next, int32_t *evflag)
-{
-    GS_LOOP(g, ns)
+// Input of the scan of the dropped slots: slot g = i s + c of cache i is
+// dropped when the new cache mask of its row lacks bit i (0 past the end).
+struct DroppedSlot {
+    int64_t ns, s;
+    const int32_t *slot_row;
+    const uint64_t *next;
+    __device__ int32_t operator()(int64_t g) const
     {
-        const int i = (int)(g / s);
-        evflag[g] = (next[slot_row[g]] >> i) & 1ull ? 0 : 1;
+        if (g >= ns) return 0;
+        return (next[slot_row[g]] >> (int)(g / s)) & 1ull ? 0 : 1;
     }
-}
+};
 
-__global__ void commit_kernel(int64_t ns, int64_t s, int64_t q, const int32_t *evflag,
-                              const int32_t *evrank, const int32_t *recv_ptr,
+__global__ void commit_kernel(int64_t ns, int64_t s, int64_t q, const int32_t *evrank,
+                              const int32_t *recv_ptr,
                               const int32_t *recv_row, int32_t *com_dst, int32_t *slot_row,
                               int32_t *slot_of, int32_t *err)
 {
     GS_LOOP(g, ns)
     {
-        if (!evflag[g]) continue;
+        if (evrank[g + 1] == evrank[g]) continue;   // slot g is kept
         const int i = (int)(g / s);
         const int32_t e = evrank[g] - evrank[(int64_t)i * s];
         const int32_t v = recv_ptr[i] + e;
@@ -869,9 +905,9 @@ struct DevLayout {
     ShuffleLayout prog;       // the row programs, at the start (word offsets)
     int64_t owner[2], cached[2], slot_of;
     int64_t kA, kB, vA, vB, flags;
-    int64_t rmask, needflag, idx, items, recv_row, wcount, recv_ptr;
+    int64_t rmask, recv_row, wcount, recv_ptr;
     int64_t counts, runstart, ell, msgbase, earr, msg_set, msg_worker, dx;
-    int64_t cw, cr, ckey, evflag, evrank, totals;
+    int64_t cw, cr, ckey, evrank, totals;
     int64_t sel, pstart;      // selection histograms (partition, then cache update); scan
     int64_t flags_bytes;      // radix tile flags
     int64_t bytes;            // total
@@ -913,9 +949,6 @@ DevLayout device_layout(int32_t n, int64_t q, int64_t s)
     D.flags_bytes = 8 * std::max(256 * tiles, scan_max / kScanItems + 1);
     D.flags = take(D.flags_bytes);
     D.rmask = take(8 * q);
-    D.needflag = take(4 * (q + 1));
-    D.idx = take(4 * (q + 1));
-    D.items = take(4 * q);
     D.recv_row = take(4 * q);
     D.wcount = take(4 * (n + 1));
     D.recv_ptr = take(4 * (n + 1));
@@ -932,7 +965,6 @@ DevLayout device_layout(int32_t n, int64_t q, int64_t s)
     D.ckey = take(8 * D.capK);
     D.sel = take(4 * D.sel_words);
     D.pstart = take(4 * ((int64_t)1 << D.pbits));
-    D.evflag = take(4 * (ns + 1));
     D.evrank = take(4 * (ns + 1));
     D.totals = take(4 * kTotalsWords);
     D.bytes = at;
@@ -992,10 +1024,9 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
 #define LAUNCHED() CK(cudaGetLastError())
 
     {
-        int32_t *evflag_end = ptr<int32_t>(ws, D.evflag) + ns;
-        const ZeroList z{{totals, counts, wcount, ell, dx, phist, evflag_end},
-                         {kTotalsWords, nm * n + 1, n + 1, nm + 1, q + 1, D.sel_words, 1},
-                         7};
+        const ZeroList z{{totals, counts, wcount, ell, dx, phist},
+                         {kTotalsWords, nm * n + 1, n + 1, nm + 1, q + 1, D.sel_words},
+                         6};
         zero_many_kernel<<<grid_for(D.sel_words + q), 256, 0, s>>>(z);
         LAUNCHED();
     }
@@ -1013,29 +1044,25 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
 
     // missing rows, their sets and the counters
     uint64_t *rmask = ptr<uint64_t>(ws, D.rmask);
-    int32_t *needflag = ptr<int32_t>(ws, D.needflag), *idx = ptr<int32_t>(ws, D.idx);
     const int local = nm * n <= 8192 ? (int)(nm * n) : 0;   // 32 KB of shared counters
     need_kernel<<<grid_for(q), 256, sizeof(int32_t) * local, s>>>(
-        q, n, owner1, cached0, rmask, needflag, next, counts, wcount, local);
+        q, n, owner1, cached0, rmask, next, counts, wcount, local);
     LAUNCHED();
     uint64_t *ko;
     int32_t *vo;
-    CK(scan_exclusive(lb, needflag, idx, q, totals + T_R, s));
-    int32_t *items = ptr<int32_t>(ws, D.items);
-    compact_kernel<<<grid_for(q), 256, 0, s>>>(q, needflag, idx, items);
-    LAUNCHED();
+    // missing rows in row order, keyed by worker
+    CK(scan_fused(lb, MissingRow{owner1, cached0}, MissingToKeys{owner1, sb.kA, sb.vA}, nullptr,
+                  q, totals + T_R, s));
 
     // received order: (worker, row)
     int32_t *recv_row = ptr<int32_t>(ws, D.recv_row), *recv_ptr = ptr<int32_t>(ws, D.recv_ptr);
-    worker_keys_kernel<<<grid_for(q), 256, 0, s>>>(totals + T_R, items, owner1, sb.kA, sb.vA);
-    LAUNCHED();
     CK(radix_sort(sb, totals + T_R, q, 0, 8, 0, s, &ko, &vo));
-    copy_i32_counted<<<grid_for(q), 256, 0, s>>>(totals + T_R, vo, recv_row);
-    LAUNCHED();
     CK(scan_exclusive(lb, wcount, recv_ptr, n + 1, totals + T_DUMMY, s));
 
-    // message order: (I, worker, row)
-    mask_keys_kernel<<<grid_for(q), 256, 0, s>>>(totals + T_R, recv_row, rmask, sb.kA, sb.vA);
+    // message order: (I, worker, row); the sort's output (B) is stored as the
+    // received rows and keyed into A
+    if (vo == sb.vA) return cudaErrorInvalidValue;   // one pass: the result is in B
+    mask_keys_kernel<<<grid_for(q), 256, 0, s>>>(totals + T_R, vo, recv_row, rmask, sb.kA, sb.vA);
     LAUNCHED();
     CK(radix_sort(sb, totals + T_R, q, 0, (n + 7) / 8 * 8, 1, s, &ko, &vo));
     const int32_t *P = vo;
@@ -1084,11 +1111,10 @@ cudaError_t plan_on_device(cm_shuffle *S, void *ws, cudaStream_t s, int32_t *tot
     LAUNCHED();
 
     // commit: dropped slots of each worker take its received rows in order
-    int32_t *evflag = ptr<int32_t>(ws, D.evflag), *evrank = ptr<int32_t>(ws, D.evrank);
-    evflag_kernel<<<grid_for(ns), 256, 0, s>>>(ns, sz, slot_row, next, evflag);
-    LAUNCHED();
-    CK(scan_exclusive(lb, evflag, evrank, ns + 1, totals + T_DUMMY, s));
-    commit_kernel<<<grid_for(ns), 256, 0, s>>>(ns, sz, q, evflag, evrank, recv_ptr, recv_row,
+    int32_t *evrank = ptr<int32_t>(ws, D.evrank);
+    CK(scan_fused(lb, DroppedSlot{ns, sz, slot_row, next}, NoEpilogue{}, evrank, ns + 1,
+                  totals + T_DUMMY, s));
+    commit_kernel<<<grid_for(ns), 256, 0, s>>>(ns, sz, q, evrank, recv_ptr, recv_row,
                                                com_dst, slot_row, slot_of, totals + T_ERR);
     check_kernel<<<1, 32, 0, s>>>(n, sz, evrank, recv_ptr, totals + T_ERR);
     LAUNCHED();

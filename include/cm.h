@@ -415,7 +415,8 @@ cm_status cm_shuffle_decode(const cm_shuffle *shuffle, const void *workspace, cm
 
 /* Bytes of device workspace for the device planner (0 if n > 16): the row
  * programs of cm_shuffle_workspace_bytes first, then the resident state and
- * scratch (about 4 q (n + 5) + 4 n s + 100 q + 24 max(q, n s) bytes). */
+ * scratch (about 4 q (n + 21) + 4 n s + 16 max(q, n s) + 8 n 2^n + 2^18 n
+ * bytes). */
 size_t cm_shuffle_device_workspace_bytes(const cm_shuffle *shuffle);
 
 /* Moves the current host state (and, after a transition, its programs) into
@@ -424,7 +425,7 @@ size_t cm_shuffle_device_workspace_bytes(const cm_shuffle *shuffle);
 cm_status cm_shuffle_device_init(cm_shuffle *shuffle, void *workspace, size_t bytes,
                                  cm_stream_t stream);
 
-/* Plans the transition t -> t+1 on the device (about 40 launches on
+/* Plans the transition t -> t+1 on the device (about 26 launches on
  * `stream`), then reads back its counts (synchronising `stream`); stats is
  * nullable.  The programs are then in place for cm_shuffle_encode, _decode
  * and _commit. */

@@ -195,6 +195,7 @@ def test_coded_gemm_writes_every_row_and_nothing_else(cm, orc, n, k, m, d, N):
     (10, 5, 1300, 64, 96, "mds"),        # L = 260: the second pair holds 4 rows
     (24, 20, 762, 64, 300, "mds"),       # pad rows in the last systematic block
     (6, 3, 900, 128, 64, "repetition"),
+    (5, 3, 100, 64, 40, "mds"),          # L = 34: a run of one block is shorter than a CTA's rows
 ])
 def test_coded_gemm_survivors_only(cm, orc, n, k, m, d, N, kind):
     """Survivors-only GEMM: the k blocks that the decode reads equal the full

@@ -141,3 +141,14 @@ def test_device_planner_refuses_without_workspace(cm):
     assert small.device_workspace_bytes() >= small.workspace_bytes()
     big = cm.Shuffle(17, 17 * 4, 8, 1, 2)
     assert big.device_workspace_bytes() == 0
+
+
+@pytest.mark.parametrize("n,q,s", [(8, 1 << 16, 1 << 14), (4, 4000, 1700), (16, 3200, 800),
+                                   (2, 40, 20)])
+def test_device_workspace_size_formula(cm, n, q, s):
+    # the size the header states for the device planner's workspace, to 10 %
+    sh = cm.Shuffle(n, q, s, 1, 2)
+    est = (sh.workspace_bytes() + 4 * q * (n + 21) + 4 * n * s + 16 * max(q, n * s)
+           + 8 * n * 2 ** n + 2 ** 18 * n)
+    got = sh.device_workspace_bytes()
+    assert 0.9 * est <= got <= 1.1 * est, (got, est)

@@ -53,7 +53,7 @@ typedef enum {
     CM_ECUDA = -4,           /* a CUDA launch or query failed */
     CM_ENOMEM = -5,          /* host allocation failed, or workspace too small */
     CM_ETIMEOUT = -6,        /* a bounded device wait gave up */
-    CM_EUNSUPPORTED = -7     /* valid request this build does not handle */
+    CM_EUNSUPPORTED = -7     /* valid request the library does not handle */
 } cm_status;
 
 typedef enum { CM_F32 = 0, CM_BF16 = 1 } cm_dtype;

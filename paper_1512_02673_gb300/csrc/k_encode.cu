@@ -233,7 +233,7 @@ __device__ __forceinline__ void encode_body(const CUtensorMap &tmF, const CUtens
     }
 }
 
-// up to 8 parity blocks per pass: the compiler's own register choice (two or
+// up to 12 parity blocks per pass: the compiler's own register choice (two or
 // three CTAs per SM); 16: capped at 128 registers, two CTAs per SM
 template <typename T, int NPG>
 __global__ void __launch_bounds__(kWarps * 32)
@@ -282,7 +282,7 @@ cudaError_t launch_passes(const CodeParams &cp, const T *A, int64_t lda, T *par,
     a.steps = (int)((cp.d + STEP - 1) / STEP);
     a.nsub = (kf + KC - 1) / KC + (kv > kf ? 1 : 0);
     void (*kern)(const CUtensorMap, const CUtensorMap, const CodeParams, const EncodeArgs);
-    if constexpr (NPG > 8)
+    if constexpr (NPG == 16)
         kern = encode_kernel16<T>;
     else
         kern = encode_kernel<T, NPG>;
@@ -324,22 +324,35 @@ cudaError_t launch_passes(const CodeParams &cp, const T *A, int64_t lda, T *par,
     return cudaSuccess;
 }
 
+// Parity blocks per pass: the smallest instance at or above n - k, so that
+// few accumulators and coefficient slots go to blocks that do not exist
+// (n - k > 16 takes several passes of 16).
+template <typename T>
+cudaError_t launch_np(const CodeParams &cp, const T *A, int64_t lda, T *par, int64_t ldp,
+                      int32_t *status, cudaStream_t s)
+{
+    const int np = cp.n - cp.k;
+    if (np <= 2) return launch_passes<T, 2>(cp, A, lda, par, ldp, status, s);
+    if (np <= 3) return launch_passes<T, 3>(cp, A, lda, par, ldp, status, s);
+    if (np <= 4) return launch_passes<T, 4>(cp, A, lda, par, ldp, status, s);
+    if (np <= 5) return launch_passes<T, 5>(cp, A, lda, par, ldp, status, s);
+    if (np <= 6) return launch_passes<T, 6>(cp, A, lda, par, ldp, status, s);
+    if (np <= 8) return launch_passes<T, 8>(cp, A, lda, par, ldp, status, s);
+    if (np <= 10) return launch_passes<T, 10>(cp, A, lda, par, ldp, status, s);
+    if (np <= 12) return launch_passes<T, 12>(cp, A, lda, par, ldp, status, s);
+    return launch_passes<T, 16>(cp, A, lda, par, ldp, status, s);
+}
+
 }  // namespace
 
 cudaError_t launch_encode_f32(const CodeParams &cp, const float *A, int64_t lda, float *par,
                               int64_t ldp, int32_t *status, cudaStream_t s)
 {
-    const int np = cp.n - cp.k;
-    if (np <= 4) return launch_passes<float, 4>(cp, A, lda, par, ldp, status, s);
-    if (np <= 8) return launch_passes<float, 8>(cp, A, lda, par, ldp, status, s);
-    return launch_passes<float, 16>(cp, A, lda, par, ldp, status, s);
+    return launch_np<float>(cp, A, lda, par, ldp, status, s);
 }
 
 cudaError_t launch_encode_bf16(const CodeParams &cp, const uint16_t *A, int64_t lda,
                                uint16_t *par, int64_t ldp, int32_t *status, cudaStream_t s)
 {
-    const int np = cp.n - cp.k;
-    if (np <= 4) return launch_passes<uint16_t, 4>(cp, A, lda, par, ldp, status, s);
-    if (np <= 8) return launch_passes<uint16_t, 8>(cp, A, lda, par, ldp, status, s);
-    return launch_passes<uint16_t, 16>(cp, A, lda, par, ldp, status, s);
+    return launch_np<uint16_t>(cp, A, lda, par, ldp, status, s);
 }

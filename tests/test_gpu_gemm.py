@@ -160,7 +160,20 @@ def test_gemm_config_sampled(cm, orc):
     got_c = C[idx[valid].to(DEV)].double().cpu().numpy()
     err = rel_cols(got_c, C_or[valid.numpy()])
     assert err.max() <= 1e-2, err.max()
-    del A, B, Bt, par, Ct, C
+    # survivors only at full size (the bench's launch): the k blocks the
+    # decode reads equal the full GEMM's bit for bit, the others untouched
+    del C
+    Cs = torch.full_like(Ct, float("nan"))
+    cm.coded_gemm_survivors(code, A, par, Bt, mask, Ct=Cs)
+    torch.cuda.synchronize()
+    sel = code.select_decodable(mask)
+    for j in range(w.n):
+        blk = slice(j * L, (j + 1) * L)
+        if (sel >> j) & 1:
+            assert torch.equal(Cs[blk], Ct[blk]), j
+        else:
+            assert bool(torch.isnan(Cs[blk]).all()), j
+    del A, B, Bt, par, Ct, Cs
     torch.cuda.empty_cache()
 
 

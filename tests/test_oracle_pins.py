@@ -49,6 +49,42 @@ def test_fig1_toy_example(orc):
         np.testing.assert_array_equal(Y[:, 0], full)
 
 
+# ---- Sec. I-A / III-A: the plain product Y = A X every decode is checked against
+
+def test_matmul_reproduces_fig1_products(orc):
+    # Fig. 1: A x is the concatenation of the two block products A1 x, A2 x,
+    # worked by hand in the fixture (an exact integer case).
+    g = read_golden("fig1_toy.txt")
+    A = np.vstack([np.array(g["A1 (2 x 3)"]), np.array(g["A2 (2 x 3)"])])
+    x = np.array(g["x (3)"]).reshape(3, 1)
+    Y = orc.matmul(A.astype(np.float32), x.astype(np.float32))
+    want = np.concatenate([g["W1 = A1 x"][0], g["W2 = A2 x"][0]])
+    np.testing.assert_array_equal(Y[:, 0], want)
+
+
+def test_matmul_small_integers_are_exact():
+    # Integer A, X with |A|,|X| <= 4 and d = 500: every partial sum is an
+    # integer below 2^53, so fp64 arithmetic must reproduce the int64 product
+    # bit for bit, whatever the summation order.
+    import oracle
+    rng = np.random.default_rng(17)
+    A = rng.integers(-4, 5, size=(1200, 500))
+    X = rng.integers(-4, 5, size=(500, 3))
+    Y = oracle.matmul(A.astype(np.float32), X.astype(np.float32))
+    np.testing.assert_array_equal(Y, (A @ X).astype(np.float64))
+
+
+@pytest.mark.parametrize("m,d,b", [(37, 101, 8), (5, 3, 7), (64, 33, 1)])
+def test_matmul_multi_vector_matches_library(orc, m, d, b):
+    # b > 1 and m != d: a transposed X index or a swapped operand shape
+    # changes the result; numpy's fp64 product is the independent reference.
+    rng = np.random.default_rng(m * 1000 + d)
+    A = rng.standard_normal((m, d)).astype(np.float32)
+    X = rng.standard_normal((d, b)).astype(np.float32)
+    want = A.astype(np.float64) @ X.astype(np.float64)
+    np.testing.assert_allclose(orc.matmul(A, X), want, rtol=1e-12, atol=1e-12)
+
+
 # ---- Sec. III-A: encoding, systematic outputs, any-k decoding -----------------
 
 def test_block_rows_padding(orc):

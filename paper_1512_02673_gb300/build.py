@@ -40,8 +40,6 @@ def sources():
 def _compile(src: str) -> tuple[str, str]:
     obj = os.path.join(BUILD, os.path.basename(src) + ".o")
     cmd = [nvcc(), "-c", src, "-o", obj, "-I", os.path.join(ROOT, "include")] + NVCC_FLAGS
-    if src.endswith(".cpp"):
-        cmd += ["-x", "cu"] if False else []
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError("nvcc failed for %s:\n%s%s" % (src, res.stdout, res.stderr))

@@ -1,6 +1,7 @@
 // Internal declarations shared by the libcm translation units.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 

@@ -23,13 +23,63 @@ static __device__ __align__(256) unsigned char g_gd_scratch[CM_GD_STATIC_SCRATCH
 
 namespace {
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-void *g_addr[kMaxDevices] = {nullptr};
+// In host code g_gd_scratch names a host-side stand-in, not device memory: the
+// array's device address belongs to the module image loaded into one CUDA
+// context, so it is looked up with cudaGetSymbolAddress (with the device
+// current) and cached per device together with the unique ID of the context
+// it came from.  A different current context on the device (after
+// cudaDeviceReset, which replaces the primary context, or a context the caller
+// created itself) has a different ID and gets a fresh lookup, never the old
+// address.  Context IDs are never reused within a process.
+using CtxGetCurrentFn = CUresult (*)(CUcontext *);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long *);
 
-// Device address of the scratch array on the current device.  In host code
-// g_gd_scratch names a host-side stand-in, not device memory, so the address
-// is looked up once per device (with that device current) and cached.
+struct DriverFns {
+    CtxGetCurrentFn get_current = nullptr;
+    CtxGetIdFn get_id = nullptr;
+};
+
+const DriverFns &driver_fns()
+{
+    static DriverFns fns;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fns.get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fns.get_id = reinterpret_cast<CtxGetIdFn>(p);
+    });
+    return fns;
+}
+
+// Unique ID of the context current on this thread (false if there is none
+// yet or the driver cannot tell; the caller then looks the address up afresh).
+bool current_context_id(unsigned long long *id)
+{
+    const DriverFns &f = driver_fns();
+    if (!f.get_current || !f.get_id) return false;
+    CUcontext ctx = nullptr;
+    if (f.get_current(&ctx) != CUDA_SUCCESS || !ctx) return false;
+    return f.get_id(ctx, id) == CUDA_SUCCESS;
+}
+
+constexpr int kMaxDevices = 64;
+struct CachedAddress {
+    bool valid = false;
+    unsigned long long ctx_id = 0;
+    void *addr = nullptr;
+};
+std::mutex g_mu;
+CachedAddress g_cache[kMaxDevices];
+
+// Device address of the scratch array in the current device's current context.
 cudaError_t scratch_address(void **out)
 {
     int dev = -1;
@@ -37,13 +87,20 @@ cudaError_t scratch_address(void **out)
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
     std::lock_guard<std::mutex> lock(g_mu);
-    if (!g_addr[dev]) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_gd_scratch);
-        if (e != cudaSuccess) return e;
-        g_addr[dev] = p;
+    CachedAddress &c = g_cache[dev];
+    unsigned long long id = 0;
+    if (c.valid && current_context_id(&id) && id == c.ctx_id) {
+        *out = c.addr;
+        return cudaSuccess;
     }
-    *out = g_addr[dev];
+    // The lookup binds the device's context to this thread if none is yet,
+    // so the context ID is read after it.
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_gd_scratch);
+    if (e != cudaSuccess) return e;
+    c.addr = p;
+    c.valid = current_context_id(&c.ctx_id);
+    *out = p;
     return cudaSuccess;
 }
 

@@ -146,3 +146,11 @@ def test_gd_workspace_and_checks(cm):
     # a product with fewer than k survivors
     assert L.cm_gd_step(cA.handle, fake, d, fake, d, cAT.handle, fake, m, fake, m, fake, fake,
                         0.1, 0b111, full, fake, ws, None, None) == cm.CM_ENOTDECODABLE
+
+
+def test_static_scratch_size_matches_header(cm):
+    # The binding's copy of CM_GD_STATIC_SCRATCH_BYTES is the header's value.
+    src = open(os.path.join(ROOT, "include", "cm.h")).read()
+    m = re.search(r"#define\s+CM_GD_STATIC_SCRATCH_BYTES\s+\((\d+)u\s*<<\s*(\d+)\)", src)
+    assert m, "CM_GD_STATIC_SCRATCH_BYTES not found in cm.h"
+    assert cm.GD_STATIC_SCRATCH_BYTES == int(m.group(1)) << int(m.group(2))

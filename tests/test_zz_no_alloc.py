@@ -44,7 +44,7 @@ def problem(cm, m, d, n, k):
     return cA, cAT, Ad, cm.encode(cA, Ad), ATd, cm.encode(cAT, ATd), y
 
 
-def test_noalloc_step_matches_workspace_step_on_two_calls(cm):
+def test_noalloc_step_matches_workspace_step_on_two_calls(cm, orc):
     m, d, n, k = 1001, 203, 20, 10
     cA, cAT, A, PA, AT, PAT, y = problem(cm, m, d, n, k)
     assert cm.gd_workspace_bytes(cA, cAT) <= cm.GD_STATIC_SCRATCH_BYTES
@@ -53,18 +53,37 @@ def test_noalloc_step_matches_workspace_step_on_two_calls(cm):
     status = torch.zeros(1, dtype=torch.int32, device=DEV)
     x_ws = torch.zeros(d, device=DEV)
     x_na = torch.zeros(d, device=DEV)
-    for t in range(2):                       # two calls in a row
+    steps = 2
+    for t in range(steps):                   # two calls in a row
         sA = cm.draw_erasures(synth.ERASURE_SEED, 2 * t, n, k)[0]
         sAT = cm.draw_erasures(synth.ERASURE_SEED, 2 * t + 1, n, k)[0]
         cm.gd_step(cA, A, PA, cAT, AT, PAT, y, x_ws, eta, sA, sAT, ws, status)
         cm.gd_step_noalloc(cA, A, PA, cAT, AT, PAT, y, x_na, eta, sA, sAT, status)
         torch.cuda.synchronize()
         assert status.item() == 0
-        a, b = x_na.double().cpu().numpy(), x_ws.double().cpu().numpy()
-        # same kernels on the same inputs: within the GD tolerance (1e-3), in
-        # practice identical
-        assert np.linalg.norm(a - b) <= 1e-3 * np.linalg.norm(b), t
-        assert np.linalg.norm(b) > 0
+        # the same kernels on the same inputs in the same order: identical
+        assert torch.equal(x_na, x_ws), t
+        assert torch.linalg.norm(x_ws).item() > 0
+    # and the iterate is the exact-gradient iterate (the oracle's fp64 GD)
+    want = orc.gd(A.cpu().numpy(), y.cpu().numpy(), eta, steps)
+    got = x_na.double().cpu().numpy()
+    assert np.linalg.norm(got - want) <= 1e-3 * np.linalg.norm(want)
+
+
+def test_noalloc_step_allocates_nothing(cm):
+    m, d, n, k = 1001, 203, 20, 10
+    cA, cAT, A, PA, AT, PAT, y = problem(cm, m, d, n, k)
+    eta = 0.5 / (m ** 0.5 + d ** 0.5) ** 2
+    x = torch.zeros(d, device=DEV)
+    mask = cm.draw_erasures(synth.ERASURE_SEED, 0, n, k)[0]
+    cm.gd_step_noalloc(cA, A, PA, cAT, AT, PAT, y, x, eta, mask, mask)   # warm-up
+    torch.cuda.synchronize()
+    free0, torch0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
+    for t in range(5):
+        cm.gd_step_noalloc(cA, A, PA, cAT, AT, PAT, y, x, eta, mask, mask)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert torch.cuda.memory_allocated() == torch0
 
 
 def test_noalloc_step_rejects_problems_beyond_the_array(cm):

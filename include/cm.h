@@ -192,8 +192,11 @@ cm_status cm_gd_step(const cm_code *code_A, const float *A, int64_t lda,
  * CM_GD_STATIC_SCRATCH_BYTES held by every GPU that loads the library until
  * the process exits.  The call allocates nothing.  Returns CM_ENOMEM when
  * cm_gd_workspace_bytes(code_A, code_AT) exceeds the array.  The first call
- * on a device looks up the array's device address (once per device, with
- * that device current); make that first call before any stream capture.
+ * on a device looks up the array's device address (with that device
+ * current) and keeps it for that device's current CUDA context; a call made
+ * under another context of the device (after cudaDeviceReset, or in a
+ * context the caller created) looks it up again.  Make the first call in
+ * each context before any stream capture.
  * All calls on a device share the array and it keeps the last call's
  * contents (nothing in it needs to start at zero); calls whose kernels
  * overlap on the GPU race on it. */

@@ -140,22 +140,20 @@ cm_status cm_draw_erasures(uint64_t seed, uint64_t counter, int32_t n, int32_t k
 /* Decoding (Sec. III-A last paragraph; Example "MDS codes").  S = the first
  * k set bits of `survivors` (ascending; extra survivors are ignored, which
  * favours the systematic workers).  The surviving results satisfy
- * Yt_S = G_S Z with Z the uncoded block products.  A small plan kernel (one
- * CTA) inverts G_S in fp64 on the device (the k-e unit rows of surviving
- * systematic workers are eliminated first, then Gauss-Jordan with partial
- * pivoting on the e x e block of the missing systematic columns) and forms
- * the rows of G_S^-1 for the e missing systematic blocks; the apply kernel,
- * launched behind it as a programmatic dependent launch, applies them to the
- * k surviving results (double-float arithmetic, about 2^-44 relative per
- * term) while surviving systematic blocks pass through.  The rows travel in
- * a ring of 256 slots in the library's static device memory: no allocation
- * per call, and at most 256 decodes (cm_decode, cm_decode_mat, cm_matmat,
- * cm_gd_step together) may be pending at once across streams.  Y (m x b fp32) is the
- * concatenation of the k decoded blocks without the appended zero rows.
- * Returns CM_ENOTDECODABLE when fewer than k bits are set; a singular G_S
- * (a zero pivot, or ||Q|| ||Q^-1|| beyond 1 / (64 eps) for the e x e block)
- * writes CM_ESINGULAR to *dev_status (nullable) and leaves the missing
- * blocks of Y unwritten (surviving systematic blocks are still copied). */
+ * Yt_S = G_S Z with Z the uncoded block products.  One launch: every CTA
+ * inverts G_S in fp64 in its own shared memory (the k-e unit rows of
+ * surviving systematic workers are eliminated first, then Gauss-Jordan with
+ * partial pivoting on the e x e block of the missing systematic columns, in
+ * one warp's registers) and forms the rows of G_S^-1 for the e missing
+ * systematic blocks, then applies them to the k surviving results
+ * (double-float arithmetic, about 2^-44 relative per term) while surviving
+ * systematic blocks pass through.  Nothing is kept between calls.  Y (m x b
+ * fp32) is the concatenation of the k decoded blocks without the appended
+ * zero rows.  Returns CM_ENOTDECODABLE when fewer than k bits are set; a
+ * singular G_S (a zero pivot, or ||Q|| ||Q^-1|| beyond 1 / (64 eps) for the
+ * e x e block) writes CM_ESINGULAR to *dev_status (nullable) and leaves the
+ * missing blocks of Y unwritten (surviving systematic blocks are still
+ * copied). */
 cm_status cm_decode(const cm_code *code, const double *Yt, uint32_t survivors,
                     int32_t b, float *Y, int32_t *dev_status, cm_stream_t stream);
 
@@ -235,8 +233,8 @@ cm_status cm_coded_gemm_survivors(const cm_code *code, const void *A, int64_t ld
 
 /* Decoding of matrix results: as cm_decode with b = N columns of fp32
  * stacked results Ct (leading dimension ldc) into C (m x N fp32, leading
- * dimension ldcc).  The decode coefficients are formed in fp64 by the same
- * plan kernel as for cm_decode and applied in fp32.  C may alias Ct (C == Ct, ldcc == ldc): surviving systematic
+ * dimension ldcc).  The decode coefficients are formed in fp64 in each CTA as
+ * for cm_decode and applied in fp32.  C may alias Ct (C == Ct, ldcc == ldc): surviving systematic
  * blocks are then already in place and only the missing ones are written. */
 cm_status cm_decode_mat(const cm_code *code, const float *Ct, int64_t ldc,
                         uint32_t survivors, int32_t N, float *C, int64_t ldcc,

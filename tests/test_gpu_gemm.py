@@ -127,7 +127,9 @@ def test_decode_mat_every_erasure_count(cm, orc):
 
 def test_gemm_config_sampled(cm, orc):
     """(16,12), A 32768 x 8192 bf16, B 8192 x 4096 bf16: sampled block rows
-    of every worker against the oracle on the same bf16 blocks."""
+    of every worker against the oracle on the same bf16 blocks, and, over all
+    4096 columns, one random row inside every 256-row tile pair of the
+    kernel's tiling plus the first and last row of every pair."""
     w = synth.GEMM
     P = synth.parity_coefficients(w.n, w.k)
     code = cm.Code(w.n, w.k, w.m, w.d, P, dtype="bf16")
@@ -160,6 +162,28 @@ def test_gemm_config_sampled(cm, orc):
     got_c = C[idx[valid].to(DEV)].double().cpu().numpy()
     err = rel_cols(got_c, C_or[valid.numpy()])
     assert err.max() <= 1e-2, err.max()
+    # every tile pair: the kernel cuts the m real rows of A and the (n-k) L
+    # parity rows into 256-row pairs of their own; the pad rows [m, kL) are
+    # stored as zeros
+    assert bool((Ct[w.m:w.k * L] == 0).all())
+    rng2 = np.random.default_rng(6)
+    rows = []
+    for lo, hi in ((0, w.m), (w.k * L, w.n * L)):
+        for t0 in range(lo, hi, 256):
+            t1 = min(hi, t0 + 256)
+            rows += [t0, t1 - 1, int(rng2.integers(t0, t1))]
+    rows = sorted(set(rows))
+    ridx = torch.tensor(rows)
+    is_a = ridx < w.m
+    coded = torch.empty((len(rows), w.d), dtype=torch.bfloat16)
+    coded[is_a] = A[ridx[is_a].to(DEV)].cpu()
+    coded[~is_a] = par[(ridx[~is_a] - w.k * L).to(DEV)].cpu()
+    # the exact products of the bf16 values, accumulated in fp64
+    want_rows = orc.matmul(coded.float().numpy(), B.float().cpu().numpy())
+    got_rows = Ct[ridx.to(DEV)].double().cpu().numpy()
+    num = np.linalg.norm(got_rows - want_rows, axis=1)
+    den = np.linalg.norm(want_rows, axis=1)
+    assert (num / den).max() <= 2 * worker_tol(w.d), (num / den).max()
     # survivors only at full size (the bench's launch): the k blocks the
     # decode reads equal the full GEMM's bit for bit, the others untouched
     del C

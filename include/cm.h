@@ -157,6 +157,32 @@ cm_status cm_draw_erasures(uint64_t seed, uint64_t counter, int32_t n, int32_t k
 cm_status cm_decode(const cm_code *code, const double *Yt, uint32_t survivors,
                     int32_t b, float *Y, int32_t *dev_status, cm_stream_t stream);
 
+/* Workspace bytes cm_matvec_decode needs for b vectors (the stacked results,
+ * n L b fp64; 0 on a bad code or b outside 1..8). */
+size_t cm_matvec_decode_workspace_bytes(const cm_code *code, int32_t b);
+
+/* The worker products and the decode in one call (Sec. III-A: the master
+ * needs only the first k results, and decoding is a fixed linear map of
+ * them): Y = A X (m x b fp32), equal bit for bit to cm_matvec (or
+ * cm_matvec_survivors) followed by cm_decode.  The decode is launched as a
+ * programmatic dependent of the products: its CTAs start on the SMs the
+ * products leave free in their last round, form the rows of G_S^-1 (the fp64
+ * elimination of cm_decode) from the kernel parameters alone, and wait for
+ * the products only before they read a result, so the decode's launch and
+ * inversion overlap the products' tail.  only_survivors = 0: all n workers
+ * compute (the protocol of Sec. III-A); 1: only the k used workers compute
+ * (the stragglers known beforehand), reading (n-k)/n fewer bytes.  S is the
+ * first k set bits of `survivors` (for a repetition code, the first survivor
+ * of each block), as for cm_decode.  ws is caller device memory of at least
+ * cm_matvec_decode_workspace_bytes(code, b) bytes, 256-byte aligned, which
+ * receives the stacked worker results (n L x b fp64; rows of workers that did
+ * not compute are left unwritten).  Two launches.  Errors as cm_matvec and
+ * cm_decode; CM_ENOMEM for a short workspace. */
+cm_status cm_matvec_decode(const cm_code *code, const float *A, int64_t lda,
+                           const float *parity, int64_t ldp, const float *X, int32_t b,
+                           uint32_t survivors, int32_t only_survivors, float *Y, void *ws,
+                           size_t ws_bytes, int32_t *dev_status, cm_stream_t stream);
+
 /* Workspace bytes cm_gd_step needs for this pair of codes (0 on bad codes). */
 size_t cm_gd_workspace_bytes(const cm_code *code_A, const cm_code *code_AT);
 
@@ -166,9 +192,12 @@ size_t cm_gd_workspace_bytes(const cm_code *code_A, const cm_code *code_AT);
  * The second uses code_AT (d x m) on AT = A^T (row-major d x m, i.e. the
  * column split of A, Sec. III-E) and its parity PAT with survivors surv_AT;
  * the result decodes to the gradient g = A^T z and x -= eta g.  x (d fp32) is
- * updated in place.  ws is caller device memory of at least
- * cm_gd_workspace_bytes(code_A, code_AT) bytes (holds both stacked results
- * and z), 256-byte aligned.  Four launches on `stream`. */
+ * updated in place.  All n workers compute each product (the protocol of
+ * Sec. III-A); each decode writes z or the step itself and is launched as a
+ * programmatic dependent of its products, as in cm_matvec_decode.  ws is
+ * caller device memory of at least cm_gd_workspace_bytes(code_A, code_AT)
+ * bytes (holds both stacked results and z), 256-byte aligned.  Four launches
+ * on `stream`. */
 cm_status cm_gd_step(const cm_code *code_A, const float *A, int64_t lda,
                      const float *PA, int64_t ldpa,
                      const cm_code *code_AT, const float *AT, int64_t ldat,
@@ -177,6 +206,18 @@ cm_status cm_gd_step(const cm_code *code_A, const float *A, int64_t lda,
                      uint32_t surv_A, uint32_t surv_AT,
                      void *ws, size_t ws_bytes, int32_t *dev_status,
                      cm_stream_t stream);
+
+/* cm_gd_step with only the k used workers of each product computing (the
+ * straggler sets known before the products run, Sec. III-A: the master needs
+ * only k results).  Same arguments, workspace and result. */
+cm_status cm_gd_step_survivors(const cm_code *code_A, const float *A, int64_t lda,
+                               const float *PA, int64_t ldpa,
+                               const cm_code *code_AT, const float *AT, int64_t ldat,
+                               const float *PAT, int64_t ldpat,
+                               const float *y, float *x, float eta,
+                               uint32_t surv_A, uint32_t surv_AT,
+                               void *ws, size_t ws_bytes, int32_t *dev_status,
+                               cm_stream_t stream);
 
 /* Size of the fixed device scratch array behind cm_gd_step_noalloc: 4 MiB. */
 #define CM_GD_STATIC_SCRATCH_BYTES (4u << 20)

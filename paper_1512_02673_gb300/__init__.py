@@ -60,6 +60,11 @@ def lib() -> ctypes.CDLL:
             "cm_draw_erasures": (st, [u64, u64, i32, i32, f64, f64, ctypes.POINTER(u32), vp]),
             "cm_decode": (st, [vp, vp, u32, i32, vp, vp, vp]),
             "cm_gd_workspace_bytes": (sz, [vp, vp]),
+            "cm_matvec_decode_workspace_bytes": (sz, [vp, i32]),
+            "cm_matvec_decode": (st, [vp, vp, i64, vp, i64, vp, i32, u32, i32, vp, vp, sz, vp,
+                                      vp]),
+            "cm_gd_step_survivors": (st, [vp, vp, i64, vp, i64, vp, vp, i64, vp, i64, vp, vp, f32,
+                                          u32, u32, vp, sz, vp, vp]),
             "cm_gd_step": (st, [vp, vp, i64, vp, i64, vp, vp, i64, vp, i64, vp, vp, f32,
                                 u32, u32, vp, sz, vp, vp]),
             "cm_gd_step_noalloc": (st, [vp, vp, i64, vp, i64, vp, vp, i64, vp, i64, vp, vp,
@@ -300,9 +305,51 @@ def gd_workspace_bytes(code_A: Code, code_AT: Code) -> int:
     return int(lib().cm_gd_workspace_bytes(code_A.handle, code_AT.handle))
 
 
+def matvec_decode_workspace_bytes(code: Code, b: int) -> int:
+    return int(lib().cm_matvec_decode_workspace_bytes(code.handle, b))
+
+
+def matvec_decode(code: Code, A: torch.Tensor, parity: torch.Tensor, X: torch.Tensor,
+                  survivors: int, only_survivors: bool = False, Y: torch.Tensor | None = None,
+                  ws: torch.Tensor | None = None,
+                  status: torch.Tensor | None = None) -> torch.Tensor:
+    """Y = A X (m x b fp32): the worker products with the decode fused into
+    their tail.  only_survivors computes only the k used workers.  ws (uint8,
+    at least matvec_decode_workspace_bytes) also holds the stacked results;
+    allocated here when not given."""
+    _dev(A, torch.float32, "A", 2)
+    _dev(parity, torch.float32, "parity", 2)
+    if X.dim() == 1:
+        X = X.view(-1, 1)
+    _dev(X, torch.float32, "X", 2)
+    _contig(X, "X")
+    if X.shape[0] != code.d:
+        raise ValueError("X must have d rows")
+    b = X.shape[1]
+    if Y is None:
+        Y = torch.empty((code.m, b), dtype=torch.float32, device=X.device)
+    _dev(Y, torch.float32, "Y", 2)
+    _contig(Y, "Y")
+    if ws is None:
+        ws = torch.empty(matvec_decode_workspace_bytes(code, b), dtype=torch.uint8,
+                         device=X.device)
+    _dev(ws, torch.uint8, "ws")
+    sp = None
+    if status is not None:
+        _dev(status, torch.int32, "status")
+        sp = status.data_ptr()
+    _check(lib().cm_matvec_decode(code.handle, A.data_ptr(), _ld(A, "A"), parity.data_ptr(),
+                                  _ld(parity, "parity"), X.data_ptr(), b, survivors,
+                                  1 if only_survivors else 0, Y.data_ptr(), ws.data_ptr(),
+                                  ws.numel(), sp, _stream()), "cm_matvec_decode")
+    return Y
+
+
 def gd_step(code_A: Code, A, PA, code_AT: Code, AT, PAT, y, x, eta: float, surv_A: int,
-            surv_AT: int, ws: torch.Tensor, status: torch.Tensor | None = None):
-    """One coded gradient step x <- x - eta A^T (A x - y), x updated in place."""
+            surv_AT: int, ws: torch.Tensor, status: torch.Tensor | None = None,
+            survivors_only: bool = False):
+    """One coded gradient step x <- x - eta A^T (A x - y), x updated in place.
+    survivors_only computes only the k used workers of each product."""
     for t, name in ((A, "A"), (PA, "PA"), (AT, "AT"), (PAT, "PAT")):
         _dev(t, torch.float32, name, 2)
     _dev(y, torch.float32, "y")
@@ -314,11 +361,11 @@ def gd_step(code_A: Code, A, PA, code_AT: Code, AT, PAT, y, x, eta: float, surv_
     if status is not None:
         _dev(status, torch.int32, "status")
         sp = status.data_ptr()
-    _check(lib().cm_gd_step(code_A.handle, A.data_ptr(), _ld(A, "A"), PA.data_ptr(),
-                            _ld(PA, "PA"), code_AT.handle, AT.data_ptr(), _ld(AT, "AT"),
-                            PAT.data_ptr(), _ld(PAT, "PAT"), y.data_ptr(), x.data_ptr(),
-                            eta, surv_A, surv_AT, ws.data_ptr(), ws.numel(), sp, _stream()),
-           "cm_gd_step")
+    fn = lib().cm_gd_step_survivors if survivors_only else lib().cm_gd_step
+    _check(fn(code_A.handle, A.data_ptr(), _ld(A, "A"), PA.data_ptr(), _ld(PA, "PA"),
+              code_AT.handle, AT.data_ptr(), _ld(AT, "AT"), PAT.data_ptr(), _ld(PAT, "PAT"),
+              y.data_ptr(), x.data_ptr(), eta, surv_A, surv_AT, ws.data_ptr(), ws.numel(), sp,
+              _stream()), "cm_gd_step_survivors" if survivors_only else "cm_gd_step")
     return x
 
 

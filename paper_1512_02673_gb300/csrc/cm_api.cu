@@ -180,7 +180,35 @@ cm_status cm_decode(const cm_code *c, const double *Yt, uint32_t survivors, int3
     if (st != CM_OK) return st;
     if (b < 1 || !Yt || !Y || ((uintptr_t)Yt & 7u) || ((uintptr_t)Y & 3u)) return CM_EINVAL;
     return from_cuda(launch_decode(code_params(c), Yt, eff, b, Y, dev_status,
-                                   DEC_PLAIN, nullptr, 0.f, (cudaStream_t)stream));
+                                   DEC_PLAIN, nullptr, 0.f, false, (cudaStream_t)stream));
+}
+
+size_t cm_matvec_decode_workspace_bytes(const cm_code *c, int32_t b)
+{
+    if (!c || b < 1 || b > 8) return 0;
+    return sizeof(double) * (size_t)c->n * c->L * b;
+}
+
+cm_status cm_matvec_decode(const cm_code *c, const float *A, int64_t lda, const float *par,
+                           int64_t ldp, const float *X, int32_t b, uint32_t survivors,
+                           int32_t only_survivors, float *Y, void *ws, size_t ws_bytes,
+                           int32_t *dev_status, cm_stream_t stream)
+{
+    if (!c || c->dt != CM_F32) return CM_EINVAL;
+    uint32_t eff;
+    cm_status st = resolve_survivors(c, survivors, &eff);
+    if (st != CM_OK) return st;
+    if (b < 1 || b > 8 || !X || !Y || ((uintptr_t)X & 3u) || ((uintptr_t)Y & 3u)) return CM_EINVAL;
+    if (!layout_ok(A, lda, c->d, 4) || !layout_ok(par, ldp, c->d, 4)) return CM_EINVAL;
+    if (!ws || ((uintptr_t)ws & 255u)) return CM_EINVAL;
+    if (ws_bytes < cm_matvec_decode_workspace_bytes(c, b)) return CM_ENOMEM;
+    const CodeParams cp = code_params(c);
+    cudaStream_t s = (cudaStream_t)stream;
+    double *Yt = (double *)ws;
+    if (launch_matvec(cp, A, lda, par, ldp, X, b, Yt, dev_status, only_survivors ? eff : 0u, s) !=
+        cudaSuccess)
+        return CM_ECUDA;
+    return from_cuda(launch_decode(cp, Yt, eff, b, Y, dev_status, DEC_PLAIN, nullptr, 0.f, true, s));
 }
 
 // Workspace of a gradient step: stacked results of both products (fp64) and
@@ -195,11 +223,17 @@ size_t cm_gd_workspace_bytes(const cm_code *cA, const cm_code *cAT)
            round256(sizeof(double) * (size_t)cAT->n * cAT->L);
 }
 
-cm_status cm_gd_step(const cm_code *cA, const float *A, int64_t lda, const float *PA,
-                     int64_t ldpa, const cm_code *cAT, const float *AT, int64_t ldat,
-                     const float *PAT, int64_t ldpat, const float *y, float *x, float eta,
-                     uint32_t surv_A, uint32_t surv_AT, void *ws, size_t ws_bytes,
-                     int32_t *dev_status, cm_stream_t stream)
+namespace {
+
+// Sec. III-E: the master multicasts x, decodes A x from any k1 results,
+// forms z = A x - y, multicasts it, decodes A^T z from any k2 results and
+// steps x <- x - eta A^T z.  Each decode writes the residual or the step
+// itself and is launched as a programmatic dependent of its products.
+cm_status gd_step(const cm_code *cA, const float *A, int64_t lda, const float *PA, int64_t ldpa,
+                  const cm_code *cAT, const float *AT, int64_t ldat, const float *PAT,
+                  int64_t ldpat, const float *y, float *x, float eta, uint32_t surv_A,
+                  uint32_t surv_AT, void *ws, size_t ws_bytes, int32_t *dev_status,
+                  cm_stream_t stream, bool only)
 {
     if (!cA || !cAT || cA->dt != CM_F32 || cAT->dt != CM_F32) return CM_EINVAL;
     if (cAT->m != cA->d || cAT->d != cA->m || cAT->n != cA->n) return CM_EINVAL;
@@ -221,22 +255,43 @@ cm_status cm_gd_step(const cm_code *cA, const float *A, int64_t lda, const float
     float *z = (float *)w;
     w += round256(sizeof(float) * (size_t)cA->m);
     double *ytAT = (double *)w;
-
     cudaStream_t s = (cudaStream_t)stream;
     CodeParams pA = code_params(cA), pAT = code_params(cAT);
-    // Sec. III-E: the master multicasts x, decodes A x from any k1 results ...
-    if (launch_matvec(pA, A, lda, PA, ldpa, x, 1, ytA, dev_status, 0u, s) != cudaSuccess)
+    if (launch_matvec(pA, A, lda, PA, ldpa, x, 1, ytA, dev_status, only ? effA : 0u, s) !=
+        cudaSuccess)
         return CM_ECUDA;
-    // ... forms z = A x - y and multicasts it ...
-    if (launch_decode(pA, ytA, effA, 1, z, dev_status, DEC_RESIDUAL, y, 0.f, s) != cudaSuccess)
+    if (launch_decode(pA, ytA, effA, 1, z, dev_status, DEC_RESIDUAL, y, 0.f, true, s) !=
+        cudaSuccess)
         return CM_ECUDA;
-    // ... decodes A^T z from any k2 results and steps x <- x - eta A^T z.
-    if (launch_matvec(pAT, AT, ldat, PAT, ldpat, z, 1, ytAT, dev_status, 0u, s) != cudaSuccess)
+    if (launch_matvec(pAT, AT, ldat, PAT, ldpat, z, 1, ytAT, dev_status, only ? effAT : 0u, s) !=
+        cudaSuccess)
         return CM_ECUDA;
-    if (launch_decode(pAT, ytAT, effAT, 1, x, dev_status, DEC_DESCENT, nullptr, eta, s) !=
+    if (launch_decode(pAT, ytAT, effAT, 1, x, dev_status, DEC_DESCENT, nullptr, eta, true, s) !=
         cudaSuccess)
         return CM_ECUDA;
     return CM_OK;
+}
+
+}  // namespace
+
+cm_status cm_gd_step(const cm_code *cA, const float *A, int64_t lda, const float *PA,
+                     int64_t ldpa, const cm_code *cAT, const float *AT, int64_t ldat,
+                     const float *PAT, int64_t ldpat, const float *y, float *x, float eta,
+                     uint32_t surv_A, uint32_t surv_AT, void *ws, size_t ws_bytes,
+                     int32_t *dev_status, cm_stream_t stream)
+{
+    return gd_step(cA, A, lda, PA, ldpa, cAT, AT, ldat, PAT, ldpat, y, x, eta, surv_A, surv_AT,
+                   ws, ws_bytes, dev_status, stream, false);
+}
+
+cm_status cm_gd_step_survivors(const cm_code *cA, const float *A, int64_t lda, const float *PA,
+                               int64_t ldpa, const cm_code *cAT, const float *AT, int64_t ldat,
+                               const float *PAT, int64_t ldpat, const float *y, float *x,
+                               float eta, uint32_t surv_A, uint32_t surv_AT, void *ws,
+                               size_t ws_bytes, int32_t *dev_status, cm_stream_t stream)
+{
+    return gd_step(cA, A, lda, PA, ldpa, cAT, AT, ldat, PAT, ldpat, y, x, eta, surv_A, surv_AT,
+                   ws, ws_bytes, dev_status, stream, true);
 }
 
 cm_status cm_coded_gemm(const cm_code *c, const void *A, int64_t lda, const void *par,

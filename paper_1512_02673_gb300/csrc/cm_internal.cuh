@@ -58,9 +58,12 @@ cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda,
 
 // Decode epilogues (Sec. III-E: the two decodes of a gradient step).
 enum DecodeMode { DEC_PLAIN = 0, DEC_RESIDUAL = 1, DEC_DESCENT = 2 };
+// dependent: launched as a programmatic dependent of the kernel before it on
+// the stream (the worker products), which it waits for before reading
+// anything but its parameters; the plan then forms while the products end.
 cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survivors,
                           int b, float *Y, int32_t *status, int mode,
-                          const float *lab, float eta, cudaStream_t s);
+                          const float *lab, float eta, bool dependent, cudaStream_t s);
 cudaError_t launch_decode_mat(const CodeParams &cp, const float *Ct, int64_t ldc,
                               uint32_t survivors, int N, float *C, int64_t ldcc,
                               int32_t *status, cudaStream_t s);

@@ -48,7 +48,13 @@ struct DecodeArgs {
     const float *lab;
     float eta;
     int64_t chunk;            // row positions per CTA
+    int32_t dependent;        // launched as a programmatic dependent of the products
 };
+
+__device__ __forceinline__ void griddep_wait()
+{
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+}
 
 __device__ __forceinline__ void store_out(const DecodeArgs &a, int64_t out, float y_hi, float y_lo)
 {
@@ -92,15 +98,29 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     const int64_t p0 = (int64_t)blockIdx.x * a.chunk;
     const int64_t n = (per_block - p0 < a.chunk ? per_block - p0 : a.chunk);
     plan_setup(a.cp, a.survivors, pl);
-    bool dec = false;
+    // As a programmatic dependent of the products, the whole plan is formed
+    // (from the kernel parameters alone) while the products finish, then the
+    // grid waits for them before it reads a result; otherwise the first
+    // tile's loads overlap the elimination.
+    const bool overlap = !a.dependent;
+    bool dec = false, rows_done = false;
+    if (!overlap) {
+        if (e > 0 && tid < 32 * NW) plan_eliminate<EMAX, NW>(pl, k);
+        __syncthreads();
+        if (e > 0 && !pl.singular) {
+            plan_rows(pl, k, Dh, Dl);
+            dec = true;
+        }
+        rows_done = true;
+        griddep_wait();
+    }
     for (int64_t t0 = 0; t0 < n; t0 += kTile) {
         const int tn = (int)(n - t0 < kTile ? n - t0 : kTile);
         const bool first = t0 == 0;
-        const bool elim = first && e > 0 && tid < 32 * NW;
-        if (elim) plan_eliminate<EMAX, NW>(pl, k);
+        if (overlap && first && e > 0 && tid < 32 * NW) plan_eliminate<EMAX, NW>(pl, k);
         // stage the tile; the eliminating warps skip the first one
         {
-            const int lo = first && e > 0 ? 32 * NW : 0;
+            const int lo = overlap && first && e > 0 ? 32 * NW : 0;
             for (int u = tid - lo; u >= 0 && u < k * tn; u += kThreads - lo) {
                 const int p = u / tn, q = u - p * tn;
                 const int s = pl.S[p];
@@ -121,13 +141,12 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
         if (e == 0) continue;
         __syncthreads();
         if (first) {
-            dec = !pl.singular;
-            if (!dec) {
-                if (blockIdx.x == 0 && tid == 0 && a.status) *a.status = CM_ESINGULAR;
-            } else {
-                plan_rows(pl, k, Dh, Dl);
+            if (pl.singular && blockIdx.x == 0 && tid == 0 && a.status) *a.status = CM_ESINGULAR;
+            if (!rows_done) {
+                dec = !pl.singular;
+                if (dec) plan_rows(pl, k, Dh, Dl);
+                __syncthreads();
             }
-            __syncthreads();
         }
         if (dec) {
             for (int u = tid; u < e * tn; u += kThreads) {
@@ -291,17 +310,31 @@ cudaError_t launch_k3(const DecodeArgs &a, unsigned grid, cudaStream_t s)
     static const cudaError_t attr =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
     if (attr != cudaSuccess) return attr;
-    kern<<<grid, kThreads, kSmem, s>>>(a);
-    return cudaGetLastError();
+    if (!a.dependent) {
+        kern<<<grid, kThreads, kSmem, s>>>(a);
+        return cudaGetLastError();
+    }
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmem;
+    cfg.stream = s;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
 }  // namespace
 
 cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survivors, int b,
                           float *Y, int32_t *status, int mode, const float *lab, float eta,
-                          cudaStream_t s)
+                          bool dependent, cudaStream_t s)
 {
     DecodeArgs a;
+    a.dependent = dependent ? 1 : 0;
     a.cp = cp;
     a.b = b;
     a.survivors = survivors;

@@ -187,6 +187,14 @@ __device__ __forceinline__ Unit unit_of(const MatvecArgs &a, int64_t g, int R)
     return u;
 }
 
+// Lets a programmatic dependent launch (the decode of these products) start:
+// its CTAs form their decode plan on SMs this grid leaves free, then wait
+// for this grid to complete before they read any result.
+__device__ __forceinline__ void griddep_launch_dependents()
+{
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
+
 template <int BP, int R, int ST, int F, int kWarps, int XF>
 __global__ void __launch_bounds__(kWarps * 32, 1)
 matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmP,
@@ -257,6 +265,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
         while (p_idx < my_pairs && p_idx < NG) produce();
 
     stage_x<BP, XF, kThreads>(a, xs, 0);
+    griddep_launch_dependents();
 
     // ---- consumer ----
     int xbuf = 0;             // X buffer of the current chunk
@@ -424,11 +433,12 @@ int matvec_rows_per_unit(int64_t L, int nw, int64_t warps)
     return fill(4) >= fill(8) + 0.02 ? 4 : 8;
 }
 
-cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, const float *par,
-                          int64_t ldp, const float *X, int b, double *Yt, int32_t *status,
-                          uint32_t only, cudaStream_t s)
+namespace {
+
+MatvecArgs matvec_args(const CodeParams &cp, const float *X, int b, double *Yt, int32_t *status,
+                       uint32_t only)
 {
-    MatvecArgs a;
+    MatvecArgs a = {};
     // workers to compute: all n, or the first k set bits of `only`
     a.nw = 0;
     for (int j = 0; j < cp.n; ++j)
@@ -444,6 +454,16 @@ cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, con
     a.b = b;
     a.groups = 0;
     a.fast16 = b == 1 && ((uintptr_t)X & 15u) == 0;
+    return a;
+}
+
+}  // namespace
+
+cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, const float *par,
+                          int64_t ldp, const float *X, int b, double *Yt, int32_t *status,
+                          uint32_t only, cudaStream_t s)
+{
+    const MatvecArgs a = matvec_args(cp, X, b, Yt, status, only);
     if (b == 1) {
         if (matvec_rows_per_unit(a.L, a.nw, (int64_t)cm_sm_count() * 8) == 4)
             return launch_bp<1, 4, 12, 16, 8>(a, A, lda, par, ldp, s);

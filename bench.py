@@ -615,8 +615,8 @@ def runtime_model_report(cm) -> dict:
 def bench_gd(cm, dev, steps: int, w: synth.GDWorkload = synth.GD) -> dict:
     """Coded GD (default: the 40000 x 8000 regression): seconds per iteration
     (4 launches: two coded products, two decodes with the residual and the
-    descent fused into them),
-    effective GB/s."""
+    descent fused into them, each a programmatic dependent of its products),
+    effective GB/s over all n workers' bytes; and the survivors-only step."""
     A, _, y = synth.regression_inputs(w, device=dev)
     AT = A.t().contiguous()
     cA = cm.Code(w.n, w.k_a, w.m, w.d, synth.parity_coefficients(w.n, w.k_a))
@@ -630,17 +630,25 @@ def bench_gd(cm, dev, steps: int, w: synth.GDWorkload = synth.GD) -> dict:
     masks = [(cm.draw_erasures(synth.ERASURE_SEED, 2 * t, w.n, w.k_a)[0],
               cm.draw_erasures(synth.ERASURE_SEED, 2 * t + 1, w.n, w.k_at)[0])
              for t in range(w.iters)]
-    for t in range(3):
-        cm.gd_step(cA, A, PA, cAT, AT, PAT, y, x, w.eta, masks[t][0], masks[t][1], ws, status)
-    x.zero_()
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
-    for t in range(w.iters):
-        cm.gd_step(cA, A, PA, cAT, AT, PAT, y, x, w.eta, masks[t][0], masks[t][1], ws, status)
-    e1.record()
-    torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / w.iters
+    def run(survivors_only):
+        x.zero_()
+        for t in range(3):
+            cm.gd_step(cA, A, PA, cAT, AT, PAT, y, x, w.eta, masks[t][0], masks[t][1], ws,
+                       status, survivors_only=survivors_only)
+        x.zero_()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for t in range(w.iters):
+            cm.gd_step(cA, A, PA, cAT, AT, PAT, y, x, w.eta, masks[t][0], masks[t][1], ws,
+                       status, survivors_only=survivors_only)
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / w.iters
+
+    ms_surv = run(True)
+    x_surv = x.clone()
+    ms = run(False)
     nb = gd_iter_bytes(w, cA.L, cAT.L)
     # the same 50 iterations as plain (uncoded) fp64 gradient descent on the
     # device: the coded iterate must follow it (Sec. III-E: decoding is exact)
@@ -649,10 +657,13 @@ def bench_gd(cm, dev, steps: int, w: synth.GDWorkload = synth.GD) -> dict:
     for t in range(w.iters):
         x64 -= w.eta * (A64.t() @ (A64 @ x64 - y64))
     rel = float(torch.linalg.norm(x.double() - x64) / torch.linalg.norm(x64))
+    rel_surv = float(torch.linalg.norm(x_surv.double() - x64) / torch.linalg.norm(x64))
     del A64
     return {"workload": w.name, "iters": w.iters, "ms_per_iter": ms,
             "gbs": nb / (ms * 1e-3) / 1e9, "launches_per_iter": 4,
-            "x50_rel_err_vs_fp64_gd": rel, "status": int(status.item())}
+            "x50_rel_err_vs_fp64_gd": rel,
+            "survivors_only": {"ms_per_iter": ms_surv, "x50_rel_err_vs_fp64_gd": rel_surv},
+            "status": int(status.item())}
 
 
 def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
@@ -769,10 +780,32 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
     torch.cuda.synchronize()
     mv = np.array([e[0].elapsed_time(e[1]) * 1e3 for e in ev])
     dec = np.array([e[1].elapsed_time(e[2]) * 1e3 for e in ev])
+    # products and decode in one call (the decode a programmatic dependent of
+    # the products), all n workers and the k survivors only: per repeat
+    ws = torch.empty(cm.matvec_decode_workspace_bytes(code, w.b), dtype=torch.uint8, device=dev)
+    one_call = {}
+    for name, only in (("all_workers", False), ("survivors_only", True)):
+        for r in range(3):
+            cm.matvec_decode(code, A, parity, X, masks[r], only_survivors=only, Y=Y, ws=ws,
+                             status=status)
+        torch.cuda.synchronize()
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(reps)]
+        torch.cuda._sleep(int(2e6 + reps * 4e5))
+        for r in range(reps):
+            if flush is not None:
+                flush.fill_(r & 255)
+            evs[r][0].record()
+            cm.matvec_decode(code, A, parity, X, masks[r], only_survivors=only, Y=Y, ws=ws,
+                             status=status)
+            evs[r][1].record()
+        torch.cuda.synchronize()
+        t = np.array([e[0].elapsed_time(e[1]) * 1e3 for e in evs])
+        one_call[name] = {"us_median": float(np.median(t)), "us_p95": float(np.percentile(t, 95))}
     nb = step_bytes(w, code.L)
     peaks = measured_peaks()
     mv_gbs = nb["matvec"] / (np.median(mv) * 1e-6) / 1e9
     return {"workload": w.name, "repeats": reps, "l2_flushed": flush is not None,
+            "matvec_decode_one_call": one_call,
             "matvec_pct_of_measured_hbm": 100.0 * mv_gbs / peaks["hbm_gbs"],
             "matvec_pct_of_nominal_hbm": 100.0 * mv_gbs / NOMINAL_HBM_GBS,
             "encode_us": enc_us,

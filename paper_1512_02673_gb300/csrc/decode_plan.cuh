@@ -16,35 +16,33 @@
 // a decode is one launch and keeps no state between calls:
 //  * plan_setup (all threads): P into shared memory (16-byte loads of the
 //    parameter space), the survivor lists by ballots in warp 0.
-//  * plan_eliminate (warp 0 alone): Q^-1 in fp64 with [Q | I] held in the
-//    warp's registers, its 2e^2 entries spread over the 32 lanes (e <= 16).
-//    No CTA barrier per column: the pivot search is one warp reduction over
-//    the lanes holding the pivot column, the multipliers and the pivot row
-//    travel by shuffles.  The elimination is fraction-free and exchanges no
-//    rows: at column c with pivot row b (the largest |W[r][c]| among rows not
-//    yet used, compared on the leading 28 bits of the magnitude, lowest row on
-//    near-ties) every other row r becomes 2^-s (piv W[r] - W[r][c] W[b]), 2^s
-//    the pivot's binade (an exact scale that keeps the rows from growing by a
-//    product of pivots).  Afterwards row prow[c] holds column c's pivot d_c
-//    and Q^-1[c][a] = W[prow[c]][e + a] / d_c, kept as (high, low) fp32 pairs.
+//  * plan_eliminate (one warp for e <= 4, else four warps, one per
+//    scheduler): Q^-1 in fp64 with [Q | I] held in registers, its 2e^2
+//    entries spread over the threads.  The pivot search is one warp
+//    reduction over the threads holding the pivot column; that warp hands
+//    the pivot key and the column to the others through shared memory (one
+//    named barrier per column), and the pivot row travels by shuffles.  The
+//    elimination is fraction-free and exchanges no rows: at column c with
+//    pivot row b (the largest |W[r][c]| among rows not yet used, compared on
+//    the leading 28 bits of the magnitude, lowest row on near-ties) every
+//    other row r becomes 2^-s (piv W[r] - W[r][c] W[b]), 2^s the pivot's
+//    binade (an exact scale that keeps the rows from growing by a product of
+//    pivots).  Afterwards row prow[c] holds column c's pivot d_c and
+//    Q^-1[c][a] = W[prow[c]][e + a] / d_c, kept as (high, low) fp32 pairs.
 //  * G_S counts as singular when a pivot is zero, subnormal or not finite, or
 //    when ||Q||_inf ||Q^-1||_inf, bounded by (e max|Q|)(e max|Q^-1|), exceeds
 //    1 / (64 eps) (evaluated in fp32: it is a threshold).
-// The apply then takes the residual form of the same rows: for each
-// surviving parity worker Ps[a],
-//   r_a = Yt_Ps[a] - sum_p P[Ps[a]][S[p]] Yt_S[p]   (p over the ks systematic survivors)
-// is the part of its result that the missing blocks produce, and
-//   missing block M[c] = sum_a Q^-1[c][a] r_a,
-// which is sum_p D[c][p] Yt_S[p] regrouped: the code coefficients enter as
-// their exact fp32 values and only the e x e inverse comes from the plan.
+//  * plan_rows (all threads): the rows D[c][p] above, from the (high, low)
+//    pairs of Q^-1 and the exact fp32 values of P in double-float arithmetic.
 //
 // fp64 runs at a small fraction of the fp32 rate on this part: each warp
 // gets about one fp64 instruction per 64 cycles, whatever the independence
 // of its instructions, and a division takes about 430 cycles.  So
 // conversions and magnitude compares go through integer bit manipulation,
 // each column of the elimination costs one fp64 multiply and one fp64 fma per
-// entry a lane holds (1, 4 or 16 entries for e <= 4, 8, 16), and the only
-// divisions are the e reciprocals of the pivots, taken in parallel.
+// entry a thread holds (1 for e <= 8, 4 for e <= 16), spread over warps on
+// different schedulers, and the only divisions are the e reciprocals of the
+// pivots, taken in parallel.
 #pragma once
 
 #include <cfloat>

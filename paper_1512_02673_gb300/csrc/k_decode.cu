@@ -2,28 +2,24 @@
 // paragraph; Example "MDS codes").
 //
 // One launch per decode and no state kept between calls: every CTA forms the
-// inverse of the e x e block Q of G_S in its own shared memory
-// (decode_plan.cuh: one warp eliminates in fp64 in registers while the other
-// threads' loads of their first surviving values are in flight), then applies
-// the rows of G_S^-1 for the missing systematic blocks in residual form:
-// r_a = Yt_Ps[a] - sum_p P[Ps[a]][S[p]] Yt_S[p] over the surviving systematic
-// blocks, then missing block M[c] = sum_a Q^-1[c][a] r_a, while surviving
-// systematic blocks pass through.  Each surviving value is read once, by the
-// thread that owns its row position, which writes all k output blocks of that
-// position.  A zero (or relatively negligible) pivot marks G_S singular:
+// decode in its own shared memory (decode_plan.cuh: the e x e block Q of G_S
+// inverted in fp64 in registers by one or four warps, then the rows D of
+// G_S^-1 for the missing systematic blocks), and applies it: missing block
+// M[c] = sum_p D[c][p] Yt_S[p] over the k surviving results, while surviving
+// systematic blocks pass through.  Each surviving value is loaded once per
+// CTA.  A zero (or relatively negligible) pivot marks G_S singular:
 // CM_ESINGULAR goes to the status word and no missing block is written
 // (surviving systematic blocks are still copied).
 //
 // fp64 arithmetic runs at a small fraction of the fp32 rate on this part, so
 // the vector decode works in double-float arithmetic on the fp32 pipe: each
-// fp64 worker result and each entry of Q^-1 is split into a (high, low) fp32
-// pair by integer bit manipulation, the code coefficients are exact fp32
-// values, products are formed exactly with an FMA and the sums are kept as
-// (sum, compensation) pairs (Knuth's TwoSum), about 2^-44 relative per term,
-// far below the rounding of the fp32 output; fp32 outputs of fp64 values are
-// rounded to nearest even by integer arithmetic.  The matrix decode (fp32
-// results of the tensor-core products) works in fp32 with both parts of
-// Q^-1.
+// fp64 worker result and each row entry is a (high, low) fp32 pair split by
+// integer bit manipulation, products are formed exactly with an FMA and the
+// sums are kept as (sum, compensation) pairs (Knuth's TwoSum), about 2^-44
+// relative per term, far below the rounding of the fp32 output; fp32 outputs
+// of fp64 values are rounded to nearest even by integer arithmetic.  The
+// matrix decode (fp32 results of the tensor-core products) applies the rows'
+// high parts in fp32.
 #include <algorithm>
 
 #include "cm_internal.cuh"
@@ -178,18 +174,23 @@ struct DecodeMatArgs {
 };
 
 // K6: fp32 results, all e missing blocks of one row position (4 columns when
-// aligned) per thread, so every surviving element is read once.  The loads of
-// a batch of survivors are issued together before their FMAs.
+// aligned) per thread, so every surviving element is read once.  Every CTA
+// forms the plan and the rows D (as K3), then streams: the loads of a batch
+// of survivors are issued together before their FMAs, which apply the rows'
+// high parts in fp32.
 template <int EMAX>
 __global__ void __launch_bounds__(kMatThreads) decode_mat_kernel(const __grid_constant__ DecodeMatArgs a)
 {
     __shared__ Plan pl;
+    __shared__ float Dh[kMaxE][CM_MAX_N], Dl[kMaxE][CM_MAX_N];
     plan_setup(a.cp, a.survivors, pl);
-    const int k = a.cp.k, e = pl.e, ks = k - e;
-    if (e > 0 && (int)(threadIdx.x >> 5) < (EMAX == 4 ? 1 : 4))
-        plan_eliminate<EMAX, EMAX == 4 ? 1 : 4>(pl, k);
+    const int k = a.cp.k, e = pl.e;
+    constexpr int NW = EMAX == 4 ? 1 : 4;
+    if (e > 0 && (int)(threadIdx.x >> 5) < NW) plan_eliminate<EMAX, NW>(pl, k);
     __syncthreads();
     const bool dec = e > 0 && !pl.singular;
+    if (dec) plan_rows(pl, k, Dh, Dl);
+    __syncthreads();
     if (e > 0 && pl.singular && blockIdx.x == 0 && threadIdx.x == 0 && a.status)
         *a.status = CM_ESINGULAR;
     const float *Ct = a.Ct;
@@ -209,26 +210,25 @@ __global__ void __launch_bounds__(kMatThreads) decode_mat_kernel(const __grid_co
          it += (int64_t)gridDim.x * blockDim.x) {
         const int64_t r = it / nw;
         const int64_t col = (it - r * nw) * W;
-        // residuals of the surviving parity workers: P[Ps[q]][s] times every
-        // surviving systematic result s subtracted from their own results
-        float4 res[EMAX];
+        float4 acc[EMAX];
 #pragma unroll
-        for (int q = 0; q < EMAX; ++q) res[q] = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int j0 = 0; j0 < ks; j0 += kBatch) {
+        for (int c = 0; c < EMAX; ++c) acc[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int p0 = 0; p0 < k; p0 += kBatch) {
             float4 v[kBatch];
 #pragma unroll
             for (int u = 0; u < kBatch; ++u) {
-                if (j0 + u < ks) {
-                    const float *src = Ct + ((int64_t)pl.S[j0 + u] * L + r) * ldc + col;
+                if (p0 + u < k) {
+                    const float *src = Ct + ((int64_t)pl.S[p0 + u] * L + r) * ldc + col;
                     v[u] = vec ? __ldg(reinterpret_cast<const float4 *>(src))
                                : make_float4(__ldg(src), 0.f, 0.f, 0.f);
                 }
             }
 #pragma unroll
             for (int u = 0; u < kBatch; ++u) {
-                if (j0 + u >= ks) break;
-                const int s = pl.S[j0 + u];
-                if (!inplace) {   // surviving systematic block passes through
+                const int p = p0 + u;
+                if (p >= k) break;
+                const int s = pl.S[p];
+                if (!inplace && s < k) {   // surviving systematic block passes through
                     const int64_t g = (int64_t)s * L + r;
                     if (g < m) {
                         float *dst = C + g * ldcc + col;
@@ -238,13 +238,13 @@ __global__ void __launch_bounds__(kMatThreads) decode_mat_kernel(const __grid_co
                 }
                 if (dec) {
 #pragma unroll
-                    for (int q = 0; q < EMAX; ++q) {
-                        if (q < e) {
-                            const float w = -pl.P[(pl.Ps[q] - k) * k + s];
-                            res[q].x = fmaf(w, v[u].x, res[q].x);
-                            res[q].y = fmaf(w, v[u].y, res[q].y);
-                            res[q].z = fmaf(w, v[u].z, res[q].z);
-                            res[q].w = fmaf(w, v[u].w, res[q].w);
+                    for (int c = 0; c < EMAX; ++c) {
+                        if (c < e) {
+                            const float w = Dh[c][p];
+                            acc[c].x = fmaf(w, v[u].x, acc[c].x);
+                            acc[c].y = fmaf(w, v[u].y, acc[c].y);
+                            acc[c].z = fmaf(w, v[u].z, acc[c].z);
+                            acc[c].w = fmaf(w, v[u].w, acc[c].w);
                         }
                     }
                 }
@@ -252,38 +252,13 @@ __global__ void __launch_bounds__(kMatThreads) decode_mat_kernel(const __grid_co
         }
         if (dec) {
 #pragma unroll
-            for (int q = 0; q < EMAX; ++q) {
-                if (q < e) {
-                    const float *src = Ct + ((int64_t)pl.Ps[q] * L + r) * ldc + col;
-                    const float4 v = vec ? __ldg(reinterpret_cast<const float4 *>(src))
-                                         : make_float4(__ldg(src), 0.f, 0.f, 0.f);
-                    res[q].x += v.x;
-                    res[q].y += v.y;
-                    res[q].z += v.z;
-                    res[q].w += v.w;
-                }
-            }
-        }
-        if (dec) {
-#pragma unroll 1
-            for (int c = 0; c < e; ++c) {
-                {
-                    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-                    for (int q = 0; q < EMAX; ++q) {
-                        if (q < e) {
-                            const float wh = pl.Qh[c][q], wl = pl.Ql[c][q];
-                            acc.x = fmaf(wh, res[q].x, fmaf(wl, res[q].x, acc.x));
-                            acc.y = fmaf(wh, res[q].y, fmaf(wl, res[q].y, acc.y));
-                            acc.z = fmaf(wh, res[q].z, fmaf(wl, res[q].z, acc.z));
-                            acc.w = fmaf(wh, res[q].w, fmaf(wl, res[q].w, acc.w));
-                        }
-                    }
+            for (int c = 0; c < EMAX; ++c) {
+                if (c < e) {
                     const int64_t g = (int64_t)pl.M[c] * L + r;
                     if (g < m) {
                         float *dst = C + g * ldcc + col;
-                        if (vec) *reinterpret_cast<float4 *>(dst) = acc;
-                        else *dst = acc.x;
+                        if (vec) *reinterpret_cast<float4 *>(dst) = acc[c];
+                        else *dst = acc[c].x;
                     }
                 }
             }

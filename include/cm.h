@@ -158,13 +158,18 @@ cm_status cm_decode(const cm_code *code, const double *Yt, uint32_t survivors,
                     int32_t b, float *Y, int32_t *dev_status, cm_stream_t stream);
 
 /* Workspace bytes cm_matvec_decode needs for b vectors (the stacked results,
- * n L b fp64; 0 on a bad code or b outside 1..8). */
+ * n L b fp64 per column segment; 0 on a bad code or b outside 1..8). */
 size_t cm_matvec_decode_workspace_bytes(const cm_code *code, int32_t b);
 
 /* The worker products and the decode in one call (Sec. III-A: the master
  * needs only the first k results, and decoding is a fixed linear map of
- * them): Y = A X (m x b fp32), equal bit for bit to cm_matvec (or
- * cm_matvec_survivors) followed by cm_decode.  The decode is launched as a
+ * them): Y = A X (m x b fp32), the result of cm_matvec (or
+ * cm_matvec_survivors) followed by cm_decode.  On small problems, whose
+ * units fill the persistent grid poorly, the products are split into 2, 4
+ * or 8 column segments done by separate shares of the SMs, and the decode
+ * adds the segments' fp64 partial sums as it loads them (Y then differs from
+ * the two calls' by the products' own rounding, short fp32 partial sums
+ * being flushed at other columns).  The decode is launched as a
  * programmatic dependent of the products: its CTAs start on the SMs the
  * products leave free in their last round, form the rows of G_S^-1 (the fp64
  * elimination of cm_decode) from the kernel parameters alone, and wait for
@@ -175,9 +180,9 @@ size_t cm_matvec_decode_workspace_bytes(const cm_code *code, int32_t b);
  * first k set bits of `survivors` (for a repetition code, the first survivor
  * of each block), as for cm_decode.  ws is caller device memory of at least
  * cm_matvec_decode_workspace_bytes(code, b) bytes, 256-byte aligned, which
- * receives the stacked worker results (n L x b fp64; rows of workers that did
- * not compute are left unwritten).  Two launches.  Errors as cm_matvec and
- * cm_decode; CM_ENOMEM for a short workspace. */
+ * receives the stacked worker results (n L x b fp64 per column segment;
+ * rows of workers that did not compute are left unwritten).  Two launches.
+ * Errors as cm_matvec and cm_decode; CM_ENOMEM for a short workspace. */
 cm_status cm_matvec_decode(const cm_code *code, const float *A, int64_t lda,
                            const float *parity, int64_t ldp, const float *X, int32_t b,
                            uint32_t survivors, int32_t only_survivors, float *Y, void *ws,

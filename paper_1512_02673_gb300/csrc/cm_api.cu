@@ -183,10 +183,19 @@ cm_status cm_decode(const cm_code *c, const double *Yt, uint32_t survivors, int3
                                    DEC_PLAIN, nullptr, 0.f, false, (cudaStream_t)stream));
 }
 
+// Partial results of the products that cm_matvec_decode may split into
+// column segments: the largest count over both worker sets.
+static int max_segments(const CodeParams &cp, int b)
+{
+    const uint32_t some = (uint32_t)((1ull << cp.k) - 1ull);   // k workers
+    const int a = matvec_segments(cp, b, 0u), s = matvec_segments(cp, b, some);
+    return a > s ? a : s;
+}
+
 size_t cm_matvec_decode_workspace_bytes(const cm_code *c, int32_t b)
 {
     if (!c || b < 1 || b > 8) return 0;
-    return sizeof(double) * (size_t)c->n * c->L * b;
+    return sizeof(double) * (size_t)c->n * c->L * b * (size_t)max_segments(code_params(c), b);
 }
 
 cm_status cm_matvec_decode(const cm_code *c, const float *A, int64_t lda, const float *par,
@@ -205,10 +214,14 @@ cm_status cm_matvec_decode(const cm_code *c, const float *A, int64_t lda, const 
     const CodeParams cp = code_params(c);
     cudaStream_t s = (cudaStream_t)stream;
     double *Yt = (double *)ws;
-    if (launch_matvec(cp, A, lda, par, ldp, X, b, Yt, dev_status, only_survivors ? eff : 0u, s) !=
+    const uint32_t only = only_survivors ? eff : 0u;
+    const int nseg = matvec_segments(cp, b, only);
+    const int64_t part = (int64_t)c->n * c->L * b;
+    if (launch_matvec_split(cp, A, lda, par, ldp, X, b, Yt, dev_status, only, nseg, part, s) !=
         cudaSuccess)
         return CM_ECUDA;
-    return from_cuda(launch_decode(cp, Yt, eff, b, Y, dev_status, DEC_PLAIN, nullptr, 0.f, true, s));
+    return from_cuda(launch_decode(cp, Yt, eff, b, Y, dev_status, DEC_PLAIN, nullptr, 0.f, true, s,
+                                   nseg, part));
 }
 
 // Workspace of a gradient step: stacked results of both products (fp64) and
@@ -218,9 +231,9 @@ static size_t round256(size_t x) { return (x + 255) & ~(size_t)255; }
 size_t cm_gd_workspace_bytes(const cm_code *cA, const cm_code *cAT)
 {
     if (!cA || !cAT) return 0;
-    return round256(sizeof(double) * (size_t)cA->n * cA->L) +
+    return round256(cm_matvec_decode_workspace_bytes(cA, 1)) +
            round256(sizeof(float) * (size_t)cA->m) +
-           round256(sizeof(double) * (size_t)cAT->n * cAT->L);
+           round256(cm_matvec_decode_workspace_bytes(cAT, 1));
 }
 
 namespace {
@@ -251,23 +264,26 @@ cm_status gd_step(const cm_code *cA, const float *A, int64_t lda, const float *P
     if (ws_bytes < cm_gd_workspace_bytes(cA, cAT)) return CM_ENOMEM;
     char *w = (char *)ws;
     double *ytA = (double *)w;
-    w += round256(sizeof(double) * (size_t)cA->n * cA->L);
+    w += round256(cm_matvec_decode_workspace_bytes(cA, 1));
     float *z = (float *)w;
     w += round256(sizeof(float) * (size_t)cA->m);
     double *ytAT = (double *)w;
     cudaStream_t s = (cudaStream_t)stream;
     CodeParams pA = code_params(cA), pAT = code_params(cAT);
-    if (launch_matvec(pA, A, lda, PA, ldpa, x, 1, ytA, dev_status, only ? effA : 0u, s) !=
+    const uint32_t onlyA = only ? effA : 0u, onlyAT = only ? effAT : 0u;
+    const int segA = matvec_segments(pA, 1, onlyA), segAT = matvec_segments(pAT, 1, onlyAT);
+    const int64_t partA = (int64_t)cA->n * cA->L, partAT = (int64_t)cAT->n * cAT->L;
+    if (launch_matvec_split(pA, A, lda, PA, ldpa, x, 1, ytA, dev_status, onlyA, segA, partA, s) !=
         cudaSuccess)
         return CM_ECUDA;
-    if (launch_decode(pA, ytA, effA, 1, z, dev_status, DEC_RESIDUAL, y, 0.f, true, s) !=
-        cudaSuccess)
+    if (launch_decode(pA, ytA, effA, 1, z, dev_status, DEC_RESIDUAL, y, 0.f, true, s, segA,
+                      partA) != cudaSuccess)
         return CM_ECUDA;
-    if (launch_matvec(pAT, AT, ldat, PAT, ldpat, z, 1, ytAT, dev_status, only ? effAT : 0u, s) !=
-        cudaSuccess)
+    if (launch_matvec_split(pAT, AT, ldat, PAT, ldpat, z, 1, ytAT, dev_status, onlyAT, segAT,
+                            partAT, s) != cudaSuccess)
         return CM_ECUDA;
-    if (launch_decode(pAT, ytAT, effAT, 1, x, dev_status, DEC_DESCENT, nullptr, eta, true, s) !=
-        cudaSuccess)
+    if (launch_decode(pAT, ytAT, effAT, 1, x, dev_status, DEC_DESCENT, nullptr, eta, true, s,
+                      segAT, partAT) != cudaSuccess)
         return CM_ECUDA;
     return CM_OK;
 }

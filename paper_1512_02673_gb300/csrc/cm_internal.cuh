@@ -55,15 +55,26 @@ int matvec_rows_per_unit(int64_t L, int nw, int64_t warps);
 cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda,
                           const float *par, int64_t ldp, const float *X, int b,
                           double *Yt, int32_t *status, uint32_t only, cudaStream_t s);
+// Column segments (1, 2, 4 or 8) for products whose consumer adds partial
+// results, and the products written as nseg partial results part_stride
+// doubles apart (nseg = 1: launch_matvec).
+int matvec_segments(const CodeParams &cp, int b, uint32_t only);
+cudaError_t launch_matvec_split(const CodeParams &cp, const float *A, int64_t lda,
+                                const float *par, int64_t ldp, const float *X, int b, double *Yt,
+                                int32_t *status, uint32_t only, int nseg, int64_t part_stride,
+                                cudaStream_t s);
 
 // Decode epilogues (Sec. III-E: the two decodes of a gradient step).
 enum DecodeMode { DEC_PLAIN = 0, DEC_RESIDUAL = 1, DEC_DESCENT = 2 };
 // dependent: launched as a programmatic dependent of the kernel before it on
 // the stream (the worker products), which it waits for before reading
 // anything but its parameters; the plan then forms while the products end.
+// nparts > 1: the products left that many partial results part_stride
+// doubles apart (column segments, launch_matvec_split), summed on load.
 cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survivors,
                           int b, float *Y, int32_t *status, int mode,
-                          const float *lab, float eta, bool dependent, cudaStream_t s);
+                          const float *lab, float eta, bool dependent, cudaStream_t s,
+                          int nparts = 1, int64_t part_stride = 0);
 cudaError_t launch_decode_mat(const CodeParams &cp, const float *Ct, int64_t ldc,
                               uint32_t survivors, int N, float *C, int64_t ldcc,
                               int32_t *status, cudaStream_t s);

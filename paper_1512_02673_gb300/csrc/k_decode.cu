@@ -45,6 +45,8 @@ struct DecodeArgs {
     float eta;
     int64_t chunk;            // row positions per CTA
     int32_t dependent;        // launched as a programmatic dependent of the products
+    int32_t nparts;           // Yt holds this many partial results of the products ...
+    int64_t part_stride;      // ... this many doubles apart; their sum is the result
 };
 
 __device__ __forceinline__ void griddep_wait()
@@ -121,7 +123,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
                 const int p = u / tn, q = u - p * tn;
                 const int s = pl.S[p];
                 const int64_t src = (int64_t)s * per_block + p0 + t0 + q;
-                const double y = a.Yt[src];
+                double y = a.Yt[src];
+                for (int h = 1; h < a.nparts; ++h) y += a.Yt[src + h * a.part_stride];
                 if (e > 0) ysm[p * kTile + q] = y;
                 if (s < k && src < mb) {      // surviving systematic block: pass through
                     if (a.mode == DEC_PLAIN) {
@@ -306,10 +309,12 @@ cudaError_t launch_k3(const DecodeArgs &a, unsigned grid, cudaStream_t s)
 
 cudaError_t launch_decode(const CodeParams &cp, const double *Yt, uint32_t survivors, int b,
                           float *Y, int32_t *status, int mode, const float *lab, float eta,
-                          bool dependent, cudaStream_t s)
+                          bool dependent, cudaStream_t s, int nparts, int64_t part_stride)
 {
     DecodeArgs a;
     a.dependent = dependent ? 1 : 0;
+    a.nparts = nparts;
+    a.part_stride = part_stride;
     a.cp = cp;
     a.b = b;
     a.survivors = survivors;

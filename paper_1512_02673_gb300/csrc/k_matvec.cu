@@ -79,6 +79,12 @@ struct MatvecArgs {
     int64_t groups;        // total work units
     int32_t nw;            // workers computed: all n, or only the k survivors
     int8_t wmap[CM_MAX_N]; // computed worker slot -> worker index
+    // column segments: CTA c sums the 128-column steps
+    // [s seg_steps, (s + 1) seg_steps) of every unit, s = c % nseg, into the
+    // partial results Yt + s part_stride (nseg = 1: whole rows into Yt)
+    int32_t nseg;
+    int32_t seg_steps;
+    int64_t part_stride;
 };
 
 __device__ __forceinline__ void cp_async16(float *dst, const float *src, int bytes)
@@ -198,7 +204,7 @@ __device__ __forceinline__ void griddep_launch_dependents()
 template <int BP, int R, int ST, int F, int kWarps, int XF>
 __global__ void __launch_bounds__(kWarps * 32, 1)
 matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmP,
-              const MatvecArgs a)
+              const __grid_constant__ MatvecArgs a)
 {
     constexpr int kThreads = kWarps * 32;
     using C = XCfg<BP, XF>;
@@ -228,11 +234,17 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     cm_fence_mbar_init();
     __syncthreads();
 
-    const int64_t total_warps = (int64_t)gridDim.x * kWarps;
-    const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
+    // this CTA's column segment; the CTAs of one segment share its units
+    const int seg = (int)(blockIdx.x % a.nseg);
+    const int64_t total_warps = (int64_t)(gridDim.x / a.nseg) * kWarps;
+    const int64_t gw = (int64_t)(blockIdx.x / a.nseg) * kWarps + warp;
     const int rounds = (int)((a.groups + total_warps - 1) / total_warps);
-    const int steps = (int)((a.d + 127) / 128);
-    const int nchunks = (int)((a.d + C::CX - 1) / C::CX);
+    const int s0 = seg * a.seg_steps;   // the segment's first step
+    const int all_steps = (int)((a.d + 127) / 128);
+    const int steps = all_steps - s0 < a.seg_steps ? all_steps - s0 : a.seg_steps;
+    const int64_t col0 = (int64_t)s0 * 128;
+    const int nchunks = (steps * 128 + C::CX - 1) / C::CX;
+    double *const Yt = a.Yt + (int64_t)seg * a.part_stride;
     // rounds in which this warp has a unit (a prefix: unit index grows with round)
     const int64_t my_rounds = gw < a.groups ? (a.groups - 1 - gw) / total_warps + 1 : 0;
     // A unit's steps go in groups of GS (the last one shorter when GS does
@@ -251,7 +263,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
         cm_mbar_arrive_expect_tx(&bar[p_g], nb * STEP_BYTES);
         for (int u = 0; u < nb; ++u)
             cm_tma_load_2d(ring + (GS * p_g + u) * S::SLOT_FLOATS, pu.parity ? &tmP : &tmA,
-                           128 * (p_s + u), pu.y, &bar[p_g]);
+                           (int32_t)(col0 + 128 * (p_s + u)), pu.y, &bar[p_g]);
         ++p_idx;
         p_g = p_g + 1 == NG ? 0 : p_g + 1;
         p_s += nb;
@@ -264,7 +276,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     if (lane == 0)
         while (p_idx < my_pairs && p_idx < NG) produce();
 
-    stage_x<BP, XF, kThreads>(a, xs, 0);
+    stage_x<BP, XF, kThreads>(a, xs, col0);
     griddep_launch_dependents();
 
     // ---- consumer ----
@@ -323,7 +335,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
             __syncthreads();   // X chunk visible; every warp is done with the other buffer
             if (ch + 1 < nchunks || round + 1 < rounds)
                 stage_x<BP, XF, kThreads>(a, xs + (xbuf ^ 1) * C::FLOATS,
-                                      ch + 1 < nchunks ? (int64_t)(ch + 1) * C::CX : 0);
+                                      col0 + (ch + 1 < nchunks ? (int64_t)(ch + 1) * C::CX : 0));
             const int ns = steps - ch * IPC < IPC ? steps - ch * IPC : IPC;
             if (has && !failed) {
                 const float *xchunk = xs + xbuf * C::FLOATS + 4 * lane;
@@ -363,14 +375,14 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
                 for (int i = 0; i < NH; ++i) {
                     const int vi = lane * NH + i;
                     const int r = vi / BP, v = vi % BP;
-                    if (v < a.b && cu.rr0 + r < a.L) a.Yt[(obase + r) * a.b + v] = acc64[i];
+                    if (v < a.b && cu.rr0 + r < a.L) Yt[(obase + r) * a.b + v] = acc64[i];
                 }
             } else {
                 constexpr int SHIFT = V == 1 ? 5 : V == 2 ? 4 : V == 4 ? 3 : V == 8 ? 2 : 1;
                 if ((lane & ((1 << SHIFT) - 1)) == 0) {
                     const int vi = lane >> SHIFT;
                     const int r = vi / BP, v = vi % BP;
-                    if (v < a.b && cu.rr0 + r < a.L) a.Yt[(obase + r) * a.b + v] = acc64[0];
+                    if (v < a.b && cu.rr0 + r < a.L) Yt[(obase + r) * a.b + v] = acc64[0];
                 }
             }
         }
@@ -406,10 +418,12 @@ cudaError_t launch_bp(MatvecArgs a, const float *A, int64_t lda, const float *pa
                                          S::TOTAL);
     if (e != cudaSuccess) return e;
     a.groups = (a.L + R - 1) / R * a.nw;
+    // CTAs per segment: as many as the SMs allow, no more than the units need
     const int64_t need = (a.groups + kWarps - 1) / kWarps;
-    int64_t grid = cm_sm_count();
-    if (grid < 1) grid = 1;
-    if (grid > need) grid = need;
+    int64_t per_seg = (cm_sm_count() > 0 ? cm_sm_count() : 1) / a.nseg;
+    if (per_seg < 1) per_seg = 1;
+    if (per_seg > need) per_seg = need;
+    const int64_t grid = per_seg * a.nseg;
     kern<<<(unsigned)grid, kThreads, S::TOTAL, s>>>(tmA, tmP, a);
     return cudaGetLastError();
 }
@@ -454,21 +468,84 @@ MatvecArgs matvec_args(const CodeParams &cp, const float *X, int b, double *Yt, 
     a.b = b;
     a.groups = 0;
     a.fast16 = b == 1 && ((uintptr_t)X & 15u) == 0;
+    a.nseg = 1;
+    a.seg_steps = (int32_t)((cp.d + 127) / 128);
+    a.part_stride = 0;
     return a;
 }
 
+// Rows per unit of the launch for these arguments (the kernel instance).
+int unit_rows(const MatvecArgs &a)
+{
+    const int sms = cm_sm_count() > 0 ? cm_sm_count() : 1;
+    if (a.b == 1) return matvec_rows_per_unit(a.L, a.nw, (int64_t)sms * 8);
+    return 8;
+}
+
+cudaError_t dispatch(const MatvecArgs &a, const float *A, int64_t lda, const float *par,
+                     int64_t ldp, cudaStream_t s)
+{
+    if (a.b == 1) {
+        if (unit_rows(a) == 4) return launch_bp<1, 4, 12, 16, 8>(a, A, lda, par, ldp, s);
+        return launch_bp<1, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
+    }
+    if (a.b <= 4) return launch_bp<4, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
+    return launch_bp<8, 8, 6, 64, 8>(a, A, lda, par, ldp, s);
+}
+
 }  // namespace
+
+// Column segments for the products of a decode that adds partial results.
+// The persistent grid runs the units in rounds over its warps; when there are
+// few units (few rows per worker, long rows: the 400 x 10000 regression of
+// Sec. III-F has 70 units of 8 rows for 1216 warps), splitting every unit's
+// columns into 2, 4 or 8 segments, each done by its own share of the CTAs,
+// puts more warps to work.  The time is modelled as rounds x (T0 + steps of
+// the segment), T0 = 5 steps the fixed cost of a unit (ring start-up, flush,
+// result stores), fitted on this part: (25,23) at 5750 x 5750 ran equally
+// fast whole (1 round of 45 steps) and in 4 segments (3 rounds of 12).  Taken
+// only when the model drops by a tenth or more and every segment keeps at
+// least 8 steps of 128 columns.
+int matvec_segments(const CodeParams &cp, int b, uint32_t only)
+{
+    const MatvecArgs a = matvec_args(cp, nullptr, b, nullptr, nullptr, only);
+    const int R = unit_rows(a);
+    const int64_t units = (a.L + R - 1) / R * a.nw;
+    const int sms = cm_sm_count() > 0 ? cm_sm_count() : 1;
+    const int steps = a.seg_steps;
+    auto cost = [&](int ns) {
+        const int64_t warps = (int64_t)(sms / ns) * 8;
+        const int seg_steps = (steps + ns - 1) / ns;
+        return (double)((units + warps - 1) / warps) * (5.0 + seg_steps);
+    };
+    int best = 1;
+    double best_c = cost(1);
+    for (int ns = 2; ns <= 8; ns *= 2) {
+        if (sms % ns || (steps + ns - 1) / ns < 8) break;
+        const double c = cost(ns);
+        if (c <= 0.9 * best_c) {
+            best = ns;
+            best_c = c;
+        }
+    }
+    return best;
+}
+
+cudaError_t launch_matvec_split(const CodeParams &cp, const float *A, int64_t lda,
+                                const float *par, int64_t ldp, const float *X, int b, double *Yt,
+                                int32_t *status, uint32_t only, int nseg, int64_t part_stride,
+                                cudaStream_t s)
+{
+    MatvecArgs a = matvec_args(cp, X, b, Yt, status, only);
+    a.nseg = nseg;
+    a.seg_steps = (a.seg_steps + nseg - 1) / nseg;
+    a.part_stride = part_stride;
+    return dispatch(a, A, lda, par, ldp, s);
+}
 
 cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, const float *par,
                           int64_t ldp, const float *X, int b, double *Yt, int32_t *status,
                           uint32_t only, cudaStream_t s)
 {
-    const MatvecArgs a = matvec_args(cp, X, b, Yt, status, only);
-    if (b == 1) {
-        if (matvec_rows_per_unit(a.L, a.nw, (int64_t)cm_sm_count() * 8) == 4)
-            return launch_bp<1, 4, 12, 16, 8>(a, A, lda, par, ldp, s);
-        return launch_bp<1, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
-    }
-    if (b <= 4) return launch_bp<4, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
-    return launch_bp<8, 8, 6, 64, 8>(a, A, lda, par, ldp, s);
+    return dispatch(matvec_args(cp, X, b, Yt, status, only), A, lda, par, ldp, s);
 }

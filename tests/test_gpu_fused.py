@@ -1,10 +1,14 @@
-"""GPU parity of the worker products with the decode fused into their tail
+"""GPU parity of the worker products and the decode in one call
 (cm_matvec_decode, Sec. III-A: the master needs only k results).
 
-The fused path runs the same operations in the same order as cm_matvec (or
-cm_matvec_survivors) followed by cm_decode, so its Y must equal theirs bit for
-bit; it is also checked against the oracle's plain A X at the contract's
-relative l2 tolerance (1e-4 per output vector).
+The one call runs the operations of cm_matvec (or cm_matvec_survivors)
+followed by cm_decode.  Its Y equals theirs bit for bit, except on small
+problems whose products it splits into column segments: each segment then
+flushes its short fp32 partial sums into fp64 at other columns, so the worker
+results differ by their own rounding (about 1e-7 relative), which the decode
+amplifies by up to the condition number of G_S (relative l2 <= 1e-5 per
+vector between the two).  Y is also checked against the oracle's plain A X at
+the contract's relative l2 tolerance (1e-4 per output vector).
 """
 import numpy as np
 import pytest
@@ -27,6 +31,13 @@ def cm():
         from paper_1512_02673_gb300 import build
         build.build()
     return cm
+
+
+def same_or_reordered(Y, Y_sep):
+    """Bit-equal, or (column segments) within the products' rounding."""
+    if torch.equal(Y, Y_sep):
+        return True
+    return rel_l2_cols(Y.cpu().numpy(), Y_sep.cpu().numpy()).max() <= 1e-5
 
 
 def separate(cm, code, A, par, X, mask, only):
@@ -55,7 +66,7 @@ def test_fused_equals_products_then_decode(cm, orc, n, k, m, d, b, lda, only):
         Y_sep = separate(cm, code, A, par, X, mask, only)
         torch.cuda.synchronize()
         assert status.item() == 0
-        assert torch.equal(Y, Y_sep), counter
+        assert same_or_reordered(Y, Y_sep), counter
         assert rel_l2_cols(Y.cpu().numpy(), want).max() <= 1e-4
 
 
@@ -80,7 +91,7 @@ def test_fused_every_erasure_count(cm, orc, only):
         Y = cm.matvec_decode(code, A, par, X, mask, only_survivors=only)
         Y_sep = separate(cm, code, A, par, X, mask, only)
         torch.cuda.synchronize()
-        assert torch.equal(Y, Y_sep), e
+        assert same_or_reordered(Y, Y_sep), e
         # the decode stage: the oracle's fp64 decode of the same products
         Yo = orc.decode(n, k, m, P.astype(np.float64), mask, Yt.cpu().numpy())
         assert rel_l2_cols(Y.cpu().numpy(), Yo).max() <= 1e-6, e

@@ -763,15 +763,23 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
     enc_us = e0.elapsed_time(e1) * 1e3
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(reps)]
     # inputs that fit in L2 are flushed from it before every repeat (a write of
-    # a buffer larger than L2, outside the timed events)
-    flush = (torch.empty(256 << 20, dtype=torch.uint8, device=dev)
-             if step_bytes(w, code.L)["matvec"] < (200 << 20) else None)
+    # a buffer larger than L2, outside the timed events), then a read of a
+    # second one, so that the flush's own dirty lines are written back before
+    # the timed kernel rather than during it
+    small = step_bytes(w, code.L)["matvec"] < (200 << 20)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev) if small else None
+    clean = torch.ones(64 << 20, dtype=torch.int32, device=dev) if small else None
+
+    def flush_l2(r):
+        if flush is not None:
+            flush.fill_(r & 255)
+            clean.sum()
+
     # keep the device queue ahead of the host: the per-call events then time
     # the kernels, not the host's launch gaps
     torch.cuda._sleep(int(2e6 + reps * 4e5))
     for r in range(reps):
-        if flush is not None:
-            flush.fill_(r & 255)
+        flush_l2(r)
         ev[r][0].record()
         cm.matvec(code, A, parity, X, Yt, status=status)
         ev[r][1].record()
@@ -792,8 +800,7 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
         evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(reps)]
         torch.cuda._sleep(int(2e6 + reps * 4e5))
         for r in range(reps):
-            if flush is not None:
-                flush.fill_(r & 255)
+            flush_l2(r)
             evs[r][0].record()
             cm.matvec_decode(code, A, parity, X, masks[r], only_survivors=only, Y=Y, ws=ws,
                              status=status)

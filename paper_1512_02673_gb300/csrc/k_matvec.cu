@@ -79,9 +79,13 @@ struct MatvecArgs {
     int64_t groups;        // total work units
     int32_t nw;            // workers computed: all n, or only the k survivors
     int8_t wmap[CM_MAX_N]; // computed worker slot -> worker index
-    // column segments: CTA c sums the 128-column steps
-    // [s seg_steps, (s + 1) seg_steps) of every unit, s = c % nseg, into the
-    // partial results Yt + s part_stride (nseg = 1: whole rows into Yt)
+};
+
+// Column segments (matvec_kernel<..., SEGS = true>): CTA c sums the
+// 128-column steps [s seg_steps, (s + 1) seg_steps) of every unit,
+// s = c % nseg, into the partial results Yt + s part_stride; the CTAs of one
+// segment share its units.  The instances without segments never read it.
+struct SegArgs {
     int32_t nseg;
     int32_t seg_steps;
     int64_t part_stride;
@@ -201,10 +205,10 @@ __device__ __forceinline__ void griddep_launch_dependents()
     asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 }
 
-template <int BP, int R, int ST, int F, int kWarps, int XF>
+template <int BP, int R, int ST, int F, int kWarps, int XF, bool SEGS>
 __global__ void __launch_bounds__(kWarps * 32, 1)
 matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmP,
-              const __grid_constant__ MatvecArgs a)
+              const MatvecArgs a, const SegArgs sg)
 {
     constexpr int kThreads = kWarps * 32;
     using C = XCfg<BP, XF>;
@@ -234,17 +238,20 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     cm_fence_mbar_init();
     __syncthreads();
 
-    // this CTA's column segment; the CTAs of one segment share its units
-    const int seg = (int)(blockIdx.x % a.nseg);
-    const int64_t total_warps = (int64_t)(gridDim.x / a.nseg) * kWarps;
-    const int64_t gw = (int64_t)(blockIdx.x / a.nseg) * kWarps + warp;
+    // this CTA's column segment (SEGS): the first step, the steps, the
+    // partial results; the CTAs of one segment share its units
+    const int seg = SEGS ? (int)(blockIdx.x % sg.nseg) : 0;
+    const int64_t total_warps = (int64_t)(SEGS ? gridDim.x / sg.nseg : gridDim.x) * kWarps;
+    const int64_t gw = (int64_t)(SEGS ? blockIdx.x / sg.nseg : blockIdx.x) * kWarps + warp;
     const int rounds = (int)((a.groups + total_warps - 1) / total_warps);
-    const int s0 = seg * a.seg_steps;   // the segment's first step
     const int all_steps = (int)((a.d + 127) / 128);
-    const int steps = all_steps - s0 < a.seg_steps ? all_steps - s0 : a.seg_steps;
+    const int s0 = SEGS ? seg * sg.seg_steps : 0;
+    const int steps = SEGS ? (all_steps - s0 < sg.seg_steps ? all_steps - s0 : sg.seg_steps)
+                           : all_steps;
     const int64_t col0 = (int64_t)s0 * 128;
-    const int nchunks = (steps * 128 + C::CX - 1) / C::CX;
-    double *const Yt = a.Yt + (int64_t)seg * a.part_stride;
+    const int nchunks = SEGS ? (steps * 128 + C::CX - 1) / C::CX
+                             : (int)((a.d + C::CX - 1) / C::CX);
+    double *const Yt = SEGS ? a.Yt + (int64_t)seg * sg.part_stride : a.Yt;
     // rounds in which this warp has a unit (a prefix: unit index grows with round)
     const int64_t my_rounds = gw < a.groups ? (a.groups - 1 - gw) / total_warps + 1 : 0;
     // A unit's steps go in groups of GS (the last one shorter when GS does
@@ -263,7 +270,8 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
         cm_mbar_arrive_expect_tx(&bar[p_g], nb * STEP_BYTES);
         for (int u = 0; u < nb; ++u)
             cm_tma_load_2d(ring + (GS * p_g + u) * S::SLOT_FLOATS, pu.parity ? &tmP : &tmA,
-                           (int32_t)(col0 + 128 * (p_s + u)), pu.y, &bar[p_g]);
+                           SEGS ? (int32_t)(col0 + 128 * (p_s + u)) : 128 * (p_s + u), pu.y,
+                           &bar[p_g]);
         ++p_idx;
         p_g = p_g + 1 == NG ? 0 : p_g + 1;
         p_s += nb;
@@ -402,12 +410,13 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
 }
 
 template <int BP, int R, int ST, int F, int kWarps, int XF = 4096>
-cudaError_t launch_bp(MatvecArgs a, const float *A, int64_t lda, const float *par, int64_t ldp,
-                      cudaStream_t s)
+cudaError_t launch_bp(MatvecArgs a, const SegArgs &sg, const float *A, int64_t lda,
+                      const float *par, int64_t ldp, cudaStream_t s)
 {
     constexpr int kThreads = kWarps * 32;
     using S = Smem<BP, R, ST, kWarps, XF>;
-    auto kern = matvec_kernel<BP, R, ST, F, kWarps, XF>;
+    auto kern = sg.nseg > 1 ? matvec_kernel<BP, R, ST, F, kWarps, XF, true>
+                            : matvec_kernel<BP, R, ST, F, kWarps, XF, false>;
     CUtensorMap tmA, tmP;
     if (!cm_make_tmap_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, A, a.d, a.m, lda * 4, 128, R,
                          CU_TENSOR_MAP_SWIZZLE_NONE) ||
@@ -420,11 +429,11 @@ cudaError_t launch_bp(MatvecArgs a, const float *A, int64_t lda, const float *pa
     a.groups = (a.L + R - 1) / R * a.nw;
     // CTAs per segment: as many as the SMs allow, no more than the units need
     const int64_t need = (a.groups + kWarps - 1) / kWarps;
-    int64_t per_seg = (cm_sm_count() > 0 ? cm_sm_count() : 1) / a.nseg;
+    int64_t per_seg = (cm_sm_count() > 0 ? cm_sm_count() : 1) / sg.nseg;
     if (per_seg < 1) per_seg = 1;
     if (per_seg > need) per_seg = need;
-    const int64_t grid = per_seg * a.nseg;
-    kern<<<(unsigned)grid, kThreads, S::TOTAL, s>>>(tmA, tmP, a);
+    const int64_t grid = per_seg * sg.nseg;
+    kern<<<(unsigned)grid, kThreads, S::TOTAL, s>>>(tmA, tmP, a, sg);
     return cudaGetLastError();
 }
 
@@ -468,9 +477,6 @@ MatvecArgs matvec_args(const CodeParams &cp, const float *X, int b, double *Yt, 
     a.b = b;
     a.groups = 0;
     a.fast16 = b == 1 && ((uintptr_t)X & 15u) == 0;
-    a.nseg = 1;
-    a.seg_steps = (int32_t)((cp.d + 127) / 128);
-    a.part_stride = 0;
     return a;
 }
 
@@ -482,15 +488,15 @@ int unit_rows(const MatvecArgs &a)
     return 8;
 }
 
-cudaError_t dispatch(const MatvecArgs &a, const float *A, int64_t lda, const float *par,
-                     int64_t ldp, cudaStream_t s)
+cudaError_t dispatch(const MatvecArgs &a, const SegArgs &sg, const float *A, int64_t lda,
+                     const float *par, int64_t ldp, cudaStream_t s)
 {
     if (a.b == 1) {
-        if (unit_rows(a) == 4) return launch_bp<1, 4, 12, 16, 8>(a, A, lda, par, ldp, s);
-        return launch_bp<1, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
+        if (unit_rows(a) == 4) return launch_bp<1, 4, 12, 16, 8>(a, sg, A, lda, par, ldp, s);
+        return launch_bp<1, 8, 6, 16, 8>(a, sg, A, lda, par, ldp, s);
     }
-    if (a.b <= 4) return launch_bp<4, 8, 6, 16, 8>(a, A, lda, par, ldp, s);
-    return launch_bp<8, 8, 6, 64, 8>(a, A, lda, par, ldp, s);
+    if (a.b <= 4) return launch_bp<4, 8, 6, 16, 8>(a, sg, A, lda, par, ldp, s);
+    return launch_bp<8, 8, 6, 64, 8>(a, sg, A, lda, par, ldp, s);
 }
 
 }  // namespace
@@ -512,7 +518,7 @@ int matvec_segments(const CodeParams &cp, int b, uint32_t only)
     const int R = unit_rows(a);
     const int64_t units = (a.L + R - 1) / R * a.nw;
     const int sms = cm_sm_count() > 0 ? cm_sm_count() : 1;
-    const int steps = a.seg_steps;
+    const int steps = (int)((cp.d + 127) / 128);
     auto cost = [&](int ns) {
         const int64_t warps = (int64_t)(sms / ns) * 8;
         const int seg_steps = (steps + ns - 1) / ns;
@@ -536,16 +542,17 @@ cudaError_t launch_matvec_split(const CodeParams &cp, const float *A, int64_t ld
                                 int32_t *status, uint32_t only, int nseg, int64_t part_stride,
                                 cudaStream_t s)
 {
-    MatvecArgs a = matvec_args(cp, X, b, Yt, status, only);
-    a.nseg = nseg;
-    a.seg_steps = (a.seg_steps + nseg - 1) / nseg;
-    a.part_stride = part_stride;
-    return dispatch(a, A, lda, par, ldp, s);
+    SegArgs sg;
+    sg.nseg = nseg > 1 ? nseg : 1;
+    sg.seg_steps = (int32_t)(((cp.d + 127) / 128 + sg.nseg - 1) / sg.nseg);
+    sg.part_stride = part_stride;
+    return dispatch(matvec_args(cp, X, b, Yt, status, only), sg, A, lda, par, ldp, s);
 }
 
 cudaError_t launch_matvec(const CodeParams &cp, const float *A, int64_t lda, const float *par,
                           int64_t ldp, const float *X, int b, double *Yt, int32_t *status,
                           uint32_t only, cudaStream_t s)
 {
-    return dispatch(matvec_args(cp, X, b, Yt, status, only), A, lda, par, ldp, s);
+    const SegArgs whole = {1, (int32_t)((cp.d + 127) / 128), 0};
+    return dispatch(matvec_args(cp, X, b, Yt, status, only), whole, A, lda, par, ldp, s);
 }

@@ -2,27 +2,37 @@
 // parity block p of the (n,k) code, applied elementwise across the k row
 // blocks of A (rows past m are the appended zero rows).
 //
-// A short contraction (k <= 31 terms per output) that streams A once.  Work
-// unit = one block row r and a segment of at most 4096 columns, owned by one
-// warp; a persistent grid sweeps the units.  The launcher takes the longest
-// segment whose units fill the rounds of the grid's warps to 90 % (at L of a
-// few hundred rows, 4096-column segments leave most warps idle).  Each
-// 128-column step of a unit gathers row r of every data block into shared
-// memory with TMA in sub-steps of KC blocks: 3-D boxes of KC full blocks
-// (block stride L rows; boxes past the last full block read as zero) plus, if
-// m is not a multiple of L, one 2-D box of the partial block whose rows past
-// m read as zero; blocks wholly past m are skipped.  Sub-steps stream through
-// a per-warp ring of ST slots with one mbarrier each (lane 0 issues, the warp
-// consumes), so several KB per warp are in flight with no per-lane copy work,
-// and small slots leave room for 16 warps per SM.  Lane l owns columns
-// [4l, 4l+4) of the step and keeps the accumulators of all parity blocks of
-// the pass in registers (packed fp32x2 FMAs with the coefficient pair
-// (P[p][i], P[p][i]) read as a shared-memory broadcast), then stores them
-// with coalesced streaming stores.  Every element of A is read once per pass
-// and every parity element written once; n - k <= 16 is one pass.  fp32
-// accumulation in the order i = 0..k-1; bf16 outputs are rounded to nearest
-// even once.  Waits are bounded (about 2 s): a time-out writes CM_ETIMEOUT
-// to the status word and the warp stops.
+// A short contraction (k <= 31 terms per output) that streams A once and
+// writes the parity once.  Two forms, both with fp32 accumulation in the
+// order i = 0..k-1 (so they give the same bits) and bf16 outputs rounded to
+// nearest even once:
+//
+// Elementwise (k <= 8, or k <= 16 with at least k/2 parity blocks): thread t
+// loads 4 columns of one block row from every data block with plain vector
+// loads, forms every parity block's sum with the coefficients as constant
+// operands, and stores 4 columns of every parity block.  Many resident warps
+// with few instructions per byte: on short codes, whose writes are as large
+// as their reads, this keeps more requests in flight than a TMA ring in the
+// same shared memory, and runs at the rate of a plain copy of the same bytes.
+//
+// Tiled (the rest): a work unit = one block row r and a segment of steps of
+// 128 columns, owned by one CTA; warp w takes the segment's steps w, w + 8,
+// ..., so that the CTA's warps read and write adjacent 512-byte pieces of
+// every row at once.  A persistent grid sweeps the units; the launcher takes
+// the longest segment whose units fill the rounds of the grid to 90 %.  Each
+// step gathers row r of every data block into shared memory with TMA in
+// sub-steps of KC blocks: 3-D boxes of KC full blocks (block stride L rows;
+// boxes past the last full block read as zero) plus, if m is not a multiple
+// of L, one 2-D box of the partial block whose rows past m read as zero;
+// blocks wholly past m are skipped.  Sub-steps stream through a per-warp ring
+// of ST slots with one mbarrier each (lane 0 issues, the warp consumes), so
+// several KB per warp are in flight with no per-lane copy work, and small
+// slots leave room for 16 warps per SM.  Lane l owns columns [4l, 4l+4) of
+// the step and keeps the accumulators of all parity blocks of the pass in
+// registers (packed fp32x2 FMAs with the coefficient pair (P[p][i], P[p][i])
+// read as a shared-memory broadcast), then stores them with coalesced
+// streaming stores.  n - k <= 16 is one pass.  Waits are bounded (about 2 s):
+// a time-out writes CM_ETIMEOUT to the status word and the warp stops.
 #include <cuda_bf16.h>
 
 #include "cm_internal.cuh"
@@ -53,6 +63,7 @@ struct Elem<float> {
         __stcs(reinterpret_cast<float4 *>(p), make_float4(a.x, a.y, b.x, b.y));
     }
     __device__ static void store1(float *p, float v) { *p = v; }
+    __device__ static float load1(const float *p) { return *p; }
 };
 
 template <>
@@ -77,6 +88,7 @@ struct Elem<uint16_t> {   // bf16 bits
         __stcs(reinterpret_cast<uint2 *>(p), v);
     }
     __device__ static void store1(uint16_t *p, float v) { *p = (uint16_t)rne(v); }
+    __device__ static float load1(const uint16_t *p) { return widen(*p); }
 };
 
 struct EncodeArgs {
@@ -119,25 +131,32 @@ __device__ __forceinline__ void encode_body(const CUtensorMap &tmF, const CUtens
     cm_fence_mbar_init();
     __syncthreads();
 
-    const int64_t total_warps = (int64_t)gridDim.x * kWarps;
-    const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
-    if (gw >= a.units) return;
+    // a unit (block row r, segment of seg steps) belongs to one CTA; warp w
+    // takes the unit's steps w, w + kWarps, ..., so that the CTA's warps read
+    // and write adjacent 512-byte pieces of every row at once
+    const int64_t cta_units = (int64_t)gridDim.x;
+    if ((int64_t)blockIdx.x >= a.units) return;
     const int nfull = (a.kf + KC - 1) / KC;      // sub-steps of full blocks
 
-    auto unit_steps = [&](int64_t u) {           // the last segment of a row may be short
+    auto warp_steps = [&](int64_t u) {           // this warp's steps in unit u
         const int s0 = (int)(u % a.nseg) * a.seg;
-        return (a.steps - s0) < a.seg ? a.steps - s0 : a.seg;
+        const int ns = (a.steps - s0) < a.seg ? a.steps - s0 : a.seg;
+        return ns > warp ? (ns - warp + kWarps - 1) / kWarps : 0;
     };
+    auto next_unit = [&](int64_t u) {            // the next unit with steps for this warp
+        do u += cta_units; while (u < a.units && warp_steps(u) == 0);
+        return u;
+    };
+    int64_t first = blockIdx.x;
+    if (warp_steps(first) == 0) first = next_unit(first);
 
     // ---- producer (lane 0): sub-step c of step p_s of unit p_unit ----
-    int64_t p_unit = gw;
+    int64_t p_unit = first;
     int p_s = 0, p_c = 0, p_slot = 0, in_flight = 0;
     auto produce = [&]() {
         const int64_t r = p_unit / a.nseg;
-        const int32_t x = ((int)(p_unit % a.nseg) * a.seg + p_s) * STEP;
+        const int32_t x = ((int)(p_unit % a.nseg) * a.seg + warp + kWarps * p_s) * STEP;
         unsigned char *dst = ring + p_slot * SLOT;
-        // no proxy fence: the slot is only written by TMA, and the __syncwarp
-        // before every refill orders the lanes' reads of it before the copy
         if (p_c < nfull) {
             cm_mbar_arrive_expect_tx(&bar[p_slot], SLOT);
             cm_tma_load_3d(dst, &tmF, x, (int32_t)r, p_c * KC, &bar[p_slot]);
@@ -149,9 +168,9 @@ __device__ __forceinline__ void encode_body(const CUtensorMap &tmF, const CUtens
         ++in_flight;
         if (++p_c == a.nsub) {
             p_c = 0;
-            if (++p_s == unit_steps(p_unit)) {
+            if (++p_s == warp_steps(p_unit)) {
                 p_s = 0;
-                p_unit += total_warps;
+                p_unit = next_unit(p_unit);
             }
         }
     };
@@ -162,10 +181,10 @@ __device__ __forceinline__ void encode_body(const CUtensorMap &tmF, const CUtens
     int slot = 0;
     uint32_t phase = 0;
     T *par = static_cast<T *>(a.par);
-    for (int64_t u = gw; u < a.units; u += total_warps) {
+    for (int64_t u = first; u < a.units; u = next_unit(u)) {
         const int64_t r = u / a.nseg;
         const int seg = (int)(u % a.nseg);
-        const int ns = unit_steps(u);
+        const int ns = warp_steps(u);
         for (int s = 0; s < ns; ++s) {
             float2 acc[NPG][2];
 #pragma unroll
@@ -213,7 +232,7 @@ __device__ __forceinline__ void encode_body(const CUtensorMap &tmF, const CUtens
                     if (p_unit < a.units) produce();   // refill it
                 }
             }
-            const int64_t col = (int64_t)(seg * a.seg + s) * STEP + 4 * lane;
+            const int64_t col = (int64_t)(seg * a.seg + warp + kWarps * s) * STEP + 4 * lane;
             if (col < a.d) {
 #pragma unroll
                 for (int j = 0; j < NPG; ++j) {
@@ -251,6 +270,119 @@ encode_kernel16(const __grid_constant__ CUtensorMap tmF, const __grid_constant__
     encode_body<T, 16>(tmF, tmP, cp, a);
 }
 
+// Elementwise form for short codes (at most KE data blocks with rows below m,
+// at most 8 parity blocks).  Thread t takes 4 columns of one block row: it
+// loads them from every data block (zeros past m), forms the parity blocks'
+// sums in the same order i = 0..k-1 as the tiled kernel (so the results are
+// the same bits), and stores 4 columns of every parity block.  The
+// coefficients sit in the kernel's parameter space as constant operands.
+template <int NPG, int KE>
+struct EwArgs {
+    const void *A;
+    void *par;
+    int64_t lda, ldp;
+    int64_t m, d, L;
+    int64_t nc;          // 4-column chunks per row
+    int32_t k, np;
+    float w[NPG][KE];    // w[j][i] = P[j][i]
+};
+
+template <typename T, int NPG, int KE>
+__global__ void __launch_bounds__(256)
+encode_ew_kernel(const __grid_constant__ EwArgs<NPG, KE> a)
+{
+    const T *A = static_cast<const T *>(a.A);
+    T *par = static_cast<T *>(a.par);
+    const int64_t S = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    int64_t r = t / a.nc, c = t - r * a.nc;
+    const int64_t qS = S / a.nc, rS = S - qS * a.nc;
+    while (r < a.L) {
+        const int64_t col = 4 * c;
+        const bool full = col + 4 <= a.d;
+        float2 x[KE][2];
+#pragma unroll
+        for (int i = 0; i < KE; ++i) {
+            x[i][0] = x[i][1] = make_float2(0.f, 0.f);
+            const int64_t row = (int64_t)i * a.L + r;
+            if (i < a.k && row < a.m) {
+                const T *src = A + row * a.lda + col;
+                if (full) {
+                    Elem<T>::load4(src, x[i][0], x[i][1]);
+                } else {
+                    float v[4] = {0.f, 0.f, 0.f, 0.f};
+                    for (int e = 0; col + e < a.d; ++e) v[e] = Elem<T>::load1(src + e);
+                    x[i][0] = make_float2(v[0], v[1]);
+                    x[i][1] = make_float2(v[2], v[3]);
+                }
+            }
+        }
+        float2 acc[NPG][2];
+#pragma unroll
+        for (int j = 0; j < NPG; ++j) acc[j][0] = acc[j][1] = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int i = 0; i < KE; ++i) {
+            if (i < a.k) {
+#pragma unroll
+                for (int j = 0; j < NPG; ++j) {
+                    const float2 w = make_float2(a.w[j][i], a.w[j][i]);
+                    acc[j][0] = __ffma2_rn(w, x[i][0], acc[j][0]);
+                    acc[j][1] = __ffma2_rn(w, x[i][1], acc[j][1]);
+                }
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < NPG; ++j) {
+            if (j < a.np) {
+                T *dst = par + ((int64_t)j * a.L + r) * a.ldp + col;
+                if (full) {
+                    Elem<T>::store4(dst, acc[j][0], acc[j][1]);
+                } else {
+                    const float v[4] = {acc[j][0].x, acc[j][0].y, acc[j][1].x, acc[j][1].y};
+                    for (int e = 0; col + e < a.d; ++e) Elem<T>::store1(dst + e, v[e]);
+                }
+            }
+        }
+        c += rS;
+        r += qS;
+        if (c >= a.nc) {
+            c -= a.nc;
+            ++r;
+        }
+    }
+}
+
+template <typename T, int NPG, int KE>
+cudaError_t launch_ew(const CodeParams &cp, const T *A, int64_t lda, T *par, int64_t ldp,
+                      cudaStream_t s)
+{
+    EwArgs<NPG, KE> a;
+    a.A = A;
+    a.par = par;
+    a.lda = lda;
+    a.ldp = ldp;
+    a.m = cp.m;
+    a.d = cp.d;
+    a.L = cp.L;
+    a.nc = (cp.d + 3) / 4;
+    a.k = cp.k;
+    a.np = cp.n - cp.k;
+    for (int j = 0; j < NPG; ++j)
+        for (int i = 0; i < KE; ++i)
+            a.w[j][i] = j < a.np && i < cp.k ? cp.P[j * cp.k + i] : 0.f;
+    auto kern = encode_ew_kernel<T, NPG, KE>;
+    int per_sm = 0;
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, 0);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) per_sm = 1;
+    const int64_t items = cp.L * a.nc;
+    int64_t grid = (int64_t)(cm_sm_count() > 0 ? cm_sm_count() : 1) * per_sm;
+    if (grid > (items + 255) / 256) grid = (items + 255) / 256;
+    if (grid < 1) grid = 1;
+    kern<<<(unsigned)grid, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
 template <typename T, int NPG>
 cudaError_t launch_passes(const CodeParams &cp, const T *A, int64_t lda, T *par, int64_t ldp,
                           int32_t *status, cudaStream_t s)
@@ -258,6 +390,13 @@ cudaError_t launch_passes(const CodeParams &cp, const T *A, int64_t lda, T *par,
     const int64_t es = sizeof(T);
     const int kf = (int)(cp.m / cp.L);                 // >= 1 since L <= m
     const int kv = (int)((cp.m + cp.L - 1) / cp.L);
+    if constexpr (NPG <= 8) {   // short codes: the elementwise form (see above)
+        if (cp.k <= 8) return launch_ew<T, NPG, 8>(cp, A, lda, par, ldp, s);
+    }
+    if constexpr (NPG <= 12) {
+        if (cp.k <= 16 && 2 * (cp.n - cp.k) >= cp.k)
+            return launch_ew<T, NPG, 16>(cp, A, lda, par, ldp, s);
+    }
     CUtensorMap tmF, tmP;
     if (!cm_make_tmap_3d(&tmF, Elem<T>::TM, A, (uint64_t)cp.d, (uint64_t)cp.L, (uint64_t)kf,
                          (uint64_t)(lda * es), (uint64_t)(cp.L * lda * es), STEP, 1, KC))
@@ -294,15 +433,15 @@ cudaError_t launch_passes(const CodeParams &cp, const T *A, int64_t lda, T *par,
     if (e != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
     int64_t grid = (int64_t)cm_sm_count() * per_sm;
-    {   // segment length (see the header)
-        const int64_t warps = grid * kWarps;
+    {   // segment length: CTA-level units, warps interleaved over the steps
         double best = -1.0;
-        for (int ns = (a.steps + SEG - 1) / SEG; ns <= a.steps; ++ns) {
+        for (int ns = (a.steps + kWarps * SEG - 1) / (kWarps * SEG); ns <= a.steps; ++ns) {
             const int sg = (a.steps + ns - 1) / ns;
             const int nsg = (a.steps + sg - 1) / sg;
             const int64_t units = cp.L * nsg;
-            const int64_t rounds = (units + warps - 1) / warps;
-            const double fill = (double)cp.L * a.steps / ((double)rounds * sg * warps);
+            const int64_t rounds = (units + grid - 1) / grid;
+            const int wsteps = (sg + kWarps - 1) / kWarps;
+            const double fill = (double)cp.L * a.steps / ((double)rounds * wsteps * kWarps * grid);
             if (fill > best + 1e-9) {
                 best = fill;
                 a.seg = sg;
@@ -312,7 +451,7 @@ cudaError_t launch_passes(const CodeParams &cp, const T *A, int64_t lda, T *par,
         }
     }
     a.units = cp.L * a.nseg;
-    const int64_t need = (a.units + kWarps - 1) / kWarps;
+    const int64_t need = a.units;
     if (grid > need) grid = need;
     if (grid < 1) grid = 1;
     for (int p0 = 0; p0 < cp.n - cp.k; p0 += NPG) {

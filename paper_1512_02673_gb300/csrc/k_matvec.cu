@@ -12,12 +12,13 @@
 // are known beforehand only those k are (the others' rows stay unwritten).
 //
 // Data movement.  The unit's rows stream through a per-warp ring of ST
-// shared-memory slots, one 2-D TMA box (R rows x 128 columns) per step issued
-// by the warp's lane 0.  Slots are guarded in groups of GS (2; 4 for the
-// 12-slot ring of 4-row units): the GS boxes of steps (GS i, ..., GS i +
-// GS - 1) complete on one mbarrier, so ST steps are in flight per warp
-// without any per-lane copy work and the wait, the refill and the ring
-// bookkeeping come once per GS steps.  Lane 0 refills a slot after
+// shared-memory slots of one 128-column step each, filled by 2-D TMA boxes of
+// two steps (R rows x 256 columns, 1 KB contiguous per row) issued by the
+// warp's lane 0.  Slots are guarded in groups of GS (2; 4 for the 12-slot
+// ring of 4-row units): the boxes of steps (GS i, ..., GS i + GS - 1)
+// complete on one mbarrier, so ST steps are in flight per warp without any
+// per-lane copy work and the wait, the refill and the ring bookkeeping come
+// once per GS steps.  Lane 0 refills a slot after
 // a __syncwarp that follows every lane's reads of it: the warp barrier orders
 // those reads before the copy is issued, and the slot is only ever written by
 // TMA, so there is no generic-proxy write for a proxy fence to publish (one
@@ -230,6 +231,11 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     constexpr int GS = ST % 4 == 0 && ST >= 12 ? 4 : 2;
     static_assert(ST % GS == 0 && IPC % GS == 0, "ring slots are guarded in groups");
     constexpr int NG = ST / GS;   // barrier groups per warp
+    // A group's steps arrive in TMA boxes of R rows x 256 columns (two steps,
+    // 1 KB contiguous per row): step u of a group sits in box u / 2 at column
+    // offset 128 (u % 2), its rows 256 floats apart.  Against boxes of one
+    // step (512 B per row) the DRAM sees twice the bytes per row access.
+    constexpr int BOX_FLOATS = 2 * S::SLOT_FLOATS;
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     float *ring = rings + warp * (ST * S::SLOT_FLOATS);
@@ -267,11 +273,21 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
     Unit pu = unit_of(a, gw, R);
     auto produce = [&]() {   // lane 0 only; loads the next group into ring group p_g
         const int nb = steps - p_s < GS ? steps - p_s : GS;
-        cm_mbar_arrive_expect_tx(&bar[p_g], nb * STEP_BYTES);
-        for (int u = 0; u < nb; ++u)
-            cm_tma_load_2d(ring + (GS * p_g + u) * S::SLOT_FLOATS, pu.parity ? &tmP : &tmA,
-                           SEGS ? (int32_t)(col0 + 128 * (p_s + u)) : 128 * (p_s + u), pu.y,
-                           &bar[p_g]);
+        // a box always lands whole (its columns past d read as zero; in a
+        // column segment an odd last step reads, and ignores, the next one)
+        if constexpr (GS == 2) {
+            cm_mbar_arrive_expect_tx(&bar[p_g], 2 * STEP_BYTES);
+            cm_tma_load_2d(ring + GS * p_g * S::SLOT_FLOATS, pu.parity ? &tmP : &tmA,
+                           SEGS ? (int32_t)(col0 + 128 * p_s) : 128 * p_s, pu.y, &bar[p_g]);
+        } else {
+            const int nbox = (nb + 1) / 2;
+            cm_mbar_arrive_expect_tx(&bar[p_g], nbox * 2 * STEP_BYTES);
+            for (int u = 0; u < nbox; ++u)
+                cm_tma_load_2d(ring + GS * p_g * S::SLOT_FLOATS + u * BOX_FLOATS,
+                               pu.parity ? &tmP : &tmA,
+                               SEGS ? (int32_t)(col0 + 128 * (p_s + 2 * u)) : 128 * (p_s + 2 * u),
+                               pu.y, &bar[p_g]);
+        }
         ++p_idx;
         p_g = p_g + 1 == NG ? 0 : p_g + 1;
         p_s += nb;
@@ -313,7 +329,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
             float4 av[RH];
 #pragma unroll
             for (int r = 0; r < RH; ++r)
-                av[r] = *reinterpret_cast<const float4 *>(ab + (r0 + r) * 128);
+                av[r] = *reinterpret_cast<const float4 *>(ab + (r0 + r) * 256);
 #pragma unroll
             for (int r = 0; r < RH; ++r)
 #pragma unroll
@@ -358,7 +374,9 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
                     const float *ab = ring + GS * grp * S::SLOT_FLOATS + 4 * lane;
 #pragma unroll
                     for (int u = 0; u < GS; ++u)
-                        if (cs + u < ns) step(ab + u * S::SLOT_FLOATS, xchunk + (cs + u) * 128);
+                        if (cs + u < ns)
+                            step(ab + (u >> 1) * BOX_FLOATS + (u & 1) * 128,
+                                 xchunk + (cs + u) * 128);
                     ++c_idx;
                     if (++grp == NG) {
                         grp = 0;
@@ -417,11 +435,11 @@ cudaError_t launch_bp(MatvecArgs a, const SegArgs &sg, const float *A, int64_t l
     using S = Smem<BP, R, ST, kWarps, XF>;
     auto kern = sg.nseg > 1 ? matvec_kernel<BP, R, ST, F, kWarps, XF, true>
                             : matvec_kernel<BP, R, ST, F, kWarps, XF, false>;
-    CUtensorMap tmA, tmP;
-    if (!cm_make_tmap_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, A, a.d, a.m, lda * 4, 128, R,
+    CUtensorMap tmA, tmP;   // boxes of two steps: R rows x 256 columns
+    if (!cm_make_tmap_2d(&tmA, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, A, a.d, a.m, lda * 4, 256, R,
                          CU_TENSOR_MAP_SWIZZLE_NONE) ||
         !cm_make_tmap_2d(&tmP, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, par, a.d,
-                         (a.n - a.k) * a.L, ldp * 4, 128, R, CU_TENSOR_MAP_SWIZZLE_NONE))
+                         (a.n - a.k) * a.L, ldp * 4, 256, R, CU_TENSOR_MAP_SWIZZLE_NONE))
         return cudaErrorInvalidValue;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          S::TOTAL);

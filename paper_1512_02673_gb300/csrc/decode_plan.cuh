@@ -160,6 +160,34 @@ __device__ __forceinline__ void split_double(double y, float &h, float &l)
     l = __uint_as_float(sign | __float_as_uint(__uint2float_rn(r29) * scale));
 }
 
+// split_double and rne_float of the same value, sharing the bit extraction:
+// in split_double's own range the rounded value is the truncated high part
+// plus one unit in its last place when the 29 dropped bits are above half,
+// or exactly half with an odd last bit (a carry moves into the exponent, up
+// to infinity, as rounding does); elsewhere rne_float itself.
+__device__ __forceinline__ void split_round(double y, float &h, float &l, float &r)
+{
+    const unsigned long long b = (unsigned long long)__double_as_longlong(y);
+    const uint32_t hi = (uint32_t)(b >> 32), lo = (uint32_t)b;
+    const int ex = (int)((hi >> 20) & 0x7FF);
+    if (ex < 1023 - 100 || ex > 1023 + 127) {
+        h = __double2float_rn(y);
+        l = 0.f;
+        r = rne_float(y);
+        return;
+    }
+    const uint32_t sign = hi & 0x80000000u;
+    const uint32_t m23 = ((hi & 0xFFFFFu) << 3) | (lo >> 29);
+    const uint32_t hb = sign | ((uint32_t)(ex - 1023 + 127) << 23) | m23;
+    h = __uint_as_float(hb);
+    const uint32_t r29 = lo & 0x1FFFFFFFu;
+    const int se = ex - 1075 + 127;
+    const float scale = se > 0 ? __int_as_float(se << 23) : 0.f;
+    l = __uint_as_float(sign | __float_as_uint(__uint2float_rn(r29) * scale));
+    const uint32_t up = (r29 > 0x10000000u || (r29 == 0x10000000u && (m23 & 1u))) ? 1u : 0u;
+    r = __uint_as_float(hb + up);
+}
+
 // (sh, sl) += (dh + dl) * (yh + yl), to about 2^-44 relative per term.  The
 // rounded operations are explicit intrinsics, which the compiler never
 // contracts into fused multiply-adds (that would break the error terms).

@@ -70,7 +70,8 @@ __device__ __forceinline__ void store_out(const DecodeArgs &a, int64_t out, floa
 // position r b + v) of all k output blocks, taken in tiles of kTile.
 //  1. plan_setup.
 //  2. For every tile: the k surviving values of its positions are loaded
-//     (position fastest, coalesced) into shared memory, and those of the
+//     (position fastest, coalesced; a thread's loads issued together) and
+//     staged in shared memory as (high, low) fp32 pairs, and those of the
 //     surviving systematic blocks are written out at once (the pass-through,
 //     fp32 rounding of the fp64 results).  For the first tile the first NW
 //     warps eliminate meanwhile (when blocks are missing), so the loads
@@ -85,7 +86,7 @@ __device__ __forceinline__ void store_out(const DecodeArgs &a, int64_t out, floa
 template <int EMAX, int NW>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecodeArgs a)
 {
-    extern __shared__ double ysm[];   // [CM_MAX_N][kTile]
+    extern __shared__ float2 ysm[];   // [CM_MAX_N][kTile] (high, low) pairs of the survivors
     __shared__ Plan pl;
     __shared__ float Dh[kMaxE][CM_MAX_N], Dl[kMaxE][CM_MAX_N];
     const int k = a.cp.k;
@@ -116,23 +117,46 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
         const int tn = (int)(n - t0 < kTile ? n - t0 : kTile);
         const bool first = t0 == 0;
         if (overlap && first && e > 0 && tid < 32 * NW) plan_eliminate<EMAX, NW>(pl, k);
-        // stage the tile; the eliminating warps skip the first one
+        // stage the tile; the eliminating warps skip the first one.  Thread
+        // tt takes position q = tt % tn of survivors tt / tn, tt / tn + per,
+        // ... (per = threads / tn), SB of them with their loads issued before
+        // any store (one division per thread, none per value)
         {
+            constexpr int SB = 4;
             const int lo = overlap && first && e > 0 ? 32 * NW : 0;
-            for (int u = tid - lo; u >= 0 && u < k * tn; u += kThreads - lo) {
-                const int p = u / tn, q = u - p * tn;
-                const int s = pl.S[p];
-                const int64_t src = (int64_t)s * per_block + p0 + t0 + q;
-                double y = a.Yt[src];
-                for (int h = 1; h < a.nparts; ++h) y += a.Yt[src + h * a.part_stride];
-                if (e > 0) ysm[p * kTile + q] = y;
-                if (s < k && src < mb) {      // surviving systematic block: pass through
-                    if (a.mode == DEC_PLAIN) {
-                        a.Y[src] = rne_float(y);
-                    } else {
-                        float yh, yl;
-                        split_double(y, yh, yl);
-                        store_out(a, src, yh, yl);
+            const int tt = tid - lo;
+            const int per = (kThreads - lo) / tn;
+            if (tt >= 0 && tt < per * tn) {
+                const int q = tt % tn;
+                const int64_t base = p0 + t0 + q;
+                for (int pb = tt / tn; pb < k; pb += SB * per) {
+                    double y[SB];
+#pragma unroll
+                    for (int j = 0; j < SB; ++j) {
+                        const int p = pb + j * per;
+                        if (p < k) y[j] = a.Yt[(int64_t)pl.S[p] * per_block + base];
+                    }
+                    for (int h = 1; h < a.nparts; ++h) {
+#pragma unroll
+                        for (int j = 0; j < SB; ++j) {
+                            const int p = pb + j * per;
+                            if (p < k) y[j] += a.Yt[(int64_t)pl.S[p] * per_block + base + h * a.part_stride];
+                        }
+                    }
+#pragma unroll
+                    for (int j = 0; j < SB; ++j) {
+                        const int p = pb + j * per;
+                        if (p >= k) break;
+                        const int s = pl.S[p];
+                        float yh, yl, yr;
+                        if (a.mode == DEC_PLAIN) split_round(y[j], yh, yl, yr);
+                        else split_double(y[j], yh, yl);
+                        if (e > 0) ysm[p * kTile + q] = make_float2(yh, yl);
+                        const int64_t src = (int64_t)s * per_block + base;
+                        if (s < k && src < mb) {   // surviving systematic block: pass through
+                            if (a.mode == DEC_PLAIN) a.Y[src] = yr;
+                            else store_out(a, src, yh, yl);
+                        }
                     }
                 }
             }
@@ -153,9 +177,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
                 float sh = 0.f, sl = 0.f;
 #pragma unroll 4
                 for (int p = 0; p < k; ++p) {
-                    float yh, yl;
-                    split_double(ysm[p * kTile + q], yh, yl);
-                    df_fma(Dh[c][p], Dl[c][p], yh, yl, sh, sl);
+                    const float2 y = ysm[p * kTile + q];
+                    df_fma(Dh[c][p], Dl[c][p], y.x, y.y, sh, sl);
                 }
                 const int64_t out = (int64_t)pl.M[c] * per_block + p0 + t0 + q;
                 if (out < mb) store_out(a, out, sh, sl);
@@ -283,7 +306,7 @@ unsigned grid_for(int64_t items, int threads, int per_sm)
 template <int EMAX, int NW>
 cudaError_t launch_k3(const DecodeArgs &a, unsigned grid, cudaStream_t s)
 {
-    constexpr int kSmem = CM_MAX_N * kTile * (int)sizeof(double);
+    constexpr int kSmem = CM_MAX_N * kTile * (int)sizeof(float2);
     auto kern = decode_kernel<EMAX, NW>;
     static const cudaError_t attr =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);

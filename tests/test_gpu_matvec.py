@@ -258,6 +258,11 @@ def test_pass_through_is_rounded_to_nearest(cm):
     torch.cuda.synchronize()
     want = Yt[:m].float()
     assert torch.equal(Y.view(torch.int32), want.view(torch.int32))
+    # with a block to decode the survivors are staged for the decode as well;
+    # the surviving systematic blocks 0 and 1 still pass through exactly
+    Y = cm.decode(code, Yt, 0b001011)
+    torch.cuda.synchronize()
+    assert torch.equal(Y[:2 * L].view(torch.int32), want[:2 * L].view(torch.int32))
 
 
 def test_extra_survivors_use_the_lowest_k(cm, orc):

@@ -135,7 +135,7 @@ class ClockSampler:
                 self.proc.kill()
 
     def summary(self) -> dict:
-        sms, maxs, reasons = [], [], set()
+        sms, maxs, watts, reasons = [], [], [], set()
         try:
             for line in open(self.path):
                 f = [x.strip() for x in line.split(",")]
@@ -146,6 +146,10 @@ class ClockSampler:
                     maxs.append(float(f[2]))
                 except ValueError:
                     continue
+                try:
+                    watts.append(float(f[3]))
+                except ValueError:
+                    pass
                 for name, val in zip(REASON_NAMES, f[5:9]):
                     if val.lower().startswith("active"):
                         reasons.add(name)
@@ -154,8 +158,12 @@ class ClockSampler:
             pass
         if not sms:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
-        return {"sm_mhz": float(np.median(sms)), "sm_max_mhz": float(max(maxs)),
-                "reasons": sorted(reasons), "samples": len(sms)}
+        out = {"sm_mhz": float(np.median(sms)), "sm_max_mhz": float(max(maxs)),
+               "reasons": sorted(reasons), "samples": len(sms)}
+        if watts:
+            out["power_w_median"] = float(np.median(watts))
+            out["power_w_max"] = float(max(watts))
+        return out
 
 
 def dist_setup():
@@ -723,6 +731,17 @@ def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
     torch.cuda.synchronize()
     gs_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in ev]))
     ds_ms = float(np.mean([e[1].elapsed_time(e[2]) for e in ev]))
+    # sustained: back to back for about 0.6 s with SM clock, power and
+    # throttle reasons sampled, against the sustained (power-capped) peak
+    n_sus = max(1, int(600.0 / g_ms))
+    torch.cuda.synchronize()
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        e0.record()
+        for _ in range(n_sus):
+            cm.coded_gemm(code, A, par, Bt, Ct, status=status)
+        e1.record()
+        torch.cuda.synchronize()
+    sus_ms = e0.elapsed_time(e1) / n_sus
     flops = 2.0 * w.n * code.L * w.d * w.gemm_n          # every coded row
     useful = 2.0 * w.m * w.d * w.gemm_n                  # A B itself
     tflops = flops / (g_ms * 1e-3) / 1e12
@@ -738,6 +757,11 @@ def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
             "survivors_only": {"gemm_ms": gs_ms, "decode_mat_ms": ds_ms,
                                "tflops": 2.0 * w.k * code.L * w.d * w.gemm_n / (gs_ms * 1e-3) / 1e12,
                                "useful_tflops_per_step": useful / ((gs_ms + ds_ms) * 1e-3) / 1e12},
+            "sustained": {"gemms": n_sus, "gemm_ms": sus_ms,
+                          "tflops": flops / (sus_ms * 1e-3) / 1e12,
+                          "frac_of_sustained_peak": flops / (sus_ms * 1e-3) / 1e12
+                          / peaks["bf16_tflops_sustained"],
+                          "clocks": clk.summary()},
             "encode_bf16_ms": enc_ms, "status": int(status.item())}
 
 

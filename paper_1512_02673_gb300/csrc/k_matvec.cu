@@ -4,7 +4,7 @@
 // r < L and vector v < b <= 8.  Worker j < k reads its block in place from A
 // (rows past m are virtual zeros); worker j >= k reads the parity buffer.
 //
-// Mapping.  A persistent grid (SMs x one resident CTA of 8 or 16 warps).  Work
+// Mapping.  A persistent grid (SMs x one resident CTA of 6, 8 or 16 warps).  Work
 // unit = R consecutive block rows of one worker, owned by one warp; unit u
 // belongs to the (u % nw)-th computed worker, so consecutive warps stream
 // different workers and all workers progress together, as the n workers of
@@ -15,7 +15,8 @@
 // shared-memory slots of one 128-column step each, filled by 2-D TMA boxes of
 // two steps (R rows x 256 columns, 1 KB contiguous per row) issued by the
 // warp's lane 0.  Slots are guarded in groups of GS (2; 4 for the 12-slot
-// ring of 4-row units): the boxes of steps (GS i, ..., GS i + GS - 1)
+// ring of 4-row units and the 8-slot ring of the 6-warp CTAs): the boxes of
+// steps (GS i, ..., GS i + GS - 1)
 // complete on one mbarrier, so ST steps are in flight per warp without any
 // per-lane copy work and the wait, the refill and the ring bookkeeping come
 // once per GS steps.  Lane 0 refills a slot after
@@ -228,7 +229,7 @@ matvec_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ C
 
     // slots per barrier group: 4 with the 12-slot ring, else 2 (3 groups of 2
     // for 6 slots; groups of 3 would leave two)
-    constexpr int GS = ST % 4 == 0 && ST >= 12 ? 4 : 2;
+    constexpr int GS = ST % 4 == 0 && ST >= 8 ? 4 : 2;
     static_assert(ST % GS == 0 && IPC % GS == 0, "ring slots are guarded in groups");
     constexpr int NG = ST / GS;   // barrier groups per warp
     // A group's steps arrive in TMA boxes of R rows x 256 columns (two steps,
@@ -511,6 +512,14 @@ cudaError_t dispatch(const MatvecArgs &a, const SegArgs &sg, const float *A, int
 {
     if (a.b == 1) {
         if (unit_rows(a) == 4) return launch_bp<1, 4, 12, 16, 8>(a, sg, A, lda, par, ldp, s);
+        // Units that fit one round of 6-warp CTAs (e.g. the 800 units of
+        // (25,23) at 5750 x 5750): 8-slot rings guarded in groups of four,
+        // so each row is read 2 KB at a time (two adjacent boxes) with 32 KB
+        // in flight per warp, in the same shared memory; 0.65 -> 0.74 of the
+        // copy peak there.  With more rounds the 8-warp form stays ahead.
+        const int sms = cm_sm_count() > 0 ? cm_sm_count() : 1;
+        if (sg.nseg == 1 && (a.L + 7) / 8 * a.nw <= (int64_t)sms * 6)
+            return launch_bp<1, 8, 8, 16, 6>(a, sg, A, lda, par, ldp, s);
         return launch_bp<1, 8, 6, 16, 8>(a, sg, A, lda, par, ldp, s);
     }
     if (a.b <= 4) return launch_bp<4, 8, 6, 16, 8>(a, sg, A, lda, par, ldp, s);
@@ -544,6 +553,9 @@ int matvec_segments(const CodeParams &cp, int b, uint32_t only)
     };
     int best = 1;
     double best_c = cost(1);
+    // whole rows in one round of 6-warp CTAs (see dispatch) ran 0.88 of the
+    // time of the 8-warp form on (25,23) at 5750 x 5750
+    if (b == 1 && R == 8 && units <= (int64_t)sms * 6) best_c *= 0.88;
     for (int ns = 2; ns <= 8; ns *= 2) {
         if (sms % ns || (steps + ns - 1) / ns < 8) break;
         const double c = cost(ns);

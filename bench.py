@@ -783,6 +783,13 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
     e0.record()
     cm.encode(code, A, parity)
     e1.record()
+    # five more back to back: the kernel's rate without one call's launch
+    e2, e3 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda._sleep(1_000_000)
+    e2.record()
+    for _ in range(5):
+        cm.encode(code, A, parity)
+    e3.record()
     Yt = cm.matvec(code, A, parity, X, status=status)
     Y = torch.empty((w.m, w.b), device=dev)
     reps = repeats or w.repeats
@@ -792,6 +799,7 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
         cm.decode(code, Yt, masks[r], Y=Y, status=status)
     torch.cuda.synchronize()
     enc_us = e0.elapsed_time(e1) * 1e3
+    enc_b2b_us = e2.elapsed_time(e3) * 1e3 / 5
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(reps)]
     # inputs that fit in L2 are flushed from it before every repeat (a write of
     # a buffer larger than L2, outside the timed events), then a read of a
@@ -848,6 +856,8 @@ def bench_repeats(cm, dev, w: synth.Workload, repeats: int | None = None) -> dic
             "matvec_pct_of_nominal_hbm": 100.0 * mv_gbs / NOMINAL_HBM_GBS,
             "encode_us": enc_us,
             "encode_gbs": nb["encode"] / (enc_us * 1e-6) / 1e9,
+            "encode_us_back_to_back": enc_b2b_us,
+            "encode_gbs_back_to_back": nb["encode"] / (enc_b2b_us * 1e-6) / 1e9,
             "matvec_us_median": float(np.median(mv)), "matvec_us_p95": float(np.percentile(mv, 95)),
             "matvec_gbs_median": nb["matvec"] / (np.median(mv) * 1e-6) / 1e9,
             "decode_us_median": float(np.median(dec)), "decode_us_p95": float(np.percentile(dec, 95)),

@@ -715,6 +715,7 @@ def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
         ev[i][2].record()
     torch.cuda.synchronize()
     g_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in ev]))
+    g_best_ms = float(min(e[0].elapsed_time(e[1]) for e in ev))
     d_ms = float(np.mean([e[1].elapsed_time(e[2]) for e in ev]))
     # survivors only: the stragglers known before the products run, only the
     # k blocks the decode reads are computed (same masks, same decode)
@@ -752,6 +753,11 @@ def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
                          "achieved": tflops, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
                          "frac": tflops / peaks["bf16_tflops"],
                          "frac_of_sustained": tflops / peaks["bf16_tflops_sustained"],
+                         # the burst peak is the best of ten cuBLAS launches:
+                         # the same statistic over these steps
+                         "achieved_best_of_steps": flops / (g_best_ms * 1e-3) / 1e12,
+                         "frac_best_of_steps": flops / (g_best_ms * 1e-3) / 1e12
+                         / peaks["bf16_tflops"],
                          "peak_source": peaks["source"] + " bf16 burst"},
             "decode_mat_ms": d_ms, "decode_mat_gbs": dec_bytes / (d_ms * 1e-3) / 1e9,
             "survivors_only": {"gemm_ms": gs_ms, "decode_mat_ms": ds_ms,

@@ -299,7 +299,10 @@ PROFILE_GEMM = synth.Workload("coded GEMM bf16 (16,12) 18432x8192x4096 (profilin
 PROFILE_SHUFFLE = synth.ShuffleWorkload("coded shuffling n=8 q=524288 s=q/4 r=256 "
                                         "(profiling case)", n=8, q=1 << 19, s=1 << 17,
                                         r=256, transitions=3)
-WORKLOADS = {"bandwidth": synth.BANDWIDTH, "profile": PROFILE}
+WORKLOADS = {"bandwidth": synth.BANDWIDTH, "profile": PROFILE,
+             # the (10,5) 12000 x 10000 config as the step (about 1 GB on the
+             # device): the short-code kernel forms, for ncu captures
+             "smallcode": synth.MATVEC}
 
 
 def config_of(w: synth.Workload) -> dict:
@@ -372,10 +375,15 @@ def run_ours(args, world, rank, local):
     # per step: the encode passes, the worker products and one decode launch
     launches = (math.ceil((w.n - w.k) / 16) + 1 + 1) * args.steps
 
+    if not full and args.workload == "smallcode":   # kernels only
+        if rank == 0:
+            print(json.dumps({"workload": w.name, "ms_per_step": ms / args.steps,
+                              "kernels_us": {k: v * 1e3 for k, v in avg.items()}}), flush=True)
+        return
     if not full:   # profiling case: kernels only, then the GEMM path once per step
         del A, parity
         torch.cuda.empty_cache()
-        gm = bench_gemm(cm, dev, PROFILE_GEMM, args.steps, args.warmup)
+        gm = bench_gemm(cm, dev, PROFILE_GEMM, args.steps, args.warmup, sustained=False)
         torch.cuda.empty_cache()
         shf = bench_shuffle(cm, dev, PROFILE_SHUFFLE)
         if rank == 0:
@@ -681,12 +689,15 @@ def bench_gd(cm, dev, steps: int, w: synth.GDWorkload = synth.GD) -> dict:
             "status": int(status.item())}
 
 
-def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
+def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int, sustained: bool = True) -> dict:
     """Coded GEMM: bf16 encode once, then per step all n worker GEMMs on the
     tensor cores and the decode of A B from the k survivors."""
     peaks = measured_peaks()
     P = synth.parity_coefficients(w.n, w.k)
     code = cm.Code(w.n, w.k, w.m, w.d, P, dtype="bf16")
+
+    def flops_all(c):
+        return 2.0 * w.n * c.L * w.d * w.gemm_n
     A, B = synth.gemm_inputs(w, device=dev)
     Bt = B.t().contiguous()
     del B
@@ -734,16 +745,22 @@ def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
     ds_ms = float(np.mean([e[1].elapsed_time(e[2]) for e in ev]))
     # sustained: back to back for about 0.6 s with SM clock, power and
     # throttle reasons sampled, against the sustained (power-capped) peak
-    n_sus = max(1, int(600.0 / g_ms))
-    torch.cuda.synchronize()
-    with ClockSampler(torch.cuda.current_device()) as clk:
-        e0.record()
-        for _ in range(n_sus):
-            cm.coded_gemm(code, A, par, Bt, Ct, status=status)
-        e1.record()
+    sus = None
+    if sustained:
+        n_sus = max(1, int(600.0 / g_ms))
         torch.cuda.synchronize()
-    sus_ms = e0.elapsed_time(e1) / n_sus
-    flops = 2.0 * w.n * code.L * w.d * w.gemm_n          # every coded row
+        with ClockSampler(torch.cuda.current_device()) as clk:
+            e0.record()
+            for _ in range(n_sus):
+                cm.coded_gemm(code, A, par, Bt, Ct, status=status)
+            e1.record()
+            torch.cuda.synchronize()
+        sus_ms = e0.elapsed_time(e1) / n_sus
+        sus = {"gemms": n_sus, "gemm_ms": sus_ms, "tflops": flops_all(code) / (sus_ms * 1e-3) / 1e12,
+               "frac_of_sustained_peak": flops_all(code) / (sus_ms * 1e-3) / 1e12
+               / peaks["bf16_tflops_sustained"],
+               "clocks": clk.summary()}
+    flops = flops_all(code)                              # every coded row
     useful = 2.0 * w.m * w.d * w.gemm_n                  # A B itself
     tflops = flops / (g_ms * 1e-3) / 1e12
     dec_bytes = w.k * code.L * w.gemm_n * 4 + w.m * w.gemm_n * 4
@@ -763,11 +780,7 @@ def bench_gemm(cm, dev, w: synth.Workload, steps: int, warmup: int) -> dict:
             "survivors_only": {"gemm_ms": gs_ms, "decode_mat_ms": ds_ms,
                                "tflops": 2.0 * w.k * code.L * w.d * w.gemm_n / (gs_ms * 1e-3) / 1e12,
                                "useful_tflops_per_step": useful / ((gs_ms + ds_ms) * 1e-3) / 1e12},
-            "sustained": {"gemms": n_sus, "gemm_ms": sus_ms,
-                          "tflops": flops / (sus_ms * 1e-3) / 1e12,
-                          "frac_of_sustained_peak": flops / (sus_ms * 1e-3) / 1e12
-                          / peaks["bf16_tflops_sustained"],
-                          "clocks": clk.summary()},
+            "sustained": sus,
             "encode_bf16_ms": enc_ms, "status": int(status.item())}
 
 
@@ -876,8 +889,10 @@ def main():
     ap.add_argument("--steps", type=int, default=40)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["bandwidth", "profile"], default="bandwidth",
-                    help="profile: a 512 MB case of the same path, for ncu captures")
+    ap.add_argument("--workload", choices=["bandwidth", "profile", "smallcode"],
+                    default="bandwidth",
+                    help="profile: a 1.3 GB case of the same path, for ncu captures; "
+                         "smallcode: the (10,5) 12000 x 10000 step (short-code kernels)")
     ap.add_argument("--no-cpu-baseline", action="store_true",
                     help="skip the oracle timing on the host cores")
     args = ap.parse_args()

@@ -126,6 +126,21 @@ __device__ __forceinline__ void stage_x(const MatvecArgs &a, float *xs, int64_t 
             const int bytes = left >= 4 ? 16 : (left > 0 ? (int)left * 4 : 0);
             cp_async16(xs + 4 * u, bytes ? X + col : X, bytes);
         }
+    } else if (kThreads % BP == 0) {
+        // thread tid always stages vector v = tid % BP, columns tid / BP +
+        // (kThreads / BP) i: pointers step, no per-element index arithmetic
+        constexpr int CS = kThreads / BP;   // columns per sweep
+        const int v = tid % BP;
+        int col = tid / BP;
+        float *dst = xs + v * C::GS + col;
+        const float *src = X + (c0 + col) * a.b + v;
+        const bool vin = v < a.b;
+        const int64_t left = a.d - c0;      // columns of X from c0 on
+#pragma unroll 4
+        for (; col < C::CX; col += CS, dst += CS, src += (int64_t)CS * a.b) {
+            const bool in = vin && col < left;
+            cp_async4(dst, in ? src : X, in ? 4 : 0);
+        }
     } else {
         for (int e = tid; e < C::CX * BP; e += kThreads) {
             const int col = e / BP, v = e % BP;

@@ -4,8 +4,9 @@
 // r < L and vector v < b <= 8.  Worker j < k reads its block in place from A
 // (rows past m are virtual zeros); worker j >= k reads the parity buffer.
 //
-// Mapping.  A persistent grid (SMs x one resident CTA of 6, 8 or 16 warps).  Work
-// unit = R consecutive block rows of one worker, owned by one warp; unit u
+// Mapping.  A persistent grid (SMs x one resident CTA of 8 warps; 6 for
+// single-round b = 1 launches).  Work unit = R consecutive block rows of one
+// worker, owned by one warp; unit u
 // belongs to the (u % nw)-th computed worker, so consecutive warps stream
 // different workers and all workers progress together, as the n workers of
 // the protocol do.  Normally all n workers are computed; when the survivors

@@ -144,10 +144,15 @@ cm_status cm_draw_erasures(uint64_t seed, uint64_t counter, int32_t n, int32_t k
  * inverts G_S in fp64 in its own shared memory (the k-e unit rows of
  * surviving systematic workers are eliminated first, then Gauss-Jordan with
  * partial pivoting on the e x e block of the missing systematic columns, in
- * one warp's registers) and forms the rows of G_S^-1 for the e missing
- * systematic blocks, then applies them to the k surviving results
- * (double-float arithmetic, about 2^-44 relative per term) while surviving
- * systematic blocks pass through.  Nothing is kept between calls.  Y (m x b
+ * the registers of one warp for e <= 4, of four for e <= 16) and forms the
+ * rows of G_S^-1 for the e missing systematic blocks, then applies them to
+ * the k surviving results (double-float arithmetic, about 2^-44 relative per
+ * term) while surviving systematic blocks pass through.  The launch is a
+ * programmatic dependent of the kernel before it on `stream`: the eliminating
+ * warps start from the kernel parameters at once and the others wait for the
+ * earlier grids before reading Yt, so after cm_matvec on the same stream the
+ * inversion overlaps the products' last round (after any other kernel the
+ * wait returns at once).  Nothing is kept between calls.  Y (m x b
  * fp32) is the concatenation of the k decoded blocks without the appended
  * zero rows.  Returns CM_ENOTDECODABLE when fewer than k bits are set; a
  * singular G_S (a zero pivot, or ||Q|| ||Q^-1|| beyond 1 / (64 eps) for the

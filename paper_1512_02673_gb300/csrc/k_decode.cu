@@ -97,10 +97,14 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     const int64_t p0 = (int64_t)blockIdx.x * a.chunk;
     const int64_t n = (per_block - p0 < a.chunk ? per_block - p0 : a.chunk);
     plan_setup(a.cp, a.survivors, pl);
-    // As a programmatic dependent of the products, the whole plan is formed
-    // (from the kernel parameters alone) while the products finish, then the
-    // grid waits for them before it reads a result; otherwise the first
-    // tile's loads overlap the elimination.
+    // Every decode is launched as a programmatic dependent of the kernel
+    // before it.  In the plan-first form (products and decode in one call)
+    // the whole plan is formed from the kernel parameters while the products
+    // finish, then the grid waits for them before it reads a result.  In the
+    // overlap form (a decode call of its own) the eliminating warps start at
+    // once and only the staging threads wait, so the elimination overlaps
+    // the previous kernel's tail (when that kernel lets dependents start, as
+    // the products do) and the first tile's loads.
     const bool overlap = !a.dependent;
     bool dec = false, rows_done = false;
     if (!overlap) {
@@ -126,6 +130,10 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
             const int lo = overlap && first && e > 0 ? 32 * NW : 0;
             const int tt = tid - lo;
             const int per = (kThreads - lo) / tn;
+            // launched as a programmatic dependent: the results are read
+            // only after the grids before this one are complete (the
+            // eliminating warps need none of them)
+            if (overlap && first && tt >= 0) griddep_wait();
             if (tt >= 0 && tt < per * tn) {
                 const int q = tt % tn;
                 const int64_t base = p0 + t0 + q;
@@ -311,10 +319,6 @@ cudaError_t launch_k3(const DecodeArgs &a, unsigned grid, cudaStream_t s)
     static const cudaError_t attr =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
     if (attr != cudaSuccess) return attr;
-    if (!a.dependent) {
-        kern<<<grid, kThreads, kSmem, s>>>(a);
-        return cudaGetLastError();
-    }
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -425,6 +425,31 @@ def test_matvec_config_100_repeats(cm, orc):
     assert max(errs) <= 1e-4, (max(errs), kappas[worst])
 
 
+def test_decode_right_behind_the_products_reads_complete_results(cm):
+    """cm_decode is launched as a programmatic dependent of the kernel before
+    it: behind the products (which let dependents start during their last
+    round) its staging threads must wait for the products to finish.  A
+    decode issued right behind a long products launch equals, bit for bit,
+    the same decode issued after a synchronize."""
+    n, k, m, d, b = 32, 24, 8192, 16384, 8
+    code = cm.Code(n, k, m, d, synth.parity_coefficients(n, k))
+    g = torch.Generator().manual_seed(11)
+    A = torch.randn((m, d), generator=g).to(DEV)
+    X = torch.randn((d, b), generator=g).to(DEV)
+    par = cm.encode(code, A)
+    Yt = torch.empty((n * code.L, b), dtype=torch.float64, device=DEV)
+    for c in range(4):
+        mask, _ = cm.draw_erasures(synth.ERASURE_SEED, c, n, k)
+        Yt.fill_(float("nan"))
+        cm.matvec(code, A, par, X, Yt)
+        Y_behind = cm.decode(code, Yt, mask)      # right behind the products
+        torch.cuda.synchronize()
+        Y_after = cm.decode(code, Yt, mask)       # after they are complete
+        torch.cuda.synchronize()
+        assert not torch.isnan(Y_behind).any()
+        assert torch.equal(Y_behind, Y_after)
+
+
 def test_bandwidth_config_every_element(cm, orc):
     """(32,24), A 65536 x 65536 fp32 (16 GiB), b = 8: the bench's launch
     configuration, checked element by element against the oracle: every

@@ -310,13 +310,15 @@ unsigned grid_for(int64_t items, int threads, int per_sm)
     return (unsigned)g;
 }
 
-// The vector decode with its shared-memory size set (once per process).
+// The vector decode, launched as a programmatic dependent.  The dynamic
+// shared-memory limit is a property of the function in each device's context,
+// so it is set on every call (about 0.2 us), as the other launchers do.
 template <int EMAX, int NW>
 cudaError_t launch_k3(const DecodeArgs &a, unsigned grid, cudaStream_t s)
 {
     constexpr int kSmem = CM_MAX_N * kTile * (int)sizeof(float2);
     auto kern = decode_kernel<EMAX, NW>;
-    static const cudaError_t attr =
+    const cudaError_t attr =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
     if (attr != cudaSuccess) return attr;
     cudaLaunchConfig_t cfg = {};

@@ -64,6 +64,8 @@
 // drained with bounded waits, and both CTAs meet at a cluster barrier before
 // the TMEM is freed and they exit, so neither touches the other's shared
 // memory while it is not live.
+#include <atomic>
+
 #include "cm_internal.cuh"
 #include "tma.cuh"
 
@@ -563,19 +565,25 @@ cudaError_t launch_coded_gemm(const CodeParams &cp, const uint16_t *A, int64_t l
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    // persistent: as many pairs as can be resident at once (the attribute and
-    // the occupancy query are the same for every call: done once, thread-safe)
-    static const int resident = [&cfg]() -> int {
-        if (cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 SMEM_BYTES) != cudaSuccess)
-            return -1;
+    // persistent: as many pairs as can be resident at once.  The shared-memory
+    // limit belongs to the function in each device's context: set on every
+    // call (about 0.2 us); the cluster occupancy is queried once per device.
+    if (cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             SMEM_BYTES) != cudaSuccess)
+        return cudaErrorInvalidConfiguration;
+    static std::atomic<int> resident_of[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return cudaErrorInvalidConfiguration;
+    int resident = dev >= 0 && dev < 64 ? resident_of[dev].load(std::memory_order_relaxed) : 0;
+    if (resident <= 0) {
         cudaLaunchConfig_t q = cfg;
         q.gridDim = dim3(2 * (unsigned)((cm_sm_count() + 1) / 2));
         int c = 0;
-        if (cudaOccupancyMaxActiveClusters(&c, gemm_kernel, &q) != cudaSuccess) return -1;
-        return c;
-    }();
-    if (resident < 0) return cudaErrorInvalidConfiguration;
+        if (cudaOccupancyMaxActiveClusters(&c, gemm_kernel, &q) != cudaSuccess)
+            return cudaErrorInvalidConfiguration;
+        resident = c;
+        if (c > 0 && dev >= 0 && dev < 64) resident_of[dev].store(c, std::memory_order_relaxed);
+    }
     int clusters = resident;
     if (clusters < 1) return cudaErrorInvalidConfiguration;
     if (clusters > g.pairs) clusters = (int)g.pairs;

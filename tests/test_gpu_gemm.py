@@ -83,6 +83,23 @@ def check_encode_bf16(orc, n, k, A, P, par):
     assert np.all(np.abs(got - want) <= tol), np.max(np.abs(got - want) - tol)
 
 
+@pytest.mark.parametrize("n,k,m,d,ld", [
+    (6, 3, 301, 203, 208),       # elementwise form (k <= 8): ragged columns and rows
+    (20, 10, 613, 257, 264),     # elementwise form with up to 16 data blocks
+    (16, 12, 500, 203, 208),     # tiled form (12 data blocks, 4 parity blocks)
+])
+def test_encode_bf16_ragged_columns(cm, orc, n, k, m, d, ld):
+    """bf16 encode on a padded row pitch with d not a multiple of 4: each
+    encode form, its 4-column chunks and its scalar tail, against the
+    oracle's bound (RNE output within one bf16 unit)."""
+    P = synth.parity_coefficients(n, k)
+    code = cm.Code(n, k, m, d, P, dtype="bf16")
+    A = synth.gaussian((m, ld), 5, dtype=torch.bfloat16).to(DEV)[:, :d]
+    par = cm.encode(code, A)
+    torch.cuda.synchronize()
+    check_encode_bf16(orc, n, k, A, P, par)
+
+
 @pytest.mark.parametrize("n,k,m,d,N", [
     (6, 3, 300, 128, 64),        # one partial column tile
     (5, 4, 517, 200, 80),        # d not a multiple of 64, N not of 256, L not of 128

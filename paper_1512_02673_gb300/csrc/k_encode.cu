@@ -25,9 +25,11 @@
 // boxes past the last full block read as zero) plus, if m is not a multiple
 // of L, one 2-D box of the partial block whose rows past m read as zero;
 // blocks wholly past m are skipped.  Sub-steps stream through a per-warp ring
-// of ST slots with one mbarrier each (lane 0 issues, the warp consumes), so
-// several KB per warp are in flight with no per-lane copy work, and small
-// slots leave room for 16 warps per SM.  Lane l owns columns [4l, 4l+4) of
+// of ST = 2 slots with one mbarrier each (lane 0 issues, the warp consumes),
+// so several KB per warp are in flight with no per-lane copy work, and small
+// rings leave room for 2 or 3 CTAs of 8 warps per SM (registers decide: 3
+// for up to 4 parity blocks).  A third slot per warp measured up to 5 %
+// slower.  Lane l owns columns [4l, 4l+4) of
 // the step and keeps the accumulators of all parity blocks of the pass in
 // registers (packed fp32x2 FMAs with the coefficient pair (P[p][i], P[p][i])
 // read as a shared-memory broadcast), then stores them with coalesced
@@ -43,7 +45,7 @@ namespace {
 constexpr int STEP = 128;       // columns per step
 constexpr int SEG = 32;         // steps per work unit, at most
 constexpr int KC = 8;           // data blocks per sub-step (one TMA box)
-constexpr int ST = 3;           // ring slots per warp
+constexpr int ST = 2;           // ring slots per warp
 constexpr int kWarps = 8;
 
 template <typename T>

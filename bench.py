@@ -415,6 +415,8 @@ def run_ours(args, world, rank, local):
     # survivors-only mode on the same workload: the straggler set is drawn
     # first and only the k surviving blocks are computed
     so = bench_survivors_only(cm, code, A, parity, X, Yt, Y, status, w, args)
+    one_call = bench_one_call(cm, code, A, parity, X, Y, status, w, avg["matvec"],
+                              so["matvec_ms"])
 
     # secondary workloads: the other rows of the hot path
     del A, parity
@@ -462,7 +464,8 @@ def run_ours(args, world, rank, local):
                 "d2h_bytes_per_step": w.m * w.b * 4},
         "gpu_launches": launches,
         "clocks": clk.summary(),
-        "secondary": {"survivors_only": so, "gemm": gemm, "gd": gd,
+        "secondary": {"survivors_only": so, "matvec_decode_one_call": one_call,
+                      "gemm": gemm, "gd": gd,
                       "matvec_100_repeats": mv100, "tiny": tiny,
                       "coded_shuffling": shuffle, "paper_shaped": paper,
                       "runtime_model": runtime_model_report(cm)},
@@ -496,6 +499,37 @@ def bench_survivors_only(cm, code, A, parity, X, Yt, Y, status, w, args) -> dict
     read = w.k * L * w.d * 4 + w.d * w.b * 4 + w.k * L * w.b * 8
     return {"matvec_ms": mv, "decode_ms": dec, "matvec_gbs": read / (mv * 1e-3) / 1e9,
             "bytes_read": read, "status": int(status.item())}
+
+
+def bench_one_call(cm, code, A, parity, X, Y, status, w, products_ms: float,
+                   survivor_products_ms: float, reps: int = 3) -> dict:
+    """Products and decode in one call (cm_matvec_decode: the decode is a
+    programmatic dependent of the products) on the headline workload, all
+    workers and survivors only; the decode's added time is the call against
+    the same products timed alone in this run."""
+    ws = torch.empty(cm.matvec_decode_workspace_bytes(code, w.b), dtype=torch.uint8,
+                     device=A.device)
+    masks = [cm.draw_erasures(synth.ERASURE_SEED, 5000 + i, w.n, w.k)[0] for i in range(reps + 2)]
+    out = {}
+    for name, only, alone in (("all_workers", False, products_ms),
+                              ("survivors_only", True, survivor_products_ms)):
+        for i in range(2):
+            cm.matvec_decode(code, A, parity, X, masks[i], only_survivors=only, Y=Y, ws=ws,
+                             status=status)
+        torch.cuda.synchronize()
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(reps)]
+        for i, (e0, e1) in enumerate(ev):
+            e0.record()
+            cm.matvec_decode(code, A, parity, X, masks[2 + i], only_survivors=only, Y=Y, ws=ws,
+                             status=status)
+            e1.record()
+        torch.cuda.synchronize()
+        ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+        out[name] = {"ms_per_call": ms, "products_alone_ms": alone,
+                     "decode_added_us": (ms - alone) * 1e3}
+    out["status"] = int(status.item())
+    return out
 
 
 def shuffle_bytes(st: dict, r: int) -> dict:

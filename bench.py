@@ -415,8 +415,7 @@ def run_ours(args, world, rank, local):
     # survivors-only mode on the same workload: the straggler set is drawn
     # first and only the k surviving blocks are computed
     so = bench_survivors_only(cm, code, A, parity, X, Yt, Y, status, w, args)
-    one_call = bench_one_call(cm, code, A, parity, X, Y, status, w, avg["matvec"],
-                              so["matvec_ms"])
+    one_call = bench_one_call(cm, code, A, parity, X, Yt, Y, status, w)
 
     # secondary workloads: the other rows of the hot path
     del A, parity
@@ -501,33 +500,48 @@ def bench_survivors_only(cm, code, A, parity, X, Yt, Y, status, w, args) -> dict
             "bytes_read": read, "status": int(status.item())}
 
 
-def bench_one_call(cm, code, A, parity, X, Y, status, w, products_ms: float,
-                   survivor_products_ms: float, reps: int = 3) -> dict:
+def bench_one_call(cm, code, A, parity, X, Yt, Y, status, w, reps: int = 8) -> dict:
     """Products and decode in one call (cm_matvec_decode: the decode is a
     programmatic dependent of the products) on the headline workload, all
-    workers and survivors only; the decode's added time is the call against
-    the same products timed alone in this run."""
+    workers and survivors only.  Each repeat times the same products alone
+    (cm_matvec / cm_matvec_survivors) and then the one call on the same
+    erasure set, so the decode's added time is a median of paired
+    differences."""
     ws = torch.empty(cm.matvec_decode_workspace_bytes(code, w.b), dtype=torch.uint8,
                      device=A.device)
     masks = [cm.draw_erasures(synth.ERASURE_SEED, 5000 + i, w.n, w.k)[0] for i in range(reps + 2)]
     out = {}
-    for name, only, alone in (("all_workers", False, products_ms),
-                              ("survivors_only", True, survivor_products_ms)):
+    for name, only in (("all_workers", False), ("survivors_only", True)):
+        def alone(m):
+            if only:
+                cm.matvec_survivors(code, A, parity, X, m, Yt=Yt, status=status)
+            else:
+                cm.matvec(code, A, parity, X, Yt, status=status)
+
+        def fused(m):
+            cm.matvec_decode(code, A, parity, X, m, only_survivors=only, Y=Y, ws=ws,
+                             status=status)
+
         for i in range(2):
-            cm.matvec_decode(code, A, parity, X, masks[i], only_survivors=only, Y=Y, ws=ws,
-                             status=status)
+            alone(masks[i])
+            fused(masks[i])
         torch.cuda.synchronize()
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(reps)]
-        for i, (e0, e1) in enumerate(ev):
-            e0.record()
-            cm.matvec_decode(code, A, parity, X, masks[2 + i], only_survivors=only, Y=Y, ws=ws,
-                             status=status)
-            e1.record()
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(reps)]
+        for i, e in enumerate(ev):
+            m = masks[2 + i]
+            e[0].record()
+            alone(m)
+            e[1].record()
+            e[2].record()
+            fused(m)
+            e[3].record()
         torch.cuda.synchronize()
-        ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
-        out[name] = {"ms_per_call": ms, "products_alone_ms": alone,
-                     "decode_added_us": (ms - alone) * 1e3}
+        t_alone = [e[0].elapsed_time(e[1]) for e in ev]
+        t_fused = [e[2].elapsed_time(e[3]) for e in ev]
+        out[name] = {"ms_per_call": float(np.median(t_fused)),
+                     "products_alone_ms": float(np.median(t_alone)),
+                     "decode_added_us": float(np.median(np.subtract(t_fused, t_alone))) * 1e3,
+                     "repeats": reps}
     out["status"] = int(status.item())
     return out
 

@@ -17,7 +17,8 @@
 //  * plan_setup (all threads): P into shared memory (16-byte loads of the
 //    parameter space), the survivor lists by ballots in warp 0.
 //  * plan_eliminate (one warp for e <= 4, else four warps, one per
-//    scheduler): Q^-1 in fp64 with [Q | I] held in registers, its 2e^2
+//    scheduler; e <= 2 in closed form, adj(Q) / det Q, by one warp):
+//    Q^-1 in fp64 with [Q | I] held in registers, its 2e^2
 //    entries spread over the threads.  The pivot search is one warp
 //    reduction over the threads holding the pivot column; that warp hands
 //    the pivot key and the column to the others through shared memory (one
@@ -203,6 +204,20 @@ __device__ __forceinline__ void df_fma(float dh, float dl, float yh, float yl, f
     sh = s1;
 }
 
+// (sh, sl) += d (yh + yl) for an fp32 coefficient d (df_fma with a zero low
+// part, one rounded product fewer).
+__device__ __forceinline__ void df_fma1(float d, float yh, float yl, float &sh, float &sl)
+{
+    const float p = __fmul_rn(d, yh);
+    const float pe = __fmaf_rn(d, yh, -p);                   // exact error of p
+    const float t = __fmul_rn(d, yl);
+    const float s1 = __fadd_rn(sh, p);                       // TwoSum(sh, p)
+    const float bb = __fsub_rn(s1, sh);
+    const float err = __fadd_rn(__fsub_rn(sh, __fsub_rn(s1, bb)), __fsub_rn(p, bb));
+    sl = __fadd_rn(sl, __fadd_rn(err, __fadd_rn(pe, t)));
+    sh = s1;
+}
+
 __device__ __forceinline__ double shfl_double(double v, int src)
 {
     const long long b = __double_as_longlong(v);
@@ -264,6 +279,53 @@ __device__ __forceinline__ void elim_sync()
     else asm volatile("bar.sync 1, %0;\n" ::"r"(NW * 32) : "memory");
 }
 
+// Q^-1 for e <= 2 in closed form, by warp 0 alone (no barrier: the other
+// eliminating warps return at once).  Q's entries are fp32 values, so their
+// products are exact in fp64: det Q = q00 q11 - q01 q10 carries one rounding
+// and Q^-1 = adj(Q) / det Q one more per entry, against a pivot, a scaling
+// and a reciprocal per column of the elimination.  G_S counts as singular when
+// det Q (Q itself for e = 1) is zero, subnormal or not finite (exactly when Q
+// is singular, short of overflow and underflow), or by the elimination's
+// condition bound.
+__device__ __forceinline__ void plan_inverse_small(Plan &pl, int k)
+{
+    const int t = threadIdx.x;
+    if (t >= 32) return;
+    const int e = pl.e;
+    // Q[r][j] = P[Ps[r]][M[j]]: row r a surviving parity worker, column j a
+    // missing block
+    const float f00 = pl.P[(pl.Ps[0] - k) * k + pl.M[0]];
+    const float f01 = e == 2 ? pl.P[(pl.Ps[0] - k) * k + pl.M[1]] : 0.f;
+    const float f10 = e == 2 ? pl.P[(pl.Ps[1] - k) * k + pl.M[0]] : 0.f;
+    const float f11 = e == 2 ? pl.P[(pl.Ps[1] - k) * k + pl.M[1]] : 0.f;
+    const float qmax = fmaxf(fmaxf(fabsf(f00), fabsf(f01)), fmaxf(fabsf(f10), fabsf(f11)));
+    const double q00 = exact_double(f00), q01 = exact_double(f01);
+    const double q10 = exact_double(f10), q11 = exact_double(f11);
+    const double det = e == 1 ? q00 : __dsub_rn(__dmul_rn(q00, q11), __dmul_rn(q01, q10));
+    const uint32_t ef =
+        (uint32_t)((unsigned long long)__double_as_longlong(det) >> 52) & 0x7FFu;
+    bool sing = ef == 0u || ef == 0x7FFu;
+    float qi = 0.f;
+    if (!sing && t < e * e) {
+        const int c = t / e, a = t - c * e;      // Q^-1[c][a] = adj(Q)[c][a] / det Q
+        double adj = 1.0;                        // e = 1
+        if (e == 2) {
+            if (c == a) adj = c == 0 ? q11 : q00;
+            else adj = c == 0 ? -q01 : -q10;
+        }
+        float h, l;
+        split_double(adj / det, h, l);
+        pl.Qh[c][a] = h;
+        pl.Ql[c][a] = l;
+        qi = fabsf(h);
+    }
+    qi = __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(qi)));
+    // not-a-number fails the comparison and counts as singular
+    if (!sing && !((float)e * qmax * ((float)e * qi) < (float)(1.0 / (64.0 * DBL_EPSILON))))
+        sing = true;
+    if (t == 0 && sing) pl.singular = 1;
+}
+
 // Q^-1 by the first NW warps of the CTA (1, or 4: one per scheduler, since
 // each warp gets about one fp64 instruction per 64 cycles); EMAX >= e is a
 // power of two (4, 8 or 16) with 2 EMAX^2 >= 32 NW.  The 2 EMAX x EMAX
@@ -289,6 +351,10 @@ __device__ __forceinline__ void plan_eliminate(Plan &pl, int k)
     constexpr int SL = T / EMAX;                 // column slots
     constexpr int EPL = 2 * EMAX * EMAX / T;     // entries per thread
     static_assert(EPL >= 1 && SL * EPL == 2 * EMAX, "layout");
+    if (pl.e <= 2) {
+        plan_inverse_small(pl, k);
+        return;
+    }
     const int t = threadIdx.x;
     const int lane = t & 31;
     const int e = pl.e;

@@ -3,17 +3,19 @@
 //
 // One launch per decode and no state kept between calls: every CTA forms the
 // decode in its own shared memory (decode_plan.cuh: the e x e block Q of G_S
-// inverted in fp64 in registers by one or four warps, then the rows D of
-// G_S^-1 for the missing systematic blocks), and applies it: missing block
-// M[c] = sum_p D[c][p] Yt_S[p] over the k surviving results, while surviving
-// systematic blocks pass through.  Each surviving value is loaded once per
-// CTA.  A zero (or relatively negligible) pivot marks G_S singular:
+// inverted in fp64 in registers by one or four warps) and applies it.  The
+// vector decode applies the rows of G_S^-1 for the missing systematic blocks
+// in two factors, Z_M = Q^-1 (Y_par - P[Ps][S_sys] Y_sys), the second formed
+// while the elimination runs; the matrix decode forms the rows D of G_S^-1
+// and sums M[c] = sum_p D[c][p] Yt_S[p] over the k surviving results.
+// Surviving systematic blocks pass through.  Each surviving value is loaded
+// once per CTA.  A zero (or relatively negligible) pivot marks G_S singular:
 // CM_ESINGULAR goes to the status word and no missing block is written
 // (surviving systematic blocks are still copied).
 //
 // fp64 arithmetic runs at a small fraction of the fp32 rate on this part, so
 // the vector decode works in double-float arithmetic on the fp32 pipe: each
-// fp64 worker result and each row entry is a (high, low) fp32 pair split by
+// fp64 worker result and each entry of Q^-1 is a (high, low) fp32 pair split by
 // integer bit manipulation, products are formed exactly with an FMA and the
 // sums are kept as (sum, compensation) pairs (Knuth's TwoSum), about 2^-44
 // relative per term, far below the rounding of the fp32 output; fp32 outputs
@@ -65,32 +67,50 @@ __device__ __forceinline__ void store_out(const DecodeArgs &a, int64_t out, floa
     }
 }
 
+// Named barrier among the warps that stage while the first NW warps
+// eliminate (barrier 2; 0 is __syncthreads, 1 the eliminating warps').
+__device__ __forceinline__ void staging_sync(int threads)
+{
+    asm volatile("bar.sync 2, %0;\n" ::"r"(threads) : "memory");
+}
+
 // K3.  A persistent grid, one CTA of 1024 threads per SM; CTA i owns the row
 // positions [i chunk, (i + 1) chunk) (row r of every block and vector v,
-// position r b + v) of all k output blocks, taken in tiles of kTile.
+// position r b + v) of all k output blocks, taken in tiles of kTile.  With
+// Y_par the results of the e surviving parity workers and Y_sys those of
+// the ks = k - e surviving systematic ones, the missing blocks are
+//   Z_M = Q^-1 R,   R = Y_par - P[Ps][S_sys] Y_sys,
+// the same rows of G_S^-1 applied in two factors: R needs only P, so it is
+// formed while the elimination runs, and what follows the elimination is a
+// sum of e terms per output.
 //  1. plan_setup.
 //  2. For every tile: the k surviving values of its positions are loaded
 //     (position fastest, coalesced; a thread's loads issued together) and
 //     staged in shared memory as (high, low) fp32 pairs, and those of the
 //     surviving systematic blocks are written out at once (the pass-through,
-//     fp32 rounding of the fp64 results).  For the first tile the first NW
-//     warps eliminate meanwhile (when blocks are missing), so the loads
-//     overlap the elimination, and the rows D of the decode follow.
-//  3. Every (missing block c, position) of the tile is one thread's item: a
-//     short loop over the k staged survivors sums D[c][p] y_p in
-//     double-float arithmetic.  Many short items keep every scheduler busy;
-//     a thread per position with all e blocks left one warp per scheduler
-//     waiting on its own dependent operations, and code that runs once per
-//     item must stay small (fully unrolled, fetching the instructions
-//     dominated).
+//     fp32 rounding of the fp64 results).  For the first tile of a decode
+//     call of its own the first NW warps eliminate meanwhile (when blocks
+//     are missing), so the loads overlap the elimination.
+//  3. Every (parity survivor a, position) of the tile is one thread's item:
+//     R[a] = y_Ps[a] - sum_p P[Ps[a]][S[p]] y_S[p] over the systematic
+//     survivors, in double-float arithmetic, written over y_Ps[a]'s slot
+//     (the only item that reads it).  The staging warps do this while the
+//     first tile's elimination is still running.
+//  4. Every (missing block c, position) is one thread's item: sum_a
+//     Q^-1[c][a] R[a] in double-float arithmetic.  Many short items keep
+//     every scheduler busy (a thread per position with all e blocks left one
+//     warp per scheduler waiting on its own dependent operations), and code
+//     that runs once per item stays small (fully unrolled loops spent most
+//     of their time fetching instructions).
 template <int EMAX, int NW>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecodeArgs a)
 {
     extern __shared__ float2 ysm[];   // [CM_MAX_N][kTile] (high, low) pairs of the survivors
     __shared__ Plan pl;
-    __shared__ float Dh[kMaxE][CM_MAX_N], Dl[kMaxE][CM_MAX_N];
+    __shared__ float Pn[kMaxE][CM_MAX_N + 1];   // -P[Ps[a]][S[p]], p < ks (padded rows)
     const int k = a.cp.k;
     const int e = missing_blocks(k, a.survivors);
+    const int ks = k - e;
     const int tid = threadIdx.x;
     const int64_t per_block = a.cp.L * a.b;
     const int64_t mb = a.cp.m * a.b;
@@ -99,42 +119,43 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
     plan_setup(a.cp, a.survivors, pl);
     // Every decode is launched as a programmatic dependent of the kernel
     // before it.  In the plan-first form (products and decode in one call)
-    // the whole plan is formed from the kernel parameters while the products
-    // finish, then the grid waits for them before it reads a result.  In the
-    // overlap form (a decode call of its own) the eliminating warps start at
-    // once and only the staging threads wait, so the elimination overlaps
-    // the previous kernel's tail (when that kernel lets dependents start, as
-    // the products do) and the first tile's loads.
+    // the eliminating warps form Q^-1 from the kernel parameters while the
+    // products finish, and every thread waits for the products before it
+    // reads a result.  In the overlap form (a decode call of its own) the
+    // eliminating warps start at once and the staging threads wait before
+    // their loads, so the elimination overlaps the previous kernel's tail
+    // (when that kernel lets dependents start, as the products do), the
+    // first tile's loads and its R.
     const bool overlap = !a.dependent;
-    bool dec = false, rows_done = false;
     if (!overlap) {
         if (e > 0 && tid < 32 * NW) plan_eliminate<EMAX, NW>(pl, k);
-        __syncthreads();
-        if (e > 0 && !pl.singular) {
-            plan_rows(pl, k, Dh, Dl);
-            dec = true;
-        }
-        rows_done = true;
         griddep_wait();
     }
+    bool dec = false;
     for (int64_t t0 = 0; t0 < n; t0 += kTile) {
         const int tn = (int)(n - t0 < kTile ? n - t0 : kTile);
         const bool first = t0 == 0;
-        if (overlap && first && e > 0 && tid < 32 * NW) plan_eliminate<EMAX, NW>(pl, k);
-        // stage the tile; the eliminating warps skip the first one.  Thread
-        // tt takes position q = tt % tn of survivors tt / tn, tt / tn + per,
-        // ... (per = threads / tn), SB of them with their loads issued before
-        // any store (one division per thread, none per value)
-        {
-            constexpr int SB = 4;
-            const int lo = overlap && first && e > 0 ? 32 * NW : 0;
+        const bool split = overlap && first && e > 0;   // the first NW warps eliminate
+        const int lo = split ? 32 * NW : 0;
+        if (split && tid < lo) {
+            plan_eliminate<EMAX, NW>(pl, k);
+            griddep_wait();   // before the later tiles' loads and any store
+        } else {
+            if (overlap && first) griddep_wait();
             const int tt = tid - lo;
+            if (first) {
+                for (int u = tt; u < e * ks; u += kThreads - lo) {
+                    const int c = u / ks, p = u - c * ks;
+                    Pn[c][p] = -pl.P[(pl.Ps[c] - k) * k + pl.S[p]];
+                }
+            }
+            // stage the tile: thread tt takes position q = tt % tn of
+            // survivors tt / tn, tt / tn + per, ... (per = threads / tn), SB
+            // of them with their loads issued before any store (one division
+            // per thread, none per value)
+            constexpr int SB = 4;
             const int per = (kThreads - lo) / tn;
-            // launched as a programmatic dependent: the results are read
-            // only after the grids before this one are complete (the
-            // eliminating warps need none of them)
-            if (overlap && first && tt >= 0) griddep_wait();
-            if (tt >= 0 && tt < per * tn) {
+            if (tt < per * tn) {
                 const int q = tt % tn;
                 const int64_t base = p0 + t0 + q;
                 for (int pb = tt / tn; pb < k; pb += SB * per) {
@@ -168,25 +189,36 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
                     }
                 }
             }
+            if (e > 0) {
+                if (split) staging_sync(kThreads - lo);
+                else __syncthreads();
+                for (int u = tt; u < e * tn; u += kThreads - lo) {
+                    const int c = u / tn, q = u - c * tn;
+                    float2 *r = &ysm[(ks + c) * kTile + q];
+                    float sh = r->x, sl = r->y;
+#pragma unroll 4
+                    for (int p = 0; p < ks; ++p) {
+                        const float2 y = ysm[p * kTile + q];
+                        df_fma1(Pn[c][p], y.x, y.y, sh, sl);
+                    }
+                    *r = make_float2(sh, sl);
+                }
+            }
         }
         if (e == 0) continue;
         __syncthreads();
         if (first) {
             if (pl.singular && blockIdx.x == 0 && tid == 0 && a.status) *a.status = CM_ESINGULAR;
-            if (!rows_done) {
-                dec = !pl.singular;
-                if (dec) plan_rows(pl, k, Dh, Dl);
-                __syncthreads();
-            }
+            dec = !pl.singular;
         }
         if (dec) {
             for (int u = tid; u < e * tn; u += kThreads) {
                 const int c = u / tn, q = u - c * tn;
                 float sh = 0.f, sl = 0.f;
 #pragma unroll 4
-                for (int p = 0; p < k; ++p) {
-                    const float2 y = ysm[p * kTile + q];
-                    df_fma(Dh[c][p], Dl[c][p], y.x, y.y, sh, sl);
+                for (int j = 0; j < e; ++j) {
+                    const float2 r = ysm[(ks + j) * kTile + q];
+                    df_fma(pl.Qh[c][j], pl.Ql[c][j], r.x, r.y, sh, sl);
                 }
                 const int64_t out = (int64_t)pl.M[c] * per_block + p0 + t0 + q;
                 if (out < mb) store_out(a, out, sh, sl);

@@ -326,6 +326,35 @@ def test_singular_generator_sets_status(cm):
     assert e.value.status == cm.CM_ENOTDECODABLE
 
 
+def test_singular_proportional_rows_and_well_posed_neighbours(cm, orc):
+    """Two missing blocks take the closed-form inverse: with parity rows
+    proportional by a power of two, q00 q11 - q01 q10 is zero exactly (fp32
+    products are exact in fp64), so the set is flagged singular; the sets of
+    the same code that avoid the pair decode to the oracle's Y = A X."""
+    n, k, m, d = 6, 3, 90, 40
+    P = synth.parity_coefficients(n, k)
+    P[1] = 2.0 * P[0]                         # rows 3 and 4 of G proportional
+    code = cm.Code(n, k, m, d, P)
+    A = synth.gaussian((m, d), 5).to(DEV)
+    X = synth.gaussian((d, 1), 6).to(DEV)
+    par = cm.encode(code, A)
+    Yt = cm.matvec(code, A, par, X)
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    L = code.L
+    Y = torch.full((m, 1), 7.0, device=DEV)
+    cm.decode(code, Yt, 0b011001, Y=Y, status=status)     # survivors {0, 3, 4}: e = 2
+    torch.cuda.synchronize()
+    assert status.item() == cm.CM_ESINGULAR
+    assert torch.all(Y[L:] == 7.0)
+    want = orc.matmul(A.cpu().numpy().astype(np.float64), X.cpu().numpy().astype(np.float64))
+    for mask in (0b101001, 0b110001, 0b101010, 0b100110, 0b001011):   # not both of rows 3, 4
+        status.zero_()
+        Y = cm.decode(code, Yt, mask, status=status)
+        torch.cuda.synchronize()
+        assert status.item() == cm.CM_OK, bin(mask)
+        assert rel_l2_cols(Y.cpu().numpy(), want).max() <= 1e-4, bin(mask)
+
+
 def test_concurrent_decodes_on_two_streams(cm, orc):
     """The decode keeps nothing between calls: hundreds of decodes queued on
     two streams at once (behind a device sleep, so they pile up and then run

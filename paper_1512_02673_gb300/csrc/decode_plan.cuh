@@ -247,11 +247,15 @@ __device__ __forceinline__ void plan_setup(const CodeParams &cp, uint32_t surviv
     const int nwarps = blockDim.x >> 5;
     const int n = cp.n, k = cp.k;
     // 16-byte loads of the parameter space, lane l of warp w taking float4
-    // number w + nwarps l
+    // number w + nwarps l (at most one per thread for CTAs of 64 threads or
+    // more: (n - k) k <= 256 floats); the first is loaded before the ballots
+    // and stored after them, so that its latency covers them
     const int n4 = ((n - k) * k + 3) / 4;
     const float4 *P4 = reinterpret_cast<const float4 *>(cp.P);
     float4 *S4 = reinterpret_cast<float4 *>(pl.P);
-    for (int i = warp + nwarps * lane; i < n4; i += nwarps * 32) S4[i] = P4[i];
+    const int i0 = warp + nwarps * lane;
+    float4 v0 = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i0 < n4) v0 = P4[i0];
     if (warp == 0) {
         const uint32_t below = (1u << lane) - 1u;
         const bool sel = lane < n && ((survivors >> lane) & 1u);
@@ -267,6 +271,8 @@ __device__ __forceinline__ void plan_setup(const CodeParams &cp, uint32_t surviv
             pl.singular = 0;
         }
     }
+    if (i0 < n4) S4[i0] = v0;
+    for (int i = i0 + nwarps * 32; i < n4; i += nwarps * 32) S4[i] = P4[i];
     __syncthreads();
 }
 

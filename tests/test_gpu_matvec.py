@@ -235,6 +235,35 @@ def test_decode_many_missing_blocks(cm, orc, n, k, e):
         assert err.max() <= 1e-6, (hex(mask), err)
 
 
+@pytest.mark.parametrize("n,k,e,b,m", [(6, 3, 2, 1, 3 * 60000 - 1), (32, 24, 8, 8, 24 * 5200),
+                                       (20, 10, 10, 2, 10 * 40000 - 7)])
+def test_decode_several_tiles_per_cta(cm, orc, n, k, e, b, m):
+    """Problems with more than 152 x 256 row positions (L b) give every CTA of
+    the decode several tiles: the first stages while the elimination runs,
+    the later ones stage with every thread.  Own decode call and products +
+    decode in one call, against the oracle's fp64 decode of the same
+    results."""
+    d = 16
+    P = synth.parity_coefficients(n, k)
+    code = cm.Code(n, k, m, d, P)
+    assert code.L * b > 152 * 256
+    A = synth.gaussian((m, d), 31).to(DEV)
+    X = synth.gaussian((d, b), 32).to(DEV)
+    par = cm.encode(code, A)
+    Yt = cm.matvec(code, A, par, X)
+    Yt_cpu = Yt.cpu().numpy()
+    drawn = cm.draw_erasures(synth.ERASURE_SEED, 77, n, k)[0]
+    for mask in _masks_with_e_missing(n, k, e, seed=n * 1000 + e) + [drawn]:
+        status = torch.zeros(1, dtype=torch.int32, device=DEV)
+        Y = cm.decode(code, Yt, mask, status=status)
+        Yf = cm.matvec_decode(code, A, par, X, mask, status=status)
+        torch.cuda.synchronize()
+        assert status.item() == 0
+        want = orc.decode(n, k, m, P.astype(np.float64), mask, Yt_cpu)
+        assert rel_l2_cols(Y.cpu().numpy(), want).max() <= 1e-6, hex(mask)
+        assert rel_l2_cols(Yf.cpu().numpy(), want).max() <= 1e-6, hex(mask)
+
+
 def test_pass_through_is_rounded_to_nearest(cm):
     """Surviving systematic blocks are the fp64 results rounded to fp32 (to
     nearest, ties to even; the kernels convert by integer arithmetic): bit

@@ -30,11 +30,14 @@
 //    binade (an exact scale that keeps the rows from growing by a product of
 //    pivots).  Afterwards row prow[c] holds column c's pivot d_c and
 //    Q^-1[c][a] = W[prow[c]][e + a] / d_c, kept as (high, low) fp32 pairs.
-//  * G_S counts as singular when a pivot is zero, subnormal or not finite, or
-//    when ||Q||_inf ||Q^-1||_inf, bounded by (e max|Q|)(e max|Q^-1|), exceeds
-//    1 / (64 eps) (evaluated in fp32: it is a threshold).
-//  * plan_rows (all threads): the rows D[c][p] above, from the (high, low)
-//    pairs of Q^-1 and the exact fp32 values of P in double-float arithmetic.
+//  * G_S counts as singular when a pivot (det Q for e <= 2) is zero,
+//    subnormal or not finite, or when ||Q||_inf ||Q^-1||_inf, bounded by
+//    (e max|Q|)(e max|Q^-1|), exceeds 1 / (64 eps) (evaluated in fp32: it is
+//    a threshold).
+//  * plan_rows (all threads; the matrix decode): the rows D[c][p] above, from
+//    the (high, low) pairs of Q^-1 and the exact fp32 values of P in
+//    double-float arithmetic.  The vector decode applies the same rows in two
+//    factors instead, Q^-1 (Yt_Ps - P[Ps][S_sys] Yt_S_sys).
 //
 // fp64 runs at a small fraction of the fp32 rate on this part: each warp
 // gets about one fp64 instruction per 64 cycles, whatever the independence
@@ -43,7 +46,7 @@
 // each column of the elimination costs one fp64 multiply and one fp64 fma per
 // entry a thread holds (1 for e <= 8, 4 for e <= 16), spread over warps on
 // different schedulers, and the only divisions are the e reciprocals of the
-// pivots, taken in parallel.
+// pivots (the e^2 entries of adj(Q) / det Q for e <= 2), taken in parallel.
 #pragma once
 
 #include <cfloat>

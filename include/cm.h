@@ -143,11 +143,13 @@ cm_status cm_draw_erasures(uint64_t seed, uint64_t counter, int32_t n, int32_t k
  * Yt_S = G_S Z with Z the uncoded block products.  One launch: every CTA
  * inverts G_S in fp64 in its own shared memory (the k-e unit rows of
  * surviving systematic workers are eliminated first, then Gauss-Jordan with
- * partial pivoting on the e x e block of the missing systematic columns, in
- * the registers of one warp for e <= 4, of four for e <= 16) and forms the
- * rows of G_S^-1 for the e missing systematic blocks, then applies them to
- * the k surviving results (double-float arithmetic, about 2^-44 relative per
- * term) while surviving systematic blocks pass through.  The launch is a
+ * partial pivoting on the e x e block Q of the missing systematic columns,
+ * in the registers of one warp for e <= 4, of four for e <= 16; adj(Q) /
+ * det Q for e <= 2) and applies the rows of G_S^-1 for the e missing
+ * systematic blocks to the k surviving results, as Q^-1 (Yt_par - P_sys
+ * Yt_sys) with the second factor formed while the inversion runs
+ * (double-float arithmetic, about 2^-44 relative per term); surviving
+ * systematic blocks pass through.  The launch is a
  * programmatic dependent of the kernel before it on `stream`: the eliminating
  * warps start from the kernel parameters at once and the others wait for the
  * earlier grids before reading Yt, so after cm_matvec on the same stream the
